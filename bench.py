@@ -1,0 +1,361 @@
+#!/usr/bin/env python
+"""GauS hot-path benchmark: fused loss + gradient + Adam iterations/s x B restarts.
+
+One step = `--inner` fused iterations (gaus_iterate: loss, gradient, Adam,
+multiplier update; Sec. 3.3, Alg. GauS) followed by one round + legalize
+(App. A) and one verify (Sec. 2.1) of all B restarts -- one outer period of
+Alg. GauS.  The default run (20 steps of 100 iterations) is the 2,000-iteration
+trajectory of the logic-network workload (V = 10,000, B = 64) from its seeded
+initial state.
+
+Prints one JSON line.  `--impl reference` times the fp64 CPU oracle on the same
+workload and metric (bounded sample per step).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+METRIC = "loss+grad+Adam iterations/s x B restarts (logic-network DAG, |V|=10k)"
+UNIT = "restart-iterations/s"
+FP32_LANES_PER_SM = 128
+SM_COUNT = 152
+SM_MAX_MHZ = 2070.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--inner", type=int, default=100, help="fused iterations per step")
+    ap.add_argument("--impl", default="gaus", choices=["gaus", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def workload(rank=0):
+    p = W.logic_network(1)
+    B = 64
+    mu, sg = W.init_state(p, B, seed=1 + rank)
+    return p, B, mu, sg
+
+
+def describe(p, B, iters):
+    return {"workload": f"{p.name}: AND/INV logic network, V={p.V}, E={p.E}, depth 120, "
+                        f"D={p.D}, 2 classes (AND limit 64, INV unlimited), unit latency, "
+                        f"Formulation A terms (Res LSE + ReLU, Com, Dep)",
+            "B": B, "V": p.V, "E": p.E, "D": p.D, "iterations_per_step": iters,
+            "init": "mu = ASAP + N(0, 2), sigma = 1.5 (seeded)", "tau": 1e-2, "rho": 1e-4, "lr": 1e-2,
+            "window_k": 6.0}
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            cmd = ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "200"]
+            if self.gpu_id is not None:
+                cmd += ["-i", str(self.gpu_id)]
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9:
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in self.rows if r[2].replace(".", "").isdigit()]
+        reasons = set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in self.rows:
+            for name, val in zip(names, r[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(self.rows)}
+
+
+# ----------------------------------------------------------------- algorithmic work
+def algorithmic_flops(torch, mu, sg, src, dst, k, D):
+    """FP32 work of one node/edge pass under the cost model of the design notes:
+    20 flop per CDF point and 8 flop per edge-bin, with the points of each
+    (node, restart) window of +-k sigma (bins = points + 1)."""
+    a = torch.clamp(torch.ceil(mu - k * sg - 0.5), 0, D - 1)
+    b = torch.clamp(torch.floor(mu + k * sg - 0.5), -1, D - 2)
+    bins = (b - a + 2).to(torch.float64)                  # (V, B)
+    n_pt = float(bins.sum())
+    # dependency edge: producer bins; communication: producer + consumer bins
+    n_eb = float((2.0 * bins[src] + bins[dst]).sum())
+    return 20.0 * n_pt + 8.0 * n_eb, n_pt, n_eb
+
+
+def gpu_arm(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2602_20427_gb300 as g
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    g.build()
+    p, B, mu0, sg0 = workload(rank)
+    hp = g.default_hparams(terms=p.terms)
+    ctx = g.Gaus(p, B, hp)
+    inner = args.inner
+    dmu0, dsg0 = torch.from_numpy(mu0).cuda(), torch.from_numpy(sg0).cuda()
+    st = ctx.new_state(dmu0, dsg0, hp.lambda0)
+    sched = torch.empty((p.V, B), dtype=torch.int32, device="cuda")
+    lstat = torch.empty(B, dtype=torch.int32, device="cuda")
+    rep = torch.empty(B * 200, dtype=torch.uint8, device="cuda")
+
+    def reset():
+        fresh = ctx.new_state(dmu0, dsg0, hp.lambda0)
+        for kk, v in fresh.items():
+            st[kk].copy_(v)
+
+    def step():
+        ctx.iterate(inner, st)
+        ctx.legalize(st["mu"], sched, lstat)
+        ctx.verify_raw(sched, rep)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    reset()
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    gpu_id = None
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(local).uuid)
+    except Exception:
+        gpu_id = None
+    sampler = ClockSampler(gpu_id) if rank == 0 else None
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.start()
+        time.sleep(0.5)
+    wall0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.fill_(k & 255)                     # L2 flush between steps (outside the events)
+        evs[k][0].record()
+        step()
+        evs[k][1].record()
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    clocks = sampler.stop() if sampler else None
+    ms = sum(a.elapsed_time(b) for a, b in evs)
+    if world > 1:
+        dist.barrier()
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    status_ok = bool(int(st["status"].abs().sum()) == 0)
+    units = args.steps * inner * B * world
+    value = units / (ms / 1e3)
+
+    # ---- kernel-level timing and algorithmic work along the same trajectory
+    reset()
+    src = torch.from_numpy(np.asarray(p.src, np.int64)).cuda()
+    dst = torch.from_numpy(np.asarray(p.dst, np.int64)).cuda()
+    k_ms = np.zeros(3)
+    flops_total, t_fwd_total, npt_total, neb_total = 0.0, 0.0, 0.0, 0.0
+    for k in range(args.steps):
+        f0, n0, e0 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
+        kms = np.array(ctx.profile_iterate(inner, st))
+        f1, n1, e1 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
+        k_ms += kms / args.steps
+        flops_total += inner * 0.5 * (f0 + f1)
+        npt_total += inner * 0.5 * (n0 + n1)
+        neb_total += inner * 0.5 * (e0 + e1)
+        t_fwd_total += inner * kms[0] * 1e-3
+    achieved = flops_total / t_fwd_total / 1e12
+    peak = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
+    traffic = None
+    prof = os.path.join(ROOT, "profiles", "k_fwd_traffic.json")
+    if os.path.exists(prof):
+        try:
+            traffic = json.load(open(prof)).get("bytes_per_launch")
+        except Exception:
+            traffic = None
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        reset()
+        h_mu = torch.from_numpy(mu0.copy()).pin_memory()
+        h_sg = torch.from_numpy(sg0.copy()).pin_memory()
+        h_sched = torch.empty((p.V, B), dtype=torch.int32).pin_memory()
+        h_rep = torch.empty(B * 200, dtype=torch.uint8).pin_memory()
+        h_loss = torch.empty(B, dtype=torch.float32).pin_memory()
+        eev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        torch.cuda.synchronize()
+        for k in range(args.steps):
+            flush.fill_(k & 255)
+            eev[k][0].record()
+            st["mu"].copy_(h_mu, non_blocking=True)
+            st["sigma"].copy_(h_sg, non_blocking=True)
+            step()
+            h_mu.copy_(st["mu"], non_blocking=True)
+            h_sg.copy_(st["sigma"], non_blocking=True)
+            h_sched.copy_(sched, non_blocking=True)
+            h_rep.copy_(rep, non_blocking=True)
+            h_loss.copy_(st["loss"], non_blocking=True)
+            eev[k][1].record()
+        torch.cuda.synchronize()
+        ems = sum(a.elapsed_time(b) for a, b in eev)
+        h2d = 2 * p.V * B * 4
+        d2h = 2 * p.V * B * 4 + p.V * B * 4 + B * 200 + B * 4
+        e2e = {"value": units / world * world / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(p, B, mu0, sg0, hp)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                "data": "synthetic (seeded logic-network DAG and initial means)",
+                "config": dict(describe(p, B, inner), l2="flushed between steps (256 MB write)",
+                               parallelism=f"restarts sharded, {world} replica(s)"),
+                "e2e": e2e, "gpu_launches": args.steps * (3 * inner + 2),
+                "clocks": clocks,
+                "roofline": {"bound": "alu", "kernel": "k_fwd (node + edge pass)", "achieved": achieved,
+                             "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
+                             "peak_note": "FP32: 152 SM x 128 lanes x 2 flop x 2070 MHz (max SM clock)",
+                             "cost_model": "20 flop per CDF point + 8 flop per edge-bin",
+                             "points_per_iter": npt_total / (args.steps * inner),
+                             "edge_bins_per_iter": neb_total / (args.steps * inner)},
+                "kernel_ms": {"k_fwd": k_ms[0], "k_finalize": k_ms[1], "k_update": k_ms[2]},
+                "status_ok": status_ok, "wall_s": wall,
+                "cpu_baseline": cpu}
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _oracle_iteration(op, ohp, mu, sg, lam, mom, step, lr):
+    import oracle
+    loss, terms, gm, gs = oracle.loss_grad(op, ohp, mu, sg, lam)
+    for th, gg, m1, v1 in ((mu, gm, mom[0], mom[1]), (sg, gs, mom[2], mom[3])):
+        flat_t, flat_m, flat_v = th.reshape(-1), m1.reshape(-1), v1.reshape(-1)
+        oracle.adam(flat_t, np.ascontiguousarray(gg.reshape(-1)), flat_m, flat_v, step, lr)
+    np.maximum(sg, 0.05, out=sg)
+    lam[:, 0] += 1e-4 * terms[:, oracle.T_VDEP]
+    lam[:, 1] += 1e-4 * terms[:, oracle.T_VRES]
+
+
+def cpu_baseline(p, B, mu0, sg0, hp, budget_s=12.0, restarts=None):
+    """The fp64 oracle, as it stands, on a bounded sample of the same workload."""
+    import oracle
+    cores = os.cpu_count() or 1
+    os.environ.setdefault("OMP_NUM_THREADS", str(cores))
+    r = restarts or min(B, cores)
+    op = oracle.OracleProblem(p)
+    ohp = oracle.hparams(tau=hp.tau, rho=hp.rho, alpha=hp.alpha, w_res=hp.w_res, w_mem=hp.w_mem, terms=p.terms)
+    mu = mu0[:, :r].astype(np.float64).copy()
+    sg = sg0[:, :r].astype(np.float64).copy()
+    lam = np.full((r, 3), 1e-6)
+    mom = [np.zeros_like(mu) for _ in range(4)]
+    t0 = time.perf_counter()
+    it = 0
+    while True:
+        it += 1
+        _oracle_iteration(op, ohp, mu, sg, lam, mom, it, hp.lr)
+        el = time.perf_counter() - t0
+        if el >= budget_s or it >= 5:
+            break
+    return {"value": r * it / el, "unit": UNIT, "cores": int(os.environ.get("OMP_NUM_THREADS", cores)),
+            "kind": "oracle", "sample": f"{it} iteration(s) of {r} restarts of {p.name}, fp64, unwindowed, "
+                                         f"{el:.1f} s"}
+
+
+def reference_arm(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    p, B, mu0, sg0 = workload(0)
+
+    class H:  # the same hyperparameters as the GPU arm
+        tau, rho, alpha, w_res, w_mem, lr = 1e-2, 1e-4, 1.0, 1.0, 1.0, 1e-2
+
+    cores = os.cpu_count() or 1
+    os.environ.setdefault("OMP_NUM_THREADS", str(cores))
+    r = min(B, cores)
+    op = oracle.OracleProblem(p)
+    ohp = oracle.hparams(tau=H.tau, rho=H.rho, alpha=H.alpha, w_res=H.w_res, w_mem=H.w_mem, terms=p.terms)
+    mu = mu0[:, :r].astype(np.float64).copy()
+    sg = sg0[:, :r].astype(np.float64).copy()
+    lam = np.full((r, 3), 1e-6)
+    mom = [np.zeros_like(mu) for _ in range(4)]
+    for w in range(args.warmup):
+        _oracle_iteration(op, ohp, mu, sg, lam, mom, w + 1, H.lr)
+    t0 = time.perf_counter()
+    for k in range(args.steps):
+        _oracle_iteration(op, ohp, mu, sg, lam, mom, args.warmup + k + 1, H.lr)
+    el = time.perf_counter() - t0
+    value = args.steps * r / el
+    sample = f"1 iteration of {r} of the {B} restarts per step, fp64 oracle, unwindowed"
+    print(json.dumps({"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1,
+                      "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+                      "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                      "data": "synthetic (seeded logic-network DAG and initial means)",
+                      "config": dict(describe(p, B, 1), sample=sample),
+                      "cpu_baseline": {"value": value, "unit": UNIT, "cores": int(os.environ["OMP_NUM_THREADS"]),
+                                       "kind": "oracle", "sample": sample},
+                      "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
+
+
+if __name__ == "__main__":
+    a = parse()
+    if a.impl == "reference":
+        reference_arm(a)
+    else:
+        gpu_arm(a)

@@ -1,0 +1,214 @@
+/*
+ * gaus.h -- C ABI of the GB300 (sm_103a) GauS hot path.
+ *
+ * GauS (arXiv 2602.20427) relaxes each operator's start step to a Gaussian
+ * X_v ~ N(mu_v, sigma_v^2) (Sec. 3.1), turns objectives and constraint
+ * violations into expectations over the rounded steps (Sec. 3.2, App. B) and
+ * minimises them with an augmented Lagrangian and Adam (Sec. 3.3).  This
+ * library evaluates that loss and its gradient, applies Adam and the
+ * multiplier update, rounds and legalizes the means (App. A), and verifies
+ * schedules (Sec. 2.1), for B independent restarts at once, on one GPU.
+ *
+ * Conventions (every entry point):
+ *  - Per-restart node arrays are (V, B) row-major fp32/int32 device arrays:
+ *    element [v * B + b] belongs to node v (the caller's id) and restart b.
+ *    Per-restart vectors are (B, K) row-major.
+ *  - The caller owns every device buffer it passes; the library owns only the
+ *    context, its device copy of the graph and its scratch memory.
+ *  - Every call is asynchronous on the context's stream.  Argument errors are
+ *    returned at once and enqueue nothing.  Data-dependent conditions (a
+ *    non-finite mu or sigma, Alg. 2 not settling) are written to per-restart
+ *    device status words and never abort the call.
+ *  - Entry points are not thread-safe on one context.
+ */
+#ifndef GAUS_H
+#define GAUS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct gaus_ctx gaus_ctx;
+
+typedef enum {
+  GAUS_OK = 0,
+  GAUS_EINVAL = 1,      /* bad argument, graph arrays disagree, size out of range */
+  GAUS_ECYCLE = 2,      /* the dependency graph has a cycle                        */
+  GAUS_EHORIZON = 3,    /* critical path longer than the horizon D                 */
+  GAUS_ENOMEM = 4,      /* device or host allocation failed                        */
+  GAUS_ECUDA = 5,       /* a CUDA runtime call failed (see gaus_last_error)        */
+  GAUS_ENONFINITE = 6,  /* per restart: a mu or sigma was NaN/Inf or sigma < 1e-30 */
+  GAUS_ENOTCONV = 7     /* per restart: Alg. 2 did not settle within |V| sweeps    */
+} gaus_status;
+
+/* Terms of the loss (bit mask).  Objectives are weighted, constraints enter the
+ * augmented Lagrangian of Sec. 3.3. */
+#define GAUS_DEP      1u  /* constraint: expected dependency violations, Eq. dep with latency    */
+#define GAUS_COM      2u  /* objective:  alpha * expected communication, App. B.1                */
+#define GAUS_RES_OBJ  4u  /* objective:  w_res * sum_c LSE_tau(expected usage of class c), App. B.2 */
+#define GAUS_RES_VIOL 8u  /* constraint: sum_c sum_t ReLU(usage - R_c), Eq. relu                 */
+#define GAUS_REG_OBJ 16u  /* objective:  w_mem * LSE_tau(expected live storage), Eq. active/max  */
+#define GAUS_REC     32u  /* constraint: expected recurrence violations, App. B.3 (II > 0)       */
+
+/* Constraint slots (lambda, multiplier update) and per-restart term values. */
+#define GAUS_K_DEP 0
+#define GAUS_K_RES 1
+#define GAUS_K_REC 2
+#define GAUS_K     3
+#define GAUS_T_RES  0   /* sum_c LSE_tau(U_c)             */
+#define GAUS_T_COM  1   /* expected communication         */
+#define GAUS_T_REG  2   /* LSE_tau(Reg)                   */
+#define GAUS_T_VDEP 3   /* expected dependency violations */
+#define GAUS_T_VRES 4   /* sum of ReLU resource excess    */
+#define GAUS_T_VREC 5   /* expected recurrence violations */
+#define GAUS_NT     6
+
+/* Scheduling problem (Sec. 2.1).  All pointers are HOST pointers, read during
+ * gaus_create and not kept.  Node ids are 0..V-1. */
+typedef struct {
+  int32_t V, E;
+  const int32_t *succ_ptr, *succ_idx;  /* CSR of edges u -> v: (V+1), (E)                    */
+  const int32_t *pred_ptr, *pred_idx;  /* CSC of the same edges: (V+1), (E); must agree      */
+  const int32_t *latency;              /* Lat(v) >= 0 (0 = chaining, Sec. 2.1), (V)          */
+  const int32_t *res_class;            /* class of v in 0..C-1, (V)                          */
+  int32_t C;                           /* number of resource classes, 1..16                  */
+  const float *limit;                  /* R_c, (C); INFINITY = unlimited                     */
+  const int32_t *demand;               /* r_v >= 0, (V); NULL = all 1                        */
+  const int32_t *bits;                 /* b_v >= 0 storage units of v's output, (V); NULL = 1 */
+  int32_t n_back;                      /* loop-carried edges j -> i with distance k (Sec. 2.1 Rec) */
+  const int32_t *back_src;             /* j, (n_back)                                         */
+  const int32_t *back_dst;             /* i, (n_back)                                         */
+  const int32_t *back_dist;            /* k >= 1, (n_back)                                    */
+  int32_t D;                           /* horizon: start steps 0..D-1 (Sec. 3.2)              */
+  int32_t II;                          /* initiation interval; 0 = regular scheduling         */
+  int32_t B;                           /* restarts per call, >= 1                             */
+} gaus_problem;
+
+typedef struct {
+  float tau;        /* LogSumExp temperature (Eq. max); paper 1e-2                     */
+  float rho;        /* ALM penalty (Sec. 3.3); paper 1e-4                               */
+  float lambda0;    /* initial multiplier the caller should use; paper 1e-6             */
+  float alpha;      /* weight of the communication objective (Formulation A)           */
+  float w_res;      /* weight of the usage LSE objective                                */
+  float w_mem;      /* weight of the storage LSE objective                              */
+  float lr;         /* Adam learning rate; paper 1e-2                                   */
+  float beta1, beta2, eps;   /* Adam; 0.9, 0.999, 1e-8                                  */
+  float window_k;   /* bins further than window_k * sigma from mu carry no mass; 6     */
+  float sigma_min;  /* sigma is clamped to >= sigma_min after each Adam step; 0.05     */
+  uint32_t terms;   /* GAUS_* bit mask                                                  */
+} gaus_hparams;
+
+/* Discrete verdict on one schedule (Sec. 2.1; App. B.1 for L_com). */
+typedef struct {
+  int64_t n_dep_viol;   /* edges u -> v with s_v < s_u + Lat(u)                       */
+  int64_t n_lat_viol;   /* nodes with s_v < 0 or s_v + Lat(v) > D                     */
+  int64_t n_rec_viol;   /* back edges with s_i + k II < s_j + Lat(j)                  */
+  int64_t n_res_viol;   /* (class, step) cells whose usage exceeds R_c (folded if II)  */
+  int64_t L_res;        /* sum over classes of peak usage (folded if II > 0)          */
+  int64_t L_com;        /* sum over edges of s_v - s_u                                */
+  int64_t L_mem;        /* max over d in [0, D) of Mem(d), leaves live until D         */
+  int64_t L_mmem;       /* max over t in [0, II) of the folded Mem (= L_mem if II = 0) */
+  int64_t peak[16];     /* per-class peak usage                                       */
+  int32_t feasible;     /* no Dep, Lat or Rec violation                               */
+  int32_t res_ok;       /* no resource cell over its limit                            */
+} gaus_report;
+
+/* State of gaus_iterate: DEVICE pointers owned by the caller. */
+typedef struct {
+  float *mu, *sigma;                   /* (V, B), updated in place                   */
+  float *m_mu, *v_mu, *m_sigma, *v_sigma; /* Adam moments (V, B), zero-initialised by the caller */
+  float *lambda;                       /* (B, GAUS_K) multipliers, updated in place   */
+  int32_t *step;                       /* (B) Adam step count, incremented each iteration */
+  float *loss;                         /* (B) out: loss of the last iteration        */
+  float *terms;                        /* (B, GAUS_NT) out: term values of the last iteration */
+  int32_t *status;                     /* (B) out: GAUS_OK or GAUS_ENONFINITE         */
+} gaus_state;
+
+/* Paper defaults (Sec. 3.3, App. C.1): tau 1e-2, rho 1e-4, lambda0 1e-6, lr 1e-2;
+ * Adam betas (0.9, 0.999), eps 1e-8; alpha = w_res = w_mem = 1; window 6 sigma;
+ * sigma_min 0.05; terms = DEP | COM | RES_OBJ.  Returns GAUS_EINVAL on NULL. */
+gaus_status gaus_default_hparams(gaus_hparams *hp);
+
+/* Validate the problem, sort it topologically (Kahn), compute ASAP/ALAP and the
+ * critical path (App. A, Alg. 1 input), build the class-sorted node order and
+ * upload the graph to the device on `cuda_stream` (a cudaStream_t; NULL = the
+ * legacy default stream).  Errors: EINVAL (arrays missing or inconsistent,
+ * CSR/CSC disagree, duplicate edge, ids out of range, C outside 1..16, D < 1,
+ * II < 0, B < 1, sizes beyond the library's limits), ECYCLE, EHORIZON, ENOMEM,
+ * ECUDA.  On success *out owns device memory until gaus_destroy. */
+gaus_status gaus_create(const gaus_problem *prob, const gaus_hparams *hp, void *cuda_stream,
+                        gaus_ctx **out);
+
+/* Replace the hyperparameters (same validation as gaus_create). */
+gaus_status gaus_set_hparams(gaus_ctx *ctx, const gaus_hparams *hp);
+
+/* Copy ASAP, ALAP (host int32 arrays of V, caller ids; either may be NULL) and
+ * the critical path length (may be NULL) computed at creation. */
+gaus_status gaus_bounds(const gaus_ctx *ctx, int32_t *asap, int32_t *alap, int32_t *cp);
+
+/* Loss of Sec. 3.3 and its gradient for B restarts:
+ *   L_b = w_res sum_c LSE_tau(U_c) + alpha L_com + w_mem LSE_tau(Reg)
+ *         + sum_{k active} (lambda[b,k] V_k + rho/2 V_k^2),
+ * with U_c(t) = sum_{cls(v)=c} r_v P_v^t (folded mod II when II > 0) and the
+ * bin masses P of Eq. round, truncated to +-window_k sigma.
+ *   mu, sigma   (V, B) device, read only.
+ *   lambda      (B, GAUS_K) device, read only.
+ *   grad_mu, grad_sigma (V, B) device, written.
+ *   loss (B), terms (B, GAUS_NT), status (B) device, written; status may be NULL.
+ * Non-finite mu/sigma or sigma < 1e-30 in restart b sets status[b] = ENONFINITE;
+ * that restart's outputs are then unspecified. */
+gaus_status gaus_loss_grad(gaus_ctx *ctx, const float *mu, const float *sigma,
+                           const float *lambda, float *grad_mu, float *grad_sigma,
+                           float *loss, float *terms, int32_t *status);
+
+/* One Adam step (torch.optim.Adam semantics, no weight decay) on mu and sigma,
+ * then sigma <- max(sigma, sigma_min) and, for every active constraint k,
+ * lambda[b,k] += rho * terms[b, V_k] (Sec. 3.3 multiplier update).
+ *   step >= 1 is the 1-based Adam step shared by all restarts.
+ * All pointers are device pointers of the shapes above. */
+gaus_status gaus_adam_step(gaus_ctx *ctx, float *mu, float *sigma, const float *grad_mu,
+                           const float *grad_sigma, float *m_mu, float *v_mu, float *m_sigma,
+                           float *v_sigma, float *lambda, const float *terms, int32_t step);
+
+/* n_iters fused iterations of Alg. GauS's inner loop (loss, gradient, Adam,
+ * multiplier update), each a replay of one captured CUDA graph.  Equivalent to
+ * gaus_loss_grad + gaus_adam_step with step = st->step[b] + 1 per iteration.
+ * Gradients are not materialised.  EINVAL on NULL state pointers or n_iters < 0. */
+gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st);
+
+/* Kernel-level timing of gaus_iterate: runs n_iters iterations exactly as
+ * gaus_iterate does, but launched one kernel at a time with a CUDA event
+ * between kernels, and adds the mean duration in milliseconds of the three
+ * kernels of an iteration to ms_out[0..2] (host array: node/edge pass,
+ * per-restart finalize, gradient + Adam).  Synchronises the context's stream.
+ * Library feature for measurement; not on the hot path. */
+gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st, double *ms_out);
+
+/* Round every mean to s = floor(mu + 1/2) (Sec. 3.3 Sampling; exact for every
+ * fp32 value) and legalize it: Alg. 1 (clamp to [ASAP, ALAP], then a forward push
+ * in topological order with +Lat(u)) when II = 0, Alg. 2 (fixed-point relaxation
+ * of forward and back edges, at most |V| sweeps) when II > 0.
+ *   mu (V, B) device; sched (V, B) int32 device, written; status (B) device,
+ *   written with OK, ENONFINITE or ENOTCONV (sched then unspecified). */
+gaus_status gaus_legalize(gaus_ctx *ctx, const float *mu, int32_t *sched, int32_t *status);
+
+/* Round only (no legalization): sched = floor(mu + 1/2). */
+gaus_status gaus_round(gaus_ctx *ctx, const float *mu, int32_t *sched);
+
+/* Verify B schedules (Sec. 2.1): sched (V, B) int32 device; rep (B) device array
+ * of gaus_report, written.  Integer arithmetic only. */
+gaus_status gaus_verify(gaus_ctx *ctx, const int32_t *sched, gaus_report *rep);
+
+/* Message of the last error on this context ("" if none), or with ctx = NULL the
+ * message of this thread's last failed gaus_create.  Valid until the next call. */
+const char *gaus_last_error(const gaus_ctx *ctx);
+
+/* Release the context and its device memory (synchronises its stream). */
+void gaus_destroy(gaus_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,482 @@
+// gaus_api.cu -- C ABI of the GauS hot path (include/gaus.h): context setup,
+// launches, the captured iteration graph, and the integer entry points.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "gaus.h"
+#include "gaus_int.cuh"
+#include "gaus_internal.h"
+#include "gaus_kernels.cuh"
+
+using namespace gaus;
+
+namespace {
+
+thread_local std::string g_create_error;
+constexpr size_t kMaxSmem = 227 * 1024;
+
+gaus_status cuda_fail(gaus_ctx *ctx, cudaError_t e, const char *what) {
+  if (ctx) ctx->err = std::string(what) + ": " + cudaGetErrorString(e);
+  return e == cudaErrorMemoryAllocation ? GAUS_ENOMEM : GAUS_ECUDA;
+}
+
+#define CK(call, what)                                   \
+  do {                                                   \
+    cudaError_t e_ = (call);                             \
+    if (e_ != cudaSuccess) return cuda_fail(ctx, e_, what); \
+  } while (0)
+
+template <typename T>
+gaus_status upload(gaus_ctx *ctx, T **dst, const std::vector<T> &src) {
+  size_t bytes = std::max<size_t>(sizeof(T), src.size() * sizeof(T));
+  CK(cudaMalloc((void **)dst, bytes), "cudaMalloc");
+  ctx->allocs.push_back(*dst);
+  if (!src.empty()) CK(cudaMemcpy(*dst, src.data(), src.size() * sizeof(T), cudaMemcpyHostToDevice), "cudaMemcpy");
+  return GAUS_OK;
+}
+
+template <typename T>
+gaus_status scratch(gaus_ctx *ctx, T **dst, size_t count) {
+  CK(cudaMalloc((void **)dst, std::max<size_t>(1, count) * sizeof(T)), "cudaMalloc scratch");
+  ctx->allocs.push_back(*dst);
+  CK(cudaMemset(*dst, 0, std::max<size_t>(1, count) * sizeof(T)), "cudaMemset");
+  return GAUS_OK;
+}
+
+#define TRY(x)                           \
+  do {                                   \
+    gaus_status s_ = (x);                \
+    if (s_ != GAUS_OK) return s_;        \
+  } while (0)
+
+IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
+  const Plan &P = ctx->plan;
+  IterArgs A;
+  A.mu = mu; A.sg = sg;
+  A.V = P.V; A.B = P.B; A.D = P.D; A.II = P.II; A.Dh = P.Dh; A.C = P.C; A.RB = ctx->RB; A.G = ctx->G;
+  A.k_win = ctx->hp.window_k; A.alpha = ctx->hp.alpha;
+  A.perm = ctx->d_perm; A.w = ctx->d_w; A.lat = ctx->d_lat;
+  A.in_ptr = ctx->d_in_ptr; A.in_src = ctx->d_in_src; A.in_lat = ctx->d_in_lat;
+  A.out_ptr = ctx->d_out_ptr; A.out_dst = ctx->d_out_dst;
+  A.bin_ptr = ctx->d_bin_ptr; A.bin_src = ctx->d_bin_src; A.bin_shift = ctx->d_bin_shift;
+  A.bout_ptr = ctx->d_bout_ptr; A.bout_dst = ctx->d_bout_dst; A.bout_shift = ctx->d_bout_shift;
+  A.seg = ctx->d_seg; A.hpart = ctx->d_hpart; A.hspan = ctx->d_hspan; A.fwd = ctx->d_fwd;
+  A.gpart = ctx->d_gpart; A.nonfinite = ctx->d_nonfinite;
+  return A;
+}
+
+using FwdKernel = void (*)(const IterArgs);
+
+FwdKernel pick_fwd(unsigned terms, int II) {
+  const bool dep = terms & GAUS_DEP, com = terms & GAUS_COM, rec = (terms & GAUS_REC) && II > 0;
+  if (dep && com && rec) return k_fwd<true, true, true>;
+  if (dep && com) return k_fwd<true, true, false>;
+  if (dep && rec) return k_fwd<true, false, true>;
+  if (dep) return k_fwd<true, false, false>;
+  if (com && rec) return k_fwd<false, true, true>;
+  if (com) return k_fwd<false, true, false>;
+  if (rec) return k_fwd<false, false, true>;
+  return k_fwd<false, false, false>;
+}
+
+// Enqueue loss + gradient (adam == false: gradient written to grad_*), or the
+// fused iteration (adam == true: Adam on the state, lambda and step updated).
+gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, const float *sg,
+                              float *lambda, bool adam, float *grad_mu, float *grad_sg, float *loss,
+                              float *terms, int32_t *status, const gaus_state *S,
+                              cudaEvent_t *ev = nullptr) {
+  if (ev) CK(cudaEventRecord(ev[0], st), "event");
+  const Plan &P = ctx->plan;
+  const unsigned on = ctx->hp.terms;
+  IterArgs A = iter_args(ctx, mu, sg);
+  FwdKernel kf = pick_fwd(on, P.II);
+  kf<<<ctx->nblk, kThreads, ctx->smem_fwd, st>>>(A);
+  CK(cudaGetLastError(), "k_fwd launch");
+  if (ev) CK(cudaEventRecord(ev[1], st), "event");
+
+  FinArgs F;
+  F.B = P.B; F.C = P.C; F.Dh = P.Dh; F.RB = ctx->RB; F.G = ctx->G;
+  F.terms = on; F.tau = ctx->hp.tau; F.rho = ctx->hp.rho; F.alpha = ctx->hp.alpha;
+  F.w_res = ctx->hp.w_res; F.w_mem = ctx->hp.w_mem;
+  F.cls_seg_ptr = ctx->d_cls_seg_ptr; F.limit = ctx->d_limit;
+  F.hpart = ctx->d_hpart; F.hspan = ctx->d_hspan; F.fwd = ctx->d_fwd;
+  F.lambda = lambda; F.update_lambda = adam ? 1 : 0; F.step = adam ? S->step : nullptr;
+  F.H = ctx->d_H; F.coef = ctx->d_coef; F.loss = loss; F.terms_out = terms;
+  F.status = status; F.nonfinite = ctx->d_nonfinite;
+  k_finalize<<<P.B, 256, ctx->smem_fin, st>>>(F);
+  CK(cudaGetLastError(), "k_finalize launch");
+  if (ev) CK(cudaEventRecord(ev[2], st), "event");
+
+  UpdArgs U;
+  U.mu = const_cast<float *>(mu); U.sg = const_cast<float *>(sg);
+  U.V = P.V; U.B = P.B; U.D = P.D; U.II = P.II; U.Dh = P.Dh; U.C = P.C; U.RB = ctx->RB; U.G = ctx->G;
+  U.k_win = ctx->hp.window_k; U.perm = ctx->d_perm; U.w = ctx->d_w; U.seg = ctx->d_seg;
+  U.gpart = ctx->d_gpart; U.H = ctx->d_H; U.coef = ctx->d_coef;
+  U.grad_mu = grad_mu; U.grad_sg = grad_sg;
+  U.m_mu = adam ? S->m_mu : nullptr; U.v_mu = adam ? S->v_mu : nullptr;
+  U.m_sg = adam ? S->m_sigma : nullptr; U.v_sg = adam ? S->v_sigma : nullptr;
+  U.step_dev = adam ? S->step : nullptr;
+  U.lr = ctx->hp.lr; U.beta1 = ctx->hp.beta1; U.beta2 = ctx->hp.beta2; U.eps = ctx->hp.eps;
+  U.sigma_min = ctx->hp.sigma_min;
+  const bool hist = on & (GAUS_RES_OBJ | GAUS_RES_VIOL);
+  if (adam) {
+    if (hist) k_update<true, true><<<ctx->nblk, kThreads, ctx->smem_upd, st>>>(U);
+    else k_update<true, false><<<ctx->nblk, kThreads, 0, st>>>(U);
+  } else {
+    if (hist) k_update<false, true><<<ctx->nblk, kThreads, ctx->smem_upd, st>>>(U);
+    else k_update<false, false><<<ctx->nblk, kThreads, 0, st>>>(U);
+  }
+  CK(cudaGetLastError(), "k_update launch");
+  if (ev) CK(cudaEventRecord(ev[3], st), "event");
+  return GAUS_OK;
+}
+
+gaus_status set_smem_attrs(gaus_ctx *ctx) {
+  const void *fwd[] = {(const void *)k_fwd<true, true, true>, (const void *)k_fwd<true, true, false>,
+                       (const void *)k_fwd<true, false, true>, (const void *)k_fwd<true, false, false>,
+                       (const void *)k_fwd<false, true, true>, (const void *)k_fwd<false, true, false>,
+                       (const void *)k_fwd<false, false, true>, (const void *)k_fwd<false, false, false>};
+  for (const void *f : fwd)
+    CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fwd), "smem attr fwd");
+  const void *upd[] = {(const void *)k_update<true, true>, (const void *)k_update<false, true>};
+  for (const void *f : upd)
+    CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_upd), "smem attr upd");
+  CK(cudaFuncSetAttribute((const void *)k_finalize, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fin),
+     "smem attr fin");
+  CK(cudaFuncSetAttribute((const void *)k_verify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_ver),
+     "smem attr ver");
+  return GAUS_OK;
+}
+
+gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
+  // Validate and plan on the host first: argument and graph errors never touch CUDA.
+  int dev = 0, nsm = 152;
+  const bool have_dev = cudaGetDevice(&dev) == cudaSuccess &&
+                        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess;
+  std::string err;
+  gaus_status st = plan_problem(prob, 4 * nsm, &ctx->plan, &err);
+  if (st != GAUS_OK) { ctx->err = err; return st; }
+  Plan &P = ctx->plan;
+  if ((ctx->hp.terms & GAUS_REC) && P.II <= 0) { ctx->err = "GAUS_REC needs II > 0"; return GAUS_EINVAL; }
+  if (ctx->hp.terms & GAUS_REG_OBJ) { ctx->err = "GAUS_REG_OBJ is not available in this build"; return GAUS_EINVAL; }
+  if (!have_dev) {
+    cudaGetLastError();
+    ctx->err = "no CUDA device";
+    return GAUS_ECUDA;
+  }
+  ctx->RB = 1;
+  while (ctx->RB < P.B && ctx->RB < 32) ctx->RB <<= 1;
+  ctx->G = (P.B + ctx->RB - 1) / ctx->RB;
+  ctx->nblk = P.nseg * ctx->G;
+  ctx->smem_fwd = (size_t)ctx->RB * P.Dh * sizeof(long long) + 3 * (size_t)kCache * kThreads * sizeof(float);
+  ctx->smem_upd = (size_t)ctx->RB * P.Dh * sizeof(float);
+  ctx->smem_fin = (size_t)P.C * P.Dh * sizeof(double);
+  ctx->smem_ver = ((size_t)P.C * P.Dh + (P.D + 1) + P.Dh) * sizeof(long long);
+  const size_t static_fwd = 3 * kThreads * sizeof(double) + 64;
+  if (ctx->smem_fwd + static_fwd > kMaxSmem || ctx->smem_upd > kMaxSmem || ctx->smem_fin > kMaxSmem ||
+      ctx->smem_ver > kMaxSmem) {
+    ctx->err = "histogram of this horizon/II does not fit in shared memory";
+    return GAUS_EINVAL;
+  }
+  TRY(set_smem_attrs(ctx));
+
+  TRY(upload(ctx, &ctx->d_perm, P.perm));
+  TRY(upload(ctx, &ctx->d_w, P.w));
+  TRY(upload(ctx, &ctx->d_bits, P.bits));
+  TRY(upload(ctx, &ctx->d_limit, P.limit));
+  TRY(upload(ctx, &ctx->d_lat, P.lat));
+  TRY(upload(ctx, &ctx->d_cls, P.cls));
+  TRY(upload(ctx, &ctx->d_in_ptr, P.in_ptr));
+  TRY(upload(ctx, &ctx->d_in_src, P.in_src));
+  TRY(upload(ctx, &ctx->d_in_lat, P.in_lat));
+  TRY(upload(ctx, &ctx->d_out_ptr, P.out_ptr));
+  TRY(upload(ctx, &ctx->d_out_dst, P.out_dst));
+  TRY(upload(ctx, &ctx->d_bin_ptr, P.bin_ptr));
+  TRY(upload(ctx, &ctx->d_bin_src, P.bin_src));
+  TRY(upload(ctx, &ctx->d_bin_shift, P.bin_shift));
+  TRY(upload(ctx, &ctx->d_bout_ptr, P.bout_ptr));
+  TRY(upload(ctx, &ctx->d_bout_dst, P.bout_dst));
+  TRY(upload(ctx, &ctx->d_bout_shift, P.bout_shift));
+  TRY(upload(ctx, &ctx->d_seg, P.seg));
+  TRY(upload(ctx, &ctx->d_cls_seg_ptr, P.cls_seg_ptr));
+  TRY(upload(ctx, &ctx->d_lvl_ptr, P.lvl_ptr));
+  TRY(upload(ctx, &ctx->d_lvl_nodes, P.lvl_nodes));
+  TRY(upload(ctx, &ctx->d_cpred_ptr, P.cpred_ptr));
+  TRY(upload(ctx, &ctx->d_cpred_src, P.cpred_src));
+  TRY(upload(ctx, &ctx->d_csucc_ptr, P.csucc_ptr));
+  TRY(upload(ctx, &ctx->d_csucc_dst, P.csucc_dst));
+  TRY(upload(ctx, &ctx->d_cback_ptr, P.cback_ptr));
+  TRY(upload(ctx, &ctx->d_cback_src, P.cback_src));
+  TRY(upload(ctx, &ctx->d_cback_shift, P.cback_shift));
+  TRY(upload(ctx, &ctx->d_c_lat, P.c_lat));
+  TRY(upload(ctx, &ctx->d_c_cls, P.c_cls));
+  TRY(upload(ctx, &ctx->d_c_dem, P.c_dem));
+  TRY(upload(ctx, &ctx->d_c_bits, P.c_bits));
+  TRY(upload(ctx, &ctx->d_e_src, P.e_src));
+  TRY(upload(ctx, &ctx->d_e_dst, P.e_dst));
+  TRY(upload(ctx, &ctx->d_b_src, P.b_src));
+  TRY(upload(ctx, &ctx->d_b_dst, P.b_dst));
+  TRY(upload(ctx, &ctx->d_b_dist, P.b_dist));
+  TRY(upload(ctx, &ctx->d_asap, P.asap));
+  TRY(upload(ctx, &ctx->d_alap, P.alap));
+
+  const size_t VB = (size_t)P.V * P.B;
+  TRY(scratch(ctx, &ctx->d_hpart, (size_t)ctx->nblk * ctx->RB * P.Dh));
+  TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
+  TRY(scratch(ctx, &ctx->d_fwd, (size_t)ctx->nblk * ctx->RB * 3));
+  TRY(scratch(ctx, &ctx->d_gpart, 6 * VB));
+  TRY(scratch(ctx, &ctx->d_H, (size_t)P.B * P.C * P.Dh));
+  TRY(scratch(ctx, &ctx->d_coef, (size_t)P.B * 4));
+  TRY(scratch(ctx, &ctx->d_nonfinite, (size_t)P.B));
+  TRY(scratch(ctx, &ctx->d_status_tmp, (size_t)P.B));
+  TRY(scratch(ctx, &ctx->d_loss_tmp, (size_t)P.B));
+  TRY(scratch(ctx, &ctx->d_terms_tmp, (size_t)P.B * GAUS_NT));
+  CK(cudaDeviceSynchronize(), "setup sync");
+  return GAUS_OK;
+}
+
+uint64_t state_hash(const gaus_state *s) {
+  const void *p[] = {s->mu, s->sigma, s->m_mu, s->v_mu, s->m_sigma, s->v_sigma,
+                     s->lambda, s->step, s->loss, s->terms, s->status};
+  uint64_t h = 1469598103934665603ull;
+  for (const void *x : p) {
+    h ^= (uint64_t)(uintptr_t)x;
+    h *= 1099511628211ull;
+  }
+  return h;
+}
+
+void drop_graph(gaus_ctx *ctx) {
+  if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
+  ctx->gexec = nullptr;
+  ctx->ghash = 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+gaus_status gaus_default_hparams(gaus_hparams *hp) {
+  if (!hp) return GAUS_EINVAL;
+  hp->tau = 1e-2f;
+  hp->rho = 1e-4f;
+  hp->lambda0 = 1e-6f;
+  hp->alpha = 1.0f;
+  hp->w_res = 1.0f;
+  hp->w_mem = 1.0f;
+  hp->lr = 1e-2f;
+  hp->beta1 = 0.9f;
+  hp->beta2 = 0.999f;
+  hp->eps = 1e-8f;
+  hp->window_k = 6.0f;
+  hp->sigma_min = 0.05f;
+  hp->terms = GAUS_DEP | GAUS_COM | GAUS_RES_OBJ;
+  return GAUS_OK;
+}
+
+gaus_status gaus_create(const gaus_problem *prob, const gaus_hparams *hp, void *cuda_stream, gaus_ctx **out) {
+  if (!out) return GAUS_EINVAL;
+  *out = nullptr;
+  std::string err;
+  gaus_status st = check_hparams(hp, &err);
+  if (st != GAUS_OK) {
+    g_create_error = err;
+    return st;
+  }
+  gaus_ctx *ctx = new (std::nothrow) gaus_ctx();
+  if (!ctx) return GAUS_ENOMEM;
+  ctx->hp = *hp;
+  ctx->stream = (cudaStream_t)cuda_stream;
+  st = build_ctx(ctx, prob);
+  if (st != GAUS_OK) {
+    g_create_error = ctx->err;
+    gaus_destroy(ctx);
+    return st;
+  }
+  *out = ctx;
+  return GAUS_OK;
+}
+
+gaus_status gaus_set_hparams(gaus_ctx *ctx, const gaus_hparams *hp) {
+  if (!ctx) return GAUS_EINVAL;
+  gaus_status st = check_hparams(hp, &ctx->err);
+  if (st != GAUS_OK) return st;
+  if ((hp->terms & GAUS_REC) && ctx->plan.II <= 0) { ctx->err = "GAUS_REC needs II > 0"; return GAUS_EINVAL; }
+  if (hp->terms & GAUS_REG_OBJ) { ctx->err = "GAUS_REG_OBJ is not available in this build"; return GAUS_EINVAL; }
+  ctx->hp = *hp;
+  drop_graph(ctx);
+  return GAUS_OK;
+}
+
+gaus_status gaus_bounds(const gaus_ctx *ctx, int32_t *asap, int32_t *alap, int32_t *cp) {
+  if (!ctx) return GAUS_EINVAL;
+  const Plan &P = ctx->plan;
+  if (asap) std::memcpy(asap, P.asap.data(), sizeof(int32_t) * P.V);
+  if (alap) std::memcpy(alap, P.alap.data(), sizeof(int32_t) * P.V);
+  if (cp) *cp = P.cp;
+  return GAUS_OK;
+}
+
+gaus_status gaus_loss_grad(gaus_ctx *ctx, const float *mu, const float *sigma, const float *lambda,
+                           float *grad_mu, float *grad_sigma, float *loss, float *terms, int32_t *status) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!mu || !sigma || !lambda || !grad_mu || !grad_sigma || !loss || !terms) {
+    ctx->err = "gaus_loss_grad: NULL pointer";
+    return GAUS_EINVAL;
+  }
+  return enqueue_iteration(ctx, ctx->stream, mu, sigma, const_cast<float *>(lambda), false, grad_mu, grad_sigma,
+                           loss, terms, status ? status : ctx->d_status_tmp, nullptr);
+}
+
+gaus_status gaus_adam_step(gaus_ctx *ctx, float *mu, float *sigma, const float *grad_mu, const float *grad_sigma,
+                           float *m_mu, float *v_mu, float *m_sigma, float *v_sigma, float *lambda,
+                           const float *terms, int32_t step) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!mu || !sigma || !grad_mu || !grad_sigma || !m_mu || !v_mu || !m_sigma || !v_sigma || !lambda || !terms ||
+      step < 1) {
+    ctx->err = "gaus_adam_step: NULL pointer or step < 1";
+    return GAUS_EINVAL;
+  }
+  const size_t n = (size_t)ctx->plan.V * ctx->plan.B;
+  const gaus_hparams &h = ctx->hp;
+  int blocks = (int)std::min<size_t>((n + 255) / 256, 4096);
+  k_adam<<<blocks, 256, 0, ctx->stream>>>(mu, sigma, grad_mu, grad_sigma, m_mu, v_mu, m_sigma, v_sigma, n, step,
+                                          h.lr, h.beta1, h.beta2, h.eps, h.sigma_min);
+  CK(cudaGetLastError(), "k_adam launch");
+  k_lambda<<<(ctx->plan.B + 127) / 128, 128, 0, ctx->stream>>>(lambda, terms, ctx->plan.B, h.terms, h.rho);
+  CK(cudaGetLastError(), "k_lambda launch");
+  return GAUS_OK;
+}
+
+gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *S) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!S || n_iters < 0 || !S->mu || !S->sigma || !S->m_mu || !S->v_mu || !S->m_sigma || !S->v_sigma ||
+      !S->lambda || !S->step || !S->loss || !S->terms || !S->status) {
+    ctx->err = "gaus_iterate: NULL state pointer or n_iters < 0";
+    return GAUS_EINVAL;
+  }
+  if (n_iters == 0) return GAUS_OK;
+  const uint64_t h = state_hash(S);
+  if (!ctx->gexec || ctx->ghash != h) {
+    drop_graph(ctx);
+    cudaStream_t cap;
+    CK(cudaStreamCreateWithFlags(&cap, cudaStreamNonBlocking), "capture stream");
+    cudaError_t e = cudaStreamBeginCapture(cap, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess) {
+      cudaStreamDestroy(cap);
+      return cuda_fail(ctx, e, "begin capture");
+    }
+    gaus_status st = enqueue_iteration(ctx, cap, S->mu, S->sigma, S->lambda, true, nullptr, nullptr, S->loss,
+                                       S->terms, S->status, S);
+    cudaGraph_t graph = nullptr;
+    e = cudaStreamEndCapture(cap, &graph);
+    cudaStreamDestroy(cap);
+    if (st != GAUS_OK) {
+      if (graph) cudaGraphDestroy(graph);
+      return st;
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "end capture");
+    e = cudaGraphInstantiate(&ctx->gexec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+      ctx->gexec = nullptr;
+      return cuda_fail(ctx, e, "graph instantiate");
+    }
+    ctx->ghash = h;
+  }
+  for (int i = 0; i < n_iters; ++i) CK(cudaGraphLaunch(ctx->gexec, ctx->stream), "graph launch");
+  return GAUS_OK;
+}
+
+gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *S, double *ms_out) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!S || !ms_out || n_iters < 0 || !S->mu || !S->sigma || !S->m_mu || !S->v_mu || !S->m_sigma ||
+      !S->v_sigma || !S->lambda || !S->step || !S->loss || !S->terms || !S->status) {
+    ctx->err = "gaus_profile_iterate: NULL pointer or n_iters < 0";
+    return GAUS_EINVAL;
+  }
+  std::vector<cudaEvent_t> ev(4 * (size_t)n_iters);
+  for (auto &e : ev) CK(cudaEventCreate(&e), "event create");
+  gaus_status st = GAUS_OK;
+  for (int i = 0; i < n_iters && st == GAUS_OK; ++i)
+    st = enqueue_iteration(ctx, ctx->stream, S->mu, S->sigma, S->lambda, true, nullptr, nullptr, S->loss,
+                           S->terms, S->status, S, &ev[4 * (size_t)i]);
+  cudaError_t e = cudaStreamSynchronize(ctx->stream);
+  double acc[3] = {0, 0, 0};
+  for (int i = 0; i < n_iters && st == GAUS_OK && e == cudaSuccess; ++i)
+    for (int k = 0; k < 3; ++k) {
+      float ms = 0.f;
+      cudaEventElapsedTime(&ms, ev[4 * (size_t)i + k], ev[4 * (size_t)i + k + 1]);
+      acc[k] += ms;
+    }
+  for (auto &x : ev) cudaEventDestroy(x);
+  if (st != GAUS_OK) return st;
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "profile sync");
+  for (int k = 0; k < 3; ++k) ms_out[k] += n_iters ? acc[k] / n_iters : 0.0;
+  return GAUS_OK;
+}
+
+gaus_status gaus_round(gaus_ctx *ctx, const float *mu, int32_t *sched) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!mu || !sched) { ctx->err = "gaus_round: NULL pointer"; return GAUS_EINVAL; }
+  const size_t n = (size_t)ctx->plan.V * ctx->plan.B;
+  k_round<<<(int)std::min<size_t>((n + 255) / 256, 4096), 256, 0, ctx->stream>>>(mu, sched, n);
+  CK(cudaGetLastError(), "k_round launch");
+  return GAUS_OK;
+}
+
+gaus_status gaus_legalize(gaus_ctx *ctx, const float *mu, int32_t *sched, int32_t *status) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!mu || !sched || !status) { ctx->err = "gaus_legalize: NULL pointer"; return GAUS_EINVAL; }
+  const Plan &P = ctx->plan;
+  LegArgs A;
+  A.mu = mu; A.s = sched; A.status = status;
+  A.V = P.V; A.B = P.B; A.D = P.D; A.II = P.II; A.nlvl = P.nlvl;
+  A.lvl_ptr = ctx->d_lvl_ptr; A.lvl_nodes = ctx->d_lvl_nodes;
+  A.pred_ptr = ctx->d_cpred_ptr; A.pred_src = ctx->d_cpred_src; A.lat = ctx->d_c_lat;
+  A.back_ptr = ctx->d_cback_ptr; A.back_src = ctx->d_cback_src; A.back_shift = ctx->d_cback_shift;
+  A.asap = ctx->d_asap; A.alap = ctx->d_alap;
+  const int grid = (P.B + 31) / 32;
+  if (P.II > 0) k_legalize_modulo<<<grid, 256, 0, ctx->stream>>>(A);
+  else k_legalize_regular<<<grid, 256, 0, ctx->stream>>>(A);
+  CK(cudaGetLastError(), "legalize launch");
+  return GAUS_OK;
+}
+
+gaus_status gaus_verify(gaus_ctx *ctx, const int32_t *sched, gaus_report *rep) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!sched || !rep) { ctx->err = "gaus_verify: NULL pointer"; return GAUS_EINVAL; }
+  const Plan &P = ctx->plan;
+  VerArgs A;
+  A.s = sched; A.rep = rep;
+  A.V = P.V; A.E = P.E; A.NB = P.NB; A.B = P.B; A.C = P.C; A.D = P.D; A.II = P.II; A.Dh = P.Dh;
+  A.e_src = ctx->d_e_src; A.e_dst = ctx->d_e_dst; A.lat = ctx->d_c_lat; A.cls = ctx->d_c_cls;
+  A.dem = ctx->d_c_dem; A.bits = ctx->d_c_bits;
+  A.b_src = ctx->d_b_src; A.b_dst = ctx->d_b_dst; A.b_dist = ctx->d_b_dist;
+  A.succ_ptr = ctx->d_csucc_ptr; A.succ_dst = ctx->d_csucc_dst; A.limit = ctx->d_limit;
+  k_verify<<<P.B, 256, ctx->smem_ver, ctx->stream>>>(A);
+  CK(cudaGetLastError(), "k_verify launch");
+  return GAUS_OK;
+}
+
+const char *gaus_last_error(const gaus_ctx *ctx) { return ctx ? ctx->err.c_str() : g_create_error.c_str(); }
+
+void gaus_destroy(gaus_ctx *ctx) {
+  if (!ctx) return;
+  if (!ctx->allocs.empty() || ctx->gexec) {
+    if (ctx->stream) cudaStreamSynchronize(ctx->stream);
+    else cudaDeviceSynchronize();
+  }
+  drop_graph(ctx);
+  for (void *p : ctx->allocs) cudaFree(p);
+  delete ctx;
+}
+
+}  // extern "C"

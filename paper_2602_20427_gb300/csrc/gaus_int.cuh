@@ -1,0 +1,268 @@
+// gaus_int.cuh -- integer kernels: rounding (Sec. 3.3 Sampling), legalization
+// (App. A, Alg. 1 and Alg. 2) and the discrete verifier (Sec. 2.1).  Bit-exact
+// by construction: integer arithmetic only, and both legalizations compute a
+// result that does not depend on the order of their updates.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "gaus_internal.h"
+
+namespace gaus {
+
+struct LegArgs {
+  const float *mu;
+  int32_t *s, *status;
+  int V, B, D, II, nlvl;
+  const int32_t *lvl_ptr, *lvl_nodes;
+  const int32_t *pred_ptr, *pred_src, *lat;
+  const int32_t *back_ptr, *back_src, *back_shift;
+  const int32_t *asap, *alap;
+};
+
+// s = floor(mu + 1/2), evaluated exactly in double for every fp32 mu.
+__device__ __forceinline__ int round_half_up(float m, bool &bad) {
+  if (!isfinite(m)) { bad = true; return 0; }
+  double x = floor((double)m + 0.5);
+  x = fmin(fmax(x, -1073741824.0), 1073741824.0);
+  return (int)x;
+}
+
+__global__ void k_round(const float *mu, int32_t *s, size_t n) {
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+    bool bad = false;
+    s[i] = round_half_up(mu[i], bad);
+  }
+}
+
+// Block = 32 restarts (lanes) x 8 node rows.  Alg. 1: clamp to [ASAP, ALAP], then
+// one forward pass level by level: s_v <- max(s_v, max_u s_u + Lat(u)).  The
+// result is the least legal schedule above the clamped input, whatever the
+// order inside a level, so it equals the sequential algorithm bit for bit.
+__global__ void __launch_bounds__(256) k_legalize_regular(const LegArgs A) {
+  const int lane = threadIdx.x & 31, row = threadIdx.x >> 5;
+  const int b = blockIdx.x * 32 + lane;
+  __shared__ int bad_lane[32];
+  if (row == 0) bad_lane[lane] = 0;
+  __syncthreads();
+  const bool bok = b < A.B;
+  if (bok)
+    for (int v = row; v < A.V; v += 8) {
+      bool bad = false;
+      int x = round_half_up(A.mu[(size_t)v * A.B + b], bad);
+      if (bad) bad_lane[lane] = 1;
+      x = max(x, A.asap[v]);
+      x = min(x, A.alap[v]);
+      A.s[(size_t)v * A.B + b] = x;
+    }
+  __syncthreads();
+  for (int l = 1; l < A.nlvl; ++l) {
+    if (bok)
+      for (int q = A.lvl_ptr[l] + row; q < A.lvl_ptr[l + 1]; q += 8) {
+        const int v = A.lvl_nodes[q];
+        int x = A.s[(size_t)v * A.B + b];
+        for (int e = A.pred_ptr[v]; e < A.pred_ptr[v + 1]; ++e) {
+          const int u = A.pred_src[e];
+          x = max(x, A.s[(size_t)u * A.B + b] + A.lat[u]);
+        }
+        A.s[(size_t)v * A.B + b] = x;
+      }
+    __syncthreads();
+  }
+  if (row == 0 && bok) A.status[b] = bad_lane[lane] ? GAUS_ENONFINITE : GAUS_OK;
+}
+
+// Alg. 2: sweeps in topological (level) order of
+//   s_v <- max(s_v, 0, max_u s_u + Lat(u), max_{(j -> v, k)} s_j + Lat(j) - k II)
+// until a sweep changes nothing, at most |V| sweeps.  The updates only raise
+// values and the iteration is bounded by the least fixed point above the
+// rounded input, which it reaches within |V| sweeps whenever the recurrences are
+// feasible, so the converged result is order independent.
+__global__ void __launch_bounds__(256) k_legalize_modulo(const LegArgs A) {
+  const int lane = threadIdx.x & 31, row = threadIdx.x >> 5;
+  const int b = blockIdx.x * 32 + lane;
+  __shared__ int bad_lane[32], changed[32], done[32];
+  __shared__ int any_changed;
+  if (row == 0) { bad_lane[lane] = 0; done[lane] = 0; }
+  __syncthreads();
+  const bool bok = b < A.B;
+  if (bok)
+    for (int v = row; v < A.V; v += 8) {
+      bool bad = false;
+      const int x = round_half_up(A.mu[(size_t)v * A.B + b], bad);
+      if (bad) bad_lane[lane] = 1;
+      A.s[(size_t)v * A.B + b] = x;
+    }
+  __syncthreads();
+  for (int sweep = 0; sweep < A.V; ++sweep) {
+    if (row == 0) changed[lane] = 0;
+    if (threadIdx.x == 0) any_changed = 0;
+    __syncthreads();
+    for (int l = 0; l < A.nlvl; ++l) {
+      if (bok)
+        for (int q = A.lvl_ptr[l] + row; q < A.lvl_ptr[l + 1]; q += 8) {
+          const int v = A.lvl_nodes[q];
+          int t = 0;
+          for (int e = A.pred_ptr[v]; e < A.pred_ptr[v + 1]; ++e) {
+            const int u = A.pred_src[e];
+            t = max(t, A.s[(size_t)u * A.B + b] + A.lat[u]);
+          }
+          for (int e = A.back_ptr[v]; e < A.back_ptr[v + 1]; ++e)
+            t = max(t, A.s[(size_t)A.back_src[e] * A.B + b] + A.back_shift[e]);
+          if (t > A.s[(size_t)v * A.B + b]) {
+            A.s[(size_t)v * A.B + b] = t;
+            changed[lane] = 1;
+          }
+        }
+      __syncthreads();
+    }
+    if (row == 0 && bok) {
+      if (!changed[lane]) done[lane] = 1;
+      else atomicOr(&any_changed, 1);
+    }
+    __syncthreads();
+    if (!any_changed) break;
+  }
+  if (row == 0 && bok)
+    A.status[b] = bad_lane[lane] ? GAUS_ENONFINITE : (done[lane] ? GAUS_OK : GAUS_ENOTCONV);
+}
+
+struct VerArgs {
+  const int32_t *s;
+  gaus_report *rep;
+  int V, E, NB, B, C, D, II, Dh;
+  const int32_t *e_src, *e_dst, *lat, *cls, *dem, *bits;
+  const int32_t *b_src, *b_dst, *b_dist;
+  const int32_t *succ_ptr, *succ_dst;
+  const float *limit;
+};
+
+__device__ __forceinline__ long long block_sum_ll(long long x, long long *buf) {
+  const int tid = threadIdx.x;
+  buf[tid] = x;
+  __syncthreads();
+  for (int s = 128; s > 0; s >>= 1) {
+    if (tid < s) buf[tid] += buf[tid + s];
+    __syncthreads();
+  }
+  const long long r = buf[0];
+  __syncthreads();
+  return r;
+}
+
+// One block (256 threads) per restart.  Shared: usage counts C*Dh (int64),
+// storage difference array D+1 (int64), folded storage Dh (int64).
+__global__ void __launch_bounds__(256) k_verify(const VerArgs A) {
+  extern __shared__ __align__(16) unsigned char smem_v[];
+  long long *cnt = reinterpret_cast<long long *>(smem_v);
+  long long *diff = cnt + (size_t)A.C * A.Dh;
+  long long *mm = diff + (A.D + 1);
+  __shared__ long long buf[256];
+  const int b = blockIdx.x, tid = threadIdx.x;
+  for (int i = tid; i < A.C * A.Dh; i += 256) cnt[i] = 0;
+  for (int i = tid; i <= A.D; i += 256) diff[i] = 0;
+  for (int i = tid; i < A.Dh; i += 256) mm[i] = 0;
+  __syncthreads();
+  auto S = [&](int v) { return A.s[(size_t)v * A.B + b]; };
+  long long ndep = 0, lcom = 0, nlat = 0, nrec = 0;
+  for (int e = tid; e < A.E; e += 256) {
+    const int u = A.e_src[e], v = A.e_dst[e];
+    const int su = S(u), sv = S(v);
+    if ((long long)sv < (long long)su + A.lat[u]) ++ndep;
+    lcom += (long long)sv - su;
+  }
+  for (int v = tid; v < A.V; v += 256) {
+    const int sv = S(v);
+    if (sv < 0 || (long long)sv + A.lat[v] > A.D) ++nlat;
+    if (sv >= 0 && sv < A.D) {
+      const int t = A.II > 0 ? sv % A.II : sv;
+      atomicAdd(reinterpret_cast<unsigned long long *>(&cnt[A.cls[v] * A.Dh + t]),
+                (unsigned long long)(long long)A.dem[v]);
+    }
+    // Mem: live on [s_v, max over successors of s_w) (leaves: until D), within [0, D)
+    long long last = A.D;
+    if (A.succ_ptr[v + 1] > A.succ_ptr[v]) {
+      last = LLONG_MIN;
+      for (int q = A.succ_ptr[v]; q < A.succ_ptr[v + 1]; ++q) last = max(last, (long long)S(A.succ_dst[q]));
+    }
+    const long long lo = max((long long)sv, 0LL), hi = min(last, (long long)A.D);
+    if (lo < hi && A.bits[v] != 0) {
+      atomicAdd(reinterpret_cast<unsigned long long *>(&diff[lo]), (unsigned long long)(long long)A.bits[v]);
+      atomicAdd(reinterpret_cast<unsigned long long *>(&diff[hi]), (unsigned long long)(-(long long)A.bits[v]));
+    }
+  }
+  if (A.II > 0)
+    for (int q = tid; q < A.NB; q += 256) {
+      const int j = A.b_src[q], i = A.b_dst[q];
+      if ((long long)S(i) + (long long)A.b_dist[q] * A.II < (long long)S(j) + A.lat[j]) ++nrec;
+    }
+  __syncthreads();
+  ndep = block_sum_ll(ndep, buf);
+  lcom = block_sum_ll(lcom, buf);
+  nlat = block_sum_ll(nlat, buf);
+  nrec = block_sum_ll(nrec, buf);
+  if (tid == 0) {
+    gaus_report R;
+    R.n_dep_viol = ndep;
+    R.n_lat_viol = nlat;
+    R.n_rec_viol = nrec;
+    R.L_com = lcom;
+    R.n_res_viol = 0;
+    R.L_res = 0;
+    for (int c = 0; c < 16; ++c) R.peak[c] = 0;
+    for (int c = 0; c < A.C; ++c) {
+      long long pk = 0;
+      const float lim = A.limit[c];
+      for (int t = 0; t < A.Dh; ++t) {
+        const long long x = cnt[c * A.Dh + t];
+        pk = max(pk, x);
+        if (isfinite(lim) && (double)x > (double)lim) R.n_res_viol++;
+      }
+      R.peak[c] = pk;
+      R.L_res += pk;
+    }
+    long long run = 0, lmem = 0;
+    for (int d = 0; d < A.D; ++d) {
+      run += diff[d];
+      lmem = max(lmem, run);
+      mm[A.II > 0 ? d % A.II : d] += run;
+    }
+    long long lmm = 0;
+    for (int t = 0; t < A.Dh; ++t) lmm = max(lmm, mm[t]);
+    R.L_mem = lmem;
+    R.L_mmem = lmm;
+    R.feasible = (ndep == 0 && nlat == 0 && nrec == 0);
+    R.res_ok = R.n_res_viol == 0;
+    A.rep[b] = R;
+  }
+}
+
+// Elementwise Adam on (V, B) arrays (gaus_adam_step), then sigma clamp.
+__global__ void k_adam(float *mu, float *sg, const float *gmu, const float *gsg, float *m1, float *v1,
+                       float *m2, float *v2, size_t n, int step, float lr, float beta1, float beta2,
+                       float eps, float sigma_min) {
+  const float bc1 = 1.0f - powf(beta1, (float)step), bc2 = 1.0f - powf(beta2, (float)step);
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+    const float g1 = gmu[i], g2 = gsg[i];
+    const float a1 = beta1 * m1[i] + (1.0f - beta1) * g1;
+    const float b1 = beta2 * v1[i] + (1.0f - beta2) * g1 * g1;
+    const float a2 = beta1 * m2[i] + (1.0f - beta1) * g2;
+    const float b2 = beta2 * v2[i] + (1.0f - beta2) * g2 * g2;
+    m1[i] = a1; v1[i] = b1; m2[i] = a2; v2[i] = b2;
+    mu[i] = mu[i] - lr * (a1 / bc1) / (sqrtf(b1 / bc2) + eps);
+    sg[i] = fmaxf(sg[i] - lr * (a2 / bc1) / (sqrtf(b2 / bc2) + eps), sigma_min);
+  }
+}
+
+// lambda[b, k] += rho * V_k for the active constraints (Sec. 3.3).
+__global__ void k_lambda(float *lambda, const float *terms, int B, unsigned on, float rho) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const float *T = terms + (size_t)b * GAUS_NT;
+  if (on & GAUS_DEP) lambda[b * GAUS_K + GAUS_K_DEP] += rho * T[GAUS_T_VDEP];
+  if (on & GAUS_RES_VIOL) lambda[b * GAUS_K + GAUS_K_RES] += rho * T[GAUS_T_VRES];
+  if (on & GAUS_REC) lambda[b * GAUS_K + GAUS_K_REC] += rho * T[GAUS_T_VREC];
+}
+
+}  // namespace gaus

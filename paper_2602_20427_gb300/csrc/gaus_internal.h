@@ -1,0 +1,104 @@
+// gaus_internal.h -- context layout shared by the host planner and the CUDA code.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "gaus.h"
+
+namespace gaus {
+
+// Threads per block of the per-(node, restart) kernels.
+constexpr int kThreads = 128;
+// Own-window points cached in shared memory per thread (longer windows recompute).
+constexpr int kCache = 32;
+// Fixed-point scale of the usage histograms: P * 2^32 accumulated in int64.
+constexpr float kFix = 4294967296.0f;
+constexpr double kInvFix = 1.0 / 4294967296.0;
+// Limits checked by gaus_create.
+constexpr int kMaxClasses = 16;
+
+// Host-side plan produced by plan_problem() (pure C++, no CUDA).
+struct Plan {
+  int V = 0, E = 0, NB = 0, C = 0, D = 0, II = 0, Dh = 0, B = 0, cp = 0;
+  std::vector<int32_t> asap, alap;        // caller order
+  std::vector<int32_t> perm;              // internal -> caller
+  std::vector<int32_t> inv;               // caller -> internal
+  std::vector<int32_t> level;             // caller order, topological level
+  // internal-order node attributes
+  std::vector<float> w, bits;
+  std::vector<int32_t> lat, cls;
+  // CSC of internal consumers: producer caller id, producer latency
+  std::vector<int32_t> in_ptr, in_src, in_lat;
+  // CSR of internal producers: consumer caller id
+  std::vector<int32_t> out_ptr, out_dst;
+  // back edges grouped by internal consumer i: producer caller id j, shift Lat(j) - k II
+  std::vector<int32_t> bin_ptr, bin_src, bin_shift;
+  // back edges grouped by internal producer j: consumer caller id i, same shift
+  std::vector<int32_t> bout_ptr, bout_dst, bout_shift;
+  // segments of internal nodes, each inside one class: start, end, class
+  std::vector<int32_t> seg;               // 3 * nseg
+  std::vector<int32_t> cls_seg_ptr;       // C + 1, segments of class c
+  int nseg = 0;
+  // caller-order data for the integer kernels
+  std::vector<int32_t> lvl_ptr, lvl_nodes;           // nodes (caller ids) by level
+  std::vector<int32_t> cpred_ptr, cpred_src;         // CSC by caller consumer id
+  std::vector<int32_t> csucc_ptr, csucc_dst;         // CSR by caller producer id
+  std::vector<int32_t> cback_ptr, cback_src, cback_shift;  // back edges by caller consumer
+  std::vector<int32_t> c_lat, c_cls, c_dem, c_bits;  // caller order
+  std::vector<int32_t> e_src, e_dst;                 // edge list (caller ids)
+  std::vector<int32_t> b_src, b_dst, b_dist;
+  std::vector<float> limit;
+  int nlvl = 0;
+  int has_reg_succ_any = 0;
+};
+
+// Returns GAUS_OK or an error with a message.
+gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err);
+gaus_status check_hparams(const gaus_hparams *hp, std::string *err);
+
+}  // namespace gaus
+
+struct gaus_ctx {
+  gaus::Plan plan;
+  gaus_hparams hp;
+  cudaStream_t stream = nullptr;
+  std::string err;
+  int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per pass
+  size_t smem_fwd = 0, smem_upd = 0, smem_fin = 0, smem_ver = 0;
+  // device graph
+  int32_t *d_perm = nullptr;
+  float *d_w = nullptr, *d_bits = nullptr, *d_limit = nullptr;
+  int32_t *d_lat = nullptr, *d_cls = nullptr;
+  int32_t *d_in_ptr = nullptr, *d_in_src = nullptr, *d_in_lat = nullptr;
+  int32_t *d_out_ptr = nullptr, *d_out_dst = nullptr;
+  int32_t *d_bin_ptr = nullptr, *d_bin_src = nullptr, *d_bin_shift = nullptr;
+  int32_t *d_bout_ptr = nullptr, *d_bout_dst = nullptr, *d_bout_shift = nullptr;
+  int32_t *d_seg = nullptr, *d_cls_seg_ptr = nullptr;
+  int32_t *d_lvl_ptr = nullptr, *d_lvl_nodes = nullptr;
+  int32_t *d_cpred_ptr = nullptr, *d_cpred_src = nullptr;
+  int32_t *d_csucc_ptr = nullptr, *d_csucc_dst = nullptr;
+  int32_t *d_cback_ptr = nullptr, *d_cback_src = nullptr, *d_cback_shift = nullptr;
+  int32_t *d_c_lat = nullptr, *d_c_cls = nullptr, *d_c_dem = nullptr, *d_c_bits = nullptr;
+  int32_t *d_e_src = nullptr, *d_e_dst = nullptr;
+  int32_t *d_b_src = nullptr, *d_b_dst = nullptr, *d_b_dist = nullptr;
+  int32_t *d_asap = nullptr, *d_alap = nullptr;
+  // scratch
+  long long *d_hpart = nullptr;  // nblk * RB * Dh fixed-point usage partials
+  int2 *d_hspan = nullptr;       // nblk folded bin span written by each block
+  double *d_fwd = nullptr;       // nblk * RB * 3 forward sums (dep, com, rec)
+  float *d_gpart = nullptr;      // 6 * V * B partial gradient sums (internal index)
+  float *d_H = nullptr;          // B * C * Dh usage adjoint dL/dU
+  float *d_coef = nullptr;       // B * 4 (c_dep, c_rec)
+  int32_t *d_nonfinite = nullptr;  // B flags
+  int32_t *d_status_tmp = nullptr; // B
+  float *d_loss_tmp = nullptr, *d_terms_tmp = nullptr;
+  // captured iteration
+  cudaGraphExec_t gexec = nullptr;
+  gaus_state gstate{};
+  uint64_t ghash = 0;
+  std::vector<void *> allocs;
+};

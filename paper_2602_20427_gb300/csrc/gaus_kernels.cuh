@@ -1,0 +1,527 @@
+// gaus_kernels.cuh -- device code of one GauS iteration (Sec. 3.2-3.3, App. B).
+//
+// Work item: one (node v, restart b).  Threads of a warp are restarts of the same
+// node (lanes = b), so every mu/sigma gather of a neighbour is one coalesced
+// 128-byte load.  Each thread keeps its own window of CDF points
+//   C_v(t) = Phi((t + 1/2 - mu_v) / sigma_v),  t in [a_v, b_v] = points within
+//   window_k * sigma_v of mu_v, with C_v(t) = 0 below and 1 above (Eq. round and
+// its open end bins), and evaluates each neighbour's CDF at the points it needs.
+//
+// k_fwd     : bin masses -> usage histogram (shared-memory int64 fixed point, one
+//             class per block, no global atomics) and every edge term from both
+//             endpoints (gathered through CSC as consumer and CSR as producer):
+//             forward sums and the unscaled partial gradients.
+// k_finalize: one block per restart -- usage per class, LogSumExp (Eq. max),
+//             ReLU (Eq. relu), the augmented-Lagrangian coefficients (Sec. 3.3).
+// k_update  : usage adjoint of the node's own window, the combined gradient and
+//             (optionally) the Adam step.
+#pragma once
+
+#include <climits>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "gaus_internal.h"
+
+namespace gaus {
+
+struct IterArgs {
+  const float *mu, *sg;  // (V, B) caller order
+  int V, B, D, II, Dh, C, RB, G;
+  float k_win, alpha;
+  const int32_t *perm;
+  const float *w;
+  const int32_t *lat;
+  const int32_t *in_ptr, *in_src, *in_lat;
+  const int32_t *out_ptr, *out_dst;
+  const int32_t *bin_ptr, *bin_src, *bin_shift;
+  const int32_t *bout_ptr, *bout_dst, *bout_shift;
+  const int32_t *seg;
+  long long *hpart;
+  int2 *hspan;
+  double *fwd;
+  float *gpart;
+  int32_t *nonfinite;
+};
+
+struct FinArgs {
+  int B, C, Dh, RB, G;
+  unsigned terms;
+  float tau, rho, alpha, w_res, w_mem;
+  const int32_t *cls_seg_ptr;
+  const float *limit;
+  const long long *hpart;
+  const int2 *hspan;
+  const double *fwd;
+  float *lambda;      // read; updated in place when update_lambda
+  int update_lambda;
+  int32_t *step;      // incremented when not NULL
+  float *H, *coef, *loss, *terms_out;
+  int32_t *status, *nonfinite;
+};
+
+struct UpdArgs {
+  float *mu, *sg;  // caller order; written when adam
+  int V, B, D, II, Dh, C, RB, G;
+  float k_win;
+  const int32_t *perm;
+  const float *w;
+  const int32_t *seg;
+  const float *gpart;
+  const float *H, *coef;
+  float *grad_mu, *grad_sg;                  // gradient mode
+  float *m_mu, *v_mu, *m_sg, *v_sg;          // Adam mode
+  const int32_t *step_dev;                   // per-restart step (Adam mode, iterate)
+  float lr, beta1, beta2, eps, sigma_min;
+};
+
+// Points t with |t + 1/2 - mu| <= k sigma, clipped to [0, D-2]; a = b + 1 when empty.
+__device__ __forceinline__ void window(float mu, float sg, float k, int D, int &a, int &b) {
+  float lo = ceilf(mu - k * sg - 0.5f), hi = floorf(mu + k * sg - 0.5f);
+  lo = fminf(fmaxf(lo, 0.0f), (float)(D - 1));
+  hi = fminf(fmaxf(hi, -1.0f), (float)(D - 2));
+  a = (int)lo;
+  b = (int)hi;
+}
+
+// Windowed CDF of a neighbour at integer point x.
+__device__ __forceinline__ float cdf_at(int x, float mu, float inv_s, int a, int b) {
+  if (x < a) return 0.0f;
+  if (x > b) return 1.0f;
+  return normcdff(((float)x + 0.5f - mu) * inv_s);
+}
+
+__device__ __forceinline__ int fold_bin(int d, int II) { return II > 0 ? d % II : d; }
+
+// A restart's (mu, sigma) is usable when both are finite and sigma >= 1e-30, so
+// that 1/sigma is finite.
+__device__ __forceinline__ bool usable(float mu, float sg) {
+  return isfinite(mu) && isfinite(sg) && sg >= 1e-30f;
+}
+
+constexpr float kInvSqrt2Pi = 0.3989422804014327f;
+constexpr float kInvSqrt2 = 0.7071067811865476f;
+
+template <bool kDep, bool kCom, bool kRec>
+__global__ void __launch_bounds__(kThreads) k_fwd(const IterArgs A) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int tid = threadIdx.x, RB = A.RB, Dh = A.Dh;
+  long long *hist = reinterpret_cast<long long *>(smem);
+  float *cC = reinterpret_cast<float *>(hist + (size_t)RB * Dh);
+  float *cF = cC + kCache * kThreads;
+  float *cZ = cF + kCache * kThreads;
+  __shared__ int s_lo, s_hi;
+  __shared__ double s_red[3][kThreads];
+
+  const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
+  const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1];
+  for (int i = tid; i < RB * Dh; i += kThreads) hist[i] = 0;
+  if (tid == 0) { s_lo = INT_MAX; s_hi = INT_MIN; }
+  __syncthreads();
+
+  const int r = tid % RB, b = g * RB + r, rows = kThreads / RB;
+  const bool bok = b < A.B;
+  const size_t VB = (size_t)A.V * A.B;
+  float fdep = 0.f, fcom = 0.f, frec = 0.f;
+  int lo = INT_MAX, hi = INT_MIN;
+
+  for (int vi = s0 + tid / RB; vi < s1; vi += rows) {
+    if (!bok) continue;
+    const int vc = A.perm[vi];
+    const size_t gi = (size_t)vi * A.B + b;
+    const float mu = A.mu[(size_t)vc * A.B + b], sg = A.sg[(size_t)vc * A.B + b];
+    if (!usable(mu, sg)) {
+      A.nonfinite[b] = 1;
+      for (int k = 0; k < 6; ++k) A.gpart[k * VB + gi] = 0.f;
+      continue;
+    }
+    const float inv_s = 1.0f / sg, wv = A.w[vi];
+    int a, bw;
+    window(mu, sg, A.k_win, A.D, a, bw);
+    const int n = bw - a + 1;
+
+    // ---- own points: cache C, phi, z*phi; bin masses into the usage histogram ----
+    // P(d) for d in [a, b+1] from Q(|z|) = Phi(-|z|) so that both tails keep
+    // relative accuracy: C = Q when z <= 0, 1 - Q otherwise.
+    float zp = 0.f, qp = 0.f;
+    for (int j = 0; j <= n; ++j) {
+      float zc = 0.f, qc = 0.f, P;
+      if (j < n) {
+        zc = ((float)(a + j) + 0.5f - mu) * inv_s;
+        qc = 0.5f * erfcf(fabsf(zc) * kInvSqrt2);
+        if (j < kCache) {
+          const float f = kInvSqrt2Pi * expf(-0.5f * zc * zc);
+          cC[j * kThreads + tid] = zc <= 0.f ? qc : 1.0f - qc;
+          cF[j * kThreads + tid] = f;
+          cZ[j * kThreads + tid] = zc * f;
+        }
+      }
+      if (n == 0) P = 1.0f;
+      else if (j == 0) P = zc <= 0.f ? qc : 1.0f - qc;
+      else if (j == n) P = zp <= 0.f ? 1.0f - qp : qp;
+      else if (zc <= 0.f) P = qc - qp;
+      else if (zp > 0.f) P = qp - qc;
+      else P = (0.5f - qc) + (0.5f - qp);
+      const long long q = __float2ll_rn(wv * P * kFix);
+      atomicAdd(reinterpret_cast<unsigned long long *>(&hist[r * Dh + fold_bin(a + j, A.II)]),
+                (unsigned long long)q);
+      zp = zc;
+      qp = qc;
+    }
+    lo = min(lo, a);
+    hi = max(hi, bw + 1);
+
+    // own point j: C, phi, z*phi (recomputed beyond the cache)
+    auto own = [&](int j, float &C, float &f, float &zf) {
+      if (j < kCache) {
+        C = cC[j * kThreads + tid];
+        f = cF[j * kThreads + tid];
+        zf = cZ[j * kThreads + tid];
+      } else {
+        const float z = ((float)(a + j) + 0.5f - mu) * inv_s;
+        const float q = 0.5f * erfcf(fabsf(z) * kInvSqrt2);
+        C = z <= 0.f ? q : 1.0f - q;
+        f = kInvSqrt2Pi * expf(-0.5f * z * z);
+        zf = z * f;
+      }
+    };
+
+    float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f;
+    // ---- in-edges u -> v (own = consumer), latency L = Lat(u) ----
+    // V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
+    // dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
+    // dL_com,e/dC_v(t) = -C_u(t)
+    if (kDep || kCom) {
+      for (int e = A.in_ptr[vi]; e < A.in_ptr[vi + 1]; ++e) {
+        const int uc = A.in_src[e], L = A.in_lat[e];
+        const float mu_u = A.mu[(size_t)uc * A.B + b], sg_u = A.sg[(size_t)uc * A.B + b];
+        if (!usable(mu_u, sg_u)) continue;
+        const float inv_u = 1.0f / sg_u;
+        int au, bu;
+        window(mu_u, sg_u, A.k_win, A.D, au, bu);
+        float c_lo = cdf_at(a - L, mu_u, inv_u, au, bu);
+        for (int j = 0; j < n; ++j) {
+          const int t = a + j;
+          const float c_hi = cdf_at(t + 1 - L, mu_u, inv_u, au, bu);
+          const float p = c_hi - c_lo;
+          float Cv, f, zf;
+          own(j, Cv, f, zf);
+          if (kDep) {
+            fdep += Cv * p;
+            Ad += p * f;
+            Bd += p * zf;
+          }
+          if (kCom) {
+            const float cu = (L == 1) ? c_hi : cdf_at(t, mu_u, inv_u, au, bu);
+            fcom += cu * (1.0f - Cv);
+            Ao -= A.alpha * cu * f;
+            Bo -= A.alpha * cu * zf;
+          }
+          c_lo = c_hi;
+        }
+        if (kDep) fdep += 1.0f - c_lo;
+      }
+    }
+    // ---- out-edges v -> w (own = producer), latency L = Lat(v) ----
+    // dV_e/dC_v(x) = -P_w(x + L);  dL_com,e/dC_v(x) = 1 - C_w(x)
+    // L_com,e part = sum_{x in own, x < a_w} C_v(x) + max(0, a_w - 1 - b_v)
+    if (kDep || kCom) {
+      const int L = A.lat[vi];
+      for (int e = A.out_ptr[vi]; e < A.out_ptr[vi + 1]; ++e) {
+        const int wc = A.out_dst[e];
+        const float mu_w = A.mu[(size_t)wc * A.B + b], sg_w = A.sg[(size_t)wc * A.B + b];
+        if (!usable(mu_w, sg_w)) continue;
+        const float inv_w = 1.0f / sg_w;
+        int aw, bw2;
+        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
+        float c_lo = cdf_at(a + L - 1, mu_w, inv_w, aw, bw2);
+        for (int j = 0; j < n; ++j) {
+          const int x = a + j;
+          const float c_hi = cdf_at(x + L, mu_w, inv_w, aw, bw2);
+          float Cv, f, zf;
+          own(j, Cv, f, zf);
+          if (kDep) {
+            const float p = c_hi - c_lo;
+            Ad -= p * f;
+            Bd -= p * zf;
+          }
+          if (kCom) {
+            const float cw = (L == 1) ? c_lo : cdf_at(x, mu_w, inv_w, aw, bw2);
+            Ao += A.alpha * (1.0f - cw) * f;
+            Bo += A.alpha * (1.0f - cw) * zf;
+            if (x < aw) fcom += Cv;
+          }
+          c_lo = c_hi;
+        }
+        if (kCom) fcom += (float)max(0, aw - 1 - bw);
+      }
+    }
+    // ---- back edges (App. B.3): a dependency with latency Lat(j) - k II ----
+    if (kRec) {
+      for (int e = A.bin_ptr[vi]; e < A.bin_ptr[vi + 1]; ++e) {  // own = consumer i
+        const int jc = A.bin_src[e], L = A.bin_shift[e];
+        const float mu_u = A.mu[(size_t)jc * A.B + b], sg_u = A.sg[(size_t)jc * A.B + b];
+        if (!usable(mu_u, sg_u)) continue;
+        const float inv_u = 1.0f / sg_u;
+        int au, bu;
+        window(mu_u, sg_u, A.k_win, A.D, au, bu);
+        float c_lo = cdf_at(a - L, mu_u, inv_u, au, bu);
+        for (int j = 0; j < n; ++j) {
+          const float c_hi = cdf_at(a + j + 1 - L, mu_u, inv_u, au, bu);
+          const float p = c_hi - c_lo;
+          float Cv, f, zf;
+          own(j, Cv, f, zf);
+          frec += Cv * p;
+          Ar += p * f;
+          Br += p * zf;
+          c_lo = c_hi;
+        }
+        frec += 1.0f - c_lo;
+      }
+      for (int e = A.bout_ptr[vi]; e < A.bout_ptr[vi + 1]; ++e) {  // own = producer j
+        const int ic = A.bout_dst[e], L = A.bout_shift[e];
+        const float mu_w = A.mu[(size_t)ic * A.B + b], sg_w = A.sg[(size_t)ic * A.B + b];
+        if (!usable(mu_w, sg_w)) continue;
+        const float inv_w = 1.0f / sg_w;
+        int aw, bw2;
+        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
+        float c_lo = cdf_at(a + L - 1, mu_w, inv_w, aw, bw2);
+        for (int j = 0; j < n; ++j) {
+          const float c_hi = cdf_at(a + j + L, mu_w, inv_w, aw, bw2);
+          const float p = c_hi - c_lo;
+          float Cv, f, zf;
+          own(j, Cv, f, zf);
+          Ar -= p * f;
+          Br -= p * zf;
+          c_lo = c_hi;
+        }
+      }
+    }
+    A.gpart[0 * VB + gi] = Ad;
+    A.gpart[1 * VB + gi] = Bd;
+    A.gpart[2 * VB + gi] = Ao;
+    A.gpart[3 * VB + gi] = Bo;
+    A.gpart[4 * VB + gi] = Ar;
+    A.gpart[5 * VB + gi] = Br;
+  }
+
+  // ---- per-restart forward sums of this block (fixed order) ----
+  s_red[0][tid] = fdep;
+  s_red[1][tid] = fcom;
+  s_red[2][tid] = frec;
+  if (lo <= hi) {
+    atomicMin(&s_lo, lo);
+    atomicMax(&s_hi, hi);
+  }
+  __syncthreads();
+  if (tid < RB) {
+    double acc[3] = {0.0, 0.0, 0.0};
+    for (int row = 0; row < rows; ++row)
+      for (int k = 0; k < 3; ++k) acc[k] += s_red[k][row * RB + tid];
+    for (int k = 0; k < 3; ++k) A.fwd[((size_t)blk * RB + tid) * 3 + k] = acc[k];
+  }
+  // ---- histogram rows restricted to the folded span the block touched ----
+  int flo = s_lo, fhi = s_hi;
+  if (flo > fhi) {
+    flo = 1;
+    fhi = 0;
+  } else if (A.II > 0) {
+    if (fhi - flo + 1 >= A.II) {
+      flo = 0;
+      fhi = A.II - 1;
+    } else {
+      const int x = flo % A.II, y = fhi % A.II;
+      if (x <= y) { flo = x; fhi = y; } else { flo = 0; fhi = A.II - 1; }
+    }
+  }
+  if (tid == 0) A.hspan[blk] = make_int2(flo, fhi);
+  const int len = fhi - flo + 1;
+  if (len > 0)
+    for (int i = tid; i < RB * len; i += kThreads) {
+      const int rr = i / len, d = flo + i % len;
+      A.hpart[((size_t)blk * RB + rr) * Dh + d] = hist[rr * Dh + d];
+    }
+}
+
+// Deterministic block reduction (blockDim.x == 256).
+__device__ __forceinline__ double block_sum(double x, double *buf) {
+  const int tid = threadIdx.x;
+  buf[tid] = x;
+  __syncthreads();
+  for (int s = 128; s > 0; s >>= 1) {
+    if (tid < s) buf[tid] += buf[tid + s];
+    __syncthreads();
+  }
+  const double r = buf[0];
+  __syncthreads();
+  return r;
+}
+__device__ __forceinline__ double block_max(double x, double *buf) {
+  const int tid = threadIdx.x;
+  buf[tid] = x;
+  __syncthreads();
+  for (int s = 128; s > 0; s >>= 1) {
+    if (tid < s) buf[tid] = fmax(buf[tid], buf[tid + s]);
+    __syncthreads();
+  }
+  const double r = buf[0];
+  __syncthreads();
+  return r;
+}
+
+// One block (256 threads) per restart.
+__global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
+  extern __shared__ __align__(16) unsigned char smem_f[];
+  double *U = reinterpret_cast<double *>(smem_f);  // C * Dh
+  __shared__ double buf[256];
+  __shared__ double s_m[kMaxClasses], s_s[kMaxClasses];
+  const int b = blockIdx.x, g = b / A.RB, r = b % A.RB, tid = threadIdx.x, Dh = A.Dh;
+
+  for (int c = 0; c < A.C; ++c)
+    for (int t = tid; t < Dh; t += 256) {
+      long long acc = 0;
+      for (int s = A.cls_seg_ptr[c]; s < A.cls_seg_ptr[c + 1]; ++s) {
+        const int blk = s * A.G + g;
+        const int2 sp = A.hspan[blk];
+        if (t >= sp.x && t <= sp.y) acc += A.hpart[((size_t)blk * A.RB + r) * Dh + t];
+      }
+      U[c * Dh + t] = (double)acc * kInvFix;
+    }
+  __syncthreads();
+
+  // forward sums of the edge terms over every block of this restart group
+  double f3[3] = {0.0, 0.0, 0.0};
+  const int nseg = A.cls_seg_ptr[A.C];
+  for (int s = tid; s < nseg; s += 256)
+    for (int k = 0; k < 3; ++k) f3[k] += A.fwd[((size_t)(s * A.G + g) * A.RB + r) * 3 + k];
+  const double vdep = block_sum(f3[0], buf);
+  const double lcom = block_sum(f3[1], buf);
+  const double vrec = block_sum(f3[2], buf);
+
+  // ReLU excess over finite limits (Eq. relu)
+  double ex = 0.0;
+  for (int i = tid; i < A.C * Dh; i += 256) {
+    const float R = A.limit[i / Dh];
+    if (isfinite(R) && U[i] > (double)R) ex += U[i] - (double)R;
+  }
+  const double vres = block_sum(ex, buf);
+
+  // LogSumExp per class (Eq. max), max shifted out
+  double lse_sum = 0.0;
+  for (int c = 0; c < A.C; ++c) {
+    double m = -1e300;
+    for (int t = tid; t < Dh; t += 256) m = fmax(m, U[c * Dh + t]);
+    m = block_max(m, buf);
+    double s = 0.0;
+    for (int t = tid; t < Dh; t += 256) s += (double)expf((float)((U[c * Dh + t] - m) / A.tau));
+    s = block_sum(s, buf);
+    if (tid == 0) { s_m[c] = m; s_s[c] = s; }
+    lse_sum += m + (double)A.tau * log(s);
+  }
+  __syncthreads();
+
+  const bool on_dep = A.terms & GAUS_DEP, on_com = A.terms & GAUS_COM;
+  const bool on_robj = A.terms & GAUS_RES_OBJ, on_rv = A.terms & GAUS_RES_VIOL;
+  const bool on_rec = A.terms & GAUS_REC;
+  const float *lam = A.lambda + (size_t)b * GAUS_K;
+  const double c_res = on_rv ? (double)lam[GAUS_K_RES] + (double)A.rho * vres : 0.0;
+  if (tid == 0) {
+    double L = 0.0;
+    if (on_robj) L += (double)A.w_res * lse_sum;
+    if (on_com) L += (double)A.alpha * lcom;
+    const double Vk[3] = {on_dep ? vdep : 0.0, on_rv ? vres : 0.0, on_rec ? vrec : 0.0};
+    const bool act[3] = {on_dep, on_rv, on_rec};
+    for (int k = 0; k < 3; ++k)
+      if (act[k]) L += (double)lam[k] * Vk[k] + 0.5 * (double)A.rho * Vk[k] * Vk[k];
+    float *T = A.terms_out + (size_t)b * GAUS_NT;
+    T[GAUS_T_RES] = on_robj ? (float)lse_sum : 0.f;
+    T[GAUS_T_COM] = on_com ? (float)lcom : 0.f;
+    T[GAUS_T_REG] = 0.f;
+    T[GAUS_T_VDEP] = (float)Vk[0];
+    T[GAUS_T_VRES] = (float)Vk[1];
+    T[GAUS_T_VREC] = (float)Vk[2];
+    A.loss[b] = (float)L;
+    A.coef[b * 4 + 0] = on_dep ? (float)((double)lam[GAUS_K_DEP] + (double)A.rho * vdep) : 0.f;
+    A.coef[b * 4 + 1] = on_rec ? (float)((double)lam[GAUS_K_REC] + (double)A.rho * vrec) : 0.f;
+    const int bad = A.nonfinite[b];
+    if (A.status) A.status[b] = bad ? GAUS_ENONFINITE : GAUS_OK;
+    A.nonfinite[b] = 0;
+    if (A.update_lambda) {
+      float *lw = A.lambda + (size_t)b * GAUS_K;
+      for (int k = 0; k < 3; ++k)
+        if (act[k]) lw[k] = (float)((double)lw[k] + (double)A.rho * Vk[k]);
+    }
+    if (A.step) A.step[b] += 1;
+  }
+  // usage adjoint dL/dU_c(t) = w_res softmax_c(t) + c_res [U_c(t) > R_c]
+  for (int i = tid; i < A.C * Dh; i += 256) {
+    const int c = i / Dh;
+    double h = 0.0;
+    if (on_robj) h += (double)A.w_res * (double)expf((float)((U[i] - s_m[c]) / A.tau)) / s_s[c];
+    const float R = A.limit[c];
+    if (on_rv && isfinite(R) && U[i] > (double)R) h += c_res;
+    A.H[(size_t)b * A.C * Dh + i] = (float)h;
+  }
+}
+
+template <bool kAdam, bool kHist>
+__global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
+  extern __shared__ __align__(16) unsigned char smem_u[];
+  float *Hs = reinterpret_cast<float *>(smem_u);  // Dh * RB
+  const int tid = threadIdx.x, RB = A.RB, Dh = A.Dh;
+  const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
+  const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1], c = A.seg[3 * segi + 2];
+  if (kHist) {
+    for (int i = tid; i < Dh * RB; i += kThreads) {
+      const int t = i / RB, rr = i % RB, bb = g * RB + rr;
+      Hs[i] = bb < A.B ? A.H[((size_t)bb * A.C + c) * Dh + t] : 0.f;
+    }
+    __syncthreads();
+  }
+  const int r = tid % RB, b = g * RB + r, rows = kThreads / RB;
+  if (b >= A.B) return;
+  const size_t VB = (size_t)A.V * A.B;
+  const float c_dep = A.coef[b * 4 + 0], c_rec = A.coef[b * 4 + 1];
+  for (int vi = s0 + tid / RB; vi < s1; vi += rows) {
+    const int vc = A.perm[vi];
+    const size_t ci = (size_t)vc * A.B + b, gi = (size_t)vi * A.B + b;
+    const float mu = A.mu[ci], sg = A.sg[ci];
+    float Ah = 0.f, Bh = 0.f;
+    const bool ok = usable(mu, sg);
+    if (kHist && ok) {
+      // dL/dC_v(t) = w_v (H(t) - H(t+1)) for the own points (P = C(t) - C(t-1))
+      const float inv_s = 1.0f / sg, wv = A.w[vi];
+      int a, bw;
+      window(mu, sg, A.k_win, A.D, a, bw);
+      for (int t = a; t <= bw; ++t) {
+        const float z = ((float)t + 0.5f - mu) * inv_s;
+        const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
+        const float gh = wv * (Hs[fold_bin(t, A.II) * RB + r] - Hs[fold_bin(t + 1, A.II) * RB + r]);
+        Ah += gh * f;
+        Bh += gh * z * f;
+      }
+    }
+    const float Asum = c_dep * A.gpart[0 * VB + gi] + A.gpart[2 * VB + gi] + c_rec * A.gpart[4 * VB + gi] + Ah;
+    const float Bsum = c_dep * A.gpart[1 * VB + gi] + A.gpart[3 * VB + gi] + c_rec * A.gpart[5 * VB + gi] + Bh;
+    // dC/dmu = -phi/sigma, dC/dsigma = -z phi/sigma
+    const float gm = ok ? -Asum / sg : 0.f, gs = ok ? -Bsum / sg : 0.f;
+    if (!kAdam) {
+      A.grad_mu[ci] = gm;
+      A.grad_sg[ci] = gs;
+    } else {
+      const int step = A.step_dev[b];
+      const float bc1 = 1.0f - powf(A.beta1, (float)step), bc2 = 1.0f - powf(A.beta2, (float)step);
+      const float m1 = A.beta1 * A.m_mu[ci] + (1.0f - A.beta1) * gm;
+      const float v1 = A.beta2 * A.v_mu[ci] + (1.0f - A.beta2) * gm * gm;
+      const float m2 = A.beta1 * A.m_sg[ci] + (1.0f - A.beta1) * gs;
+      const float v2 = A.beta2 * A.v_sg[ci] + (1.0f - A.beta2) * gs * gs;
+      A.m_mu[ci] = m1; A.v_mu[ci] = v1; A.m_sg[ci] = m2; A.v_sg[ci] = v2;
+      const float nmu = mu - A.lr * (m1 / bc1) / (sqrtf(v1 / bc2) + A.eps);
+      const float nsg = sg - A.lr * (m2 / bc1) / (sqrtf(v2 / bc2) + A.eps);
+      A.mu[ci] = nmu;
+      A.sg[ci] = fmaxf(nsg, A.sigma_min);
+    }
+  }
+}
+
+}  // namespace gaus

@@ -1,0 +1,255 @@
+// gaus_plan.cpp -- host planner of gaus_create: validation, topological order,
+// ASAP/ALAP (App. A, Alg. 1 input), class-sorted node order and the flat arrays the
+// kernels read.  Pure C++; no CUDA calls.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <numeric>
+#include <string>
+#include <vector>
+
+#include "gaus_internal.h"
+
+namespace gaus {
+
+static gaus_status fail(std::string *err, gaus_status st, const char *msg) {
+  if (err) *err = msg;
+  return st;
+}
+
+gaus_status check_hparams(const gaus_hparams *hp, std::string *err) {
+  if (!hp) return fail(err, GAUS_EINVAL, "hparams is NULL");
+  const float pos[] = {hp->tau, hp->lr, hp->window_k, hp->sigma_min};
+  for (float x : pos)
+    if (!(x > 0.0f) || !std::isfinite(x)) return fail(err, GAUS_EINVAL, "tau, lr, window_k and sigma_min must be finite and > 0");
+  const float nonneg[] = {hp->rho, hp->alpha, hp->w_res, hp->w_mem, hp->eps, hp->lambda0};
+  for (float x : nonneg)
+    if (!(x >= 0.0f) || !std::isfinite(x)) return fail(err, GAUS_EINVAL, "rho, alpha, w_res, w_mem, eps, lambda0 must be finite and >= 0");
+  if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f && hp->beta2 >= 0.0f && hp->beta2 < 1.0f))
+    return fail(err, GAUS_EINVAL, "Adam betas must lie in [0, 1)");
+  if (hp->terms & ~63u) return fail(err, GAUS_EINVAL, "unknown term bits");
+  return GAUS_OK;
+}
+
+static bool valid_csr(int V, int E, const int32_t *ptr, const int32_t *idx) {
+  if (!ptr || (E > 0 && !idx)) return false;
+  if (ptr[0] != 0 || ptr[V] != E) return false;
+  for (int v = 0; v < V; ++v)
+    if (ptr[v + 1] < ptr[v]) return false;
+  for (int e = 0; e < E; ++e)
+    if (idx[e] < 0 || idx[e] >= V) return false;
+  return true;
+}
+
+gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err) {
+  if (!p) return fail(err, GAUS_EINVAL, "problem is NULL");
+  const int V = p->V, E = p->E, C = p->C, NB = p->n_back;
+  if (V < 1 || E < 0 || NB < 0) return fail(err, GAUS_EINVAL, "V >= 1, E >= 0, n_back >= 0 required");
+  if (C < 1 || C > kMaxClasses) return fail(err, GAUS_EINVAL, "C must lie in 1..16");
+  if (p->D < 1 || p->II < 0 || p->B < 1) return fail(err, GAUS_EINVAL, "D >= 1, II >= 0, B >= 1 required");
+  if ((int64_t)V * p->B >= (int64_t)1 << 31 || (int64_t)V * p->D >= (int64_t)1 << 31)
+    return fail(err, GAUS_EINVAL, "V * B and V * D must stay below 2^31");
+  if (p->D > 65536) return fail(err, GAUS_EINVAL, "D must be <= 65536");
+  if (!valid_csr(V, E, p->succ_ptr, p->succ_idx)) return fail(err, GAUS_EINVAL, "invalid CSR (succ_ptr/succ_idx)");
+  if (!valid_csr(V, E, p->pred_ptr, p->pred_idx)) return fail(err, GAUS_EINVAL, "invalid CSC (pred_ptr/pred_idx)");
+  if (!p->latency || !p->res_class || !p->limit) return fail(err, GAUS_EINVAL, "latency, res_class and limit are required");
+  if (NB > 0 && (!p->back_src || !p->back_dst || !p->back_dist)) return fail(err, GAUS_EINVAL, "back-edge arrays missing");
+
+  // edge list from CSR; CSC must describe the same set; no duplicates or self loops
+  std::vector<int64_t> ecsr(E), ecsc(E);
+  for (int u = 0; u < V; ++u)
+    for (int q = p->succ_ptr[u]; q < p->succ_ptr[u + 1]; ++q) {
+      if (p->succ_idx[q] == u) return fail(err, GAUS_ECYCLE, "self loop");
+      ecsr[q] = (int64_t)u * V + p->succ_idx[q];
+    }
+  for (int v = 0; v < V; ++v)
+    for (int q = p->pred_ptr[v]; q < p->pred_ptr[v + 1]; ++q) ecsc[q] = (int64_t)p->pred_idx[q] * V + v;
+  std::sort(ecsr.begin(), ecsr.end());
+  std::sort(ecsc.begin(), ecsc.end());
+  if (ecsr != ecsc) return fail(err, GAUS_EINVAL, "CSR and CSC describe different edges");
+  for (int e = 1; e < E; ++e)
+    if (ecsr[e] == ecsr[e - 1]) return fail(err, GAUS_EINVAL, "duplicate edge");
+
+  Plan &P = *out;
+  P = Plan();
+  P.V = V; P.E = E; P.NB = NB; P.C = C; P.D = p->D; P.II = p->II; P.B = p->B;
+  P.Dh = p->II > 0 ? p->II : p->D;
+  for (int v = 0; v < V; ++v) {
+    if (p->latency[v] < 0 || p->latency[v] > p->D) return fail(err, GAUS_EINVAL, "latency must lie in 0..D");
+    if (p->res_class[v] < 0 || p->res_class[v] >= C) return fail(err, GAUS_EINVAL, "res_class out of range");
+    if (p->demand && p->demand[v] < 0) return fail(err, GAUS_EINVAL, "demand must be >= 0");
+    if (p->bits && p->bits[v] < 0) return fail(err, GAUS_EINVAL, "bits must be >= 0");
+  }
+  for (int c = 0; c < C; ++c)
+    if (!(p->limit[c] >= 0.0f)) return fail(err, GAUS_EINVAL, "limit must be >= 0 or INFINITY");
+  for (int q = 0; q < NB; ++q) {
+    if (p->back_src[q] < 0 || p->back_src[q] >= V || p->back_dst[q] < 0 || p->back_dst[q] >= V)
+      return fail(err, GAUS_EINVAL, "back edge endpoint out of range");
+    if (p->back_dist[q] < 1) return fail(err, GAUS_EINVAL, "back edge distance must be >= 1");
+  }
+
+  // Kahn's algorithm and topological levels
+  std::vector<int32_t> indeg(V), order;
+  order.reserve(V);
+  for (int v = 0; v < V; ++v) indeg[v] = p->pred_ptr[v + 1] - p->pred_ptr[v];
+  for (int v = 0; v < V; ++v)
+    if (!indeg[v]) order.push_back(v);
+  P.level.assign(V, 0);
+  for (size_t h = 0; h < order.size(); ++h) {
+    int u = order[h];
+    for (int q = p->succ_ptr[u]; q < p->succ_ptr[u + 1]; ++q) {
+      int w = p->succ_idx[q];
+      P.level[w] = std::max(P.level[w], P.level[u] + 1);
+      if (--indeg[w] == 0) order.push_back(w);
+    }
+  }
+  if ((int)order.size() != V) return fail(err, GAUS_ECYCLE, "the dependency graph has a cycle");
+
+  // ASAP_v = max_u ASAP_u + Lat(u); CP = max ASAP_v + Lat(v); ALAP_v = min(D - Lat(v), min_w ALAP_w - Lat(v))
+  P.asap.assign(V, 0);
+  for (int u : order)
+    for (int q = p->succ_ptr[u]; q < p->succ_ptr[u + 1]; ++q) {
+      int w = p->succ_idx[q];
+      P.asap[w] = std::max(P.asap[w], P.asap[u] + p->latency[u]);
+    }
+  P.cp = 0;
+  for (int v = 0; v < V; ++v) P.cp = std::max(P.cp, P.asap[v] + p->latency[v]);
+  if (P.cp > p->D) return fail(err, GAUS_EHORIZON, "critical path longer than the horizon D");
+  P.alap.assign(V, 0);
+  for (int h = V - 1; h >= 0; --h) {
+    int v = order[h];
+    int a = p->D - p->latency[v];
+    for (int q = p->succ_ptr[v]; q < p->succ_ptr[v + 1]; ++q) a = std::min(a, P.alap[p->succ_idx[q]] - p->latency[v]);
+    P.alap[v] = a;
+  }
+
+  // caller-order attributes
+  P.c_lat.assign(p->latency, p->latency + V);
+  P.c_cls.assign(p->res_class, p->res_class + V);
+  P.c_dem.resize(V);
+  P.c_bits.resize(V);
+  for (int v = 0; v < V; ++v) {
+    P.c_dem[v] = p->demand ? p->demand[v] : 1;
+    P.c_bits[v] = p->bits ? p->bits[v] : 1;
+  }
+  P.limit.assign(p->limit, p->limit + C);
+  P.e_src.resize(E);
+  P.e_dst.resize(E);
+  for (int u = 0; u < V; ++u)
+    for (int q = p->succ_ptr[u]; q < p->succ_ptr[u + 1]; ++q) { P.e_src[q] = u; P.e_dst[q] = p->succ_idx[q]; }
+  P.b_src.assign(p->back_src, p->back_src + NB);
+  P.b_dst.assign(p->back_dst, p->back_dst + NB);
+  P.b_dist.assign(p->back_dist, p->back_dist + NB);
+
+  // internal order: by class, then topological level, then caller id
+  P.perm.resize(V);
+  std::iota(P.perm.begin(), P.perm.end(), 0);
+  std::stable_sort(P.perm.begin(), P.perm.end(), [&](int a, int b) {
+    if (P.c_cls[a] != P.c_cls[b]) return P.c_cls[a] < P.c_cls[b];
+    return P.level[a] < P.level[b];
+  });
+  P.inv.resize(V);
+  for (int i = 0; i < V; ++i) P.inv[P.perm[i]] = i;
+  P.w.resize(V); P.bits.resize(V); P.lat.resize(V); P.cls.resize(V);
+  for (int i = 0; i < V; ++i) {
+    int v = P.perm[i];
+    P.w[i] = (float)P.c_dem[v];
+    P.bits[i] = (float)P.c_bits[v];
+    P.lat[i] = P.c_lat[v];
+    P.cls[i] = P.c_cls[v];
+  }
+  // internal CSC / CSR (neighbours stored by caller id)
+  P.in_ptr.assign(V + 1, 0);
+  P.out_ptr.assign(V + 1, 0);
+  for (int i = 0; i < V; ++i) {
+    int v = P.perm[i];
+    P.in_ptr[i + 1] = P.in_ptr[i] + (p->pred_ptr[v + 1] - p->pred_ptr[v]);
+    P.out_ptr[i + 1] = P.out_ptr[i] + (p->succ_ptr[v + 1] - p->succ_ptr[v]);
+  }
+  P.in_src.resize(E); P.in_lat.resize(E); P.out_dst.resize(E);
+  for (int i = 0; i < V; ++i) {
+    int v = P.perm[i];
+    int o = P.in_ptr[i];
+    for (int q = p->pred_ptr[v]; q < p->pred_ptr[v + 1]; ++q, ++o) {
+      P.in_src[o] = p->pred_idx[q];
+      P.in_lat[o] = p->latency[p->pred_idx[q]];
+    }
+    o = P.out_ptr[i];
+    for (int q = p->succ_ptr[v]; q < p->succ_ptr[v + 1]; ++q, ++o) P.out_dst[o] = p->succ_idx[q];
+  }
+  // back edges: shift = Lat(j) - k II (a back edge acts as a dependency with that latency)
+  P.bin_ptr.assign(V + 1, 0);
+  P.bout_ptr.assign(V + 1, 0);
+  for (int q = 0; q < NB; ++q) {
+    P.bin_ptr[P.inv[p->back_dst[q]] + 1]++;
+    P.bout_ptr[P.inv[p->back_src[q]] + 1]++;
+  }
+  for (int i = 0; i < V; ++i) { P.bin_ptr[i + 1] += P.bin_ptr[i]; P.bout_ptr[i + 1] += P.bout_ptr[i]; }
+  P.bin_src.resize(NB); P.bin_shift.resize(NB); P.bout_dst.resize(NB); P.bout_shift.resize(NB);
+  {
+    std::vector<int32_t> fi(P.bin_ptr.begin(), P.bin_ptr.end() - 1), fo(P.bout_ptr.begin(), P.bout_ptr.end() - 1);
+    for (int q = 0; q < NB; ++q) {
+      int j = p->back_src[q], i = p->back_dst[q];
+      int shift = p->latency[j] - p->back_dist[q] * p->II;
+      int a = fi[P.inv[i]]++;
+      P.bin_src[a] = j; P.bin_shift[a] = shift;
+      int b = fo[P.inv[j]]++;
+      P.bout_dst[b] = i; P.bout_shift[b] = shift;
+    }
+  }
+  // caller-order CSC / CSR / back edges for the integer kernels
+  P.cpred_ptr.assign(p->pred_ptr, p->pred_ptr + V + 1);
+  P.cpred_src.assign(p->pred_idx, p->pred_idx + E);
+  P.csucc_ptr.assign(p->succ_ptr, p->succ_ptr + V + 1);
+  P.csucc_dst.assign(p->succ_idx, p->succ_idx + E);
+  P.cback_ptr.assign(V + 1, 0);
+  for (int q = 0; q < NB; ++q) P.cback_ptr[p->back_dst[q] + 1]++;
+  for (int v = 0; v < V; ++v) P.cback_ptr[v + 1] += P.cback_ptr[v];
+  P.cback_src.resize(NB); P.cback_shift.resize(NB);
+  {
+    std::vector<int32_t> f(P.cback_ptr.begin(), P.cback_ptr.end() - 1);
+    for (int q = 0; q < NB; ++q) {
+      int a = f[p->back_dst[q]]++;
+      P.cback_src[a] = p->back_src[q];
+      P.cback_shift[a] = p->latency[p->back_src[q]] - p->back_dist[q] * p->II;
+    }
+  }
+  // nodes by topological level (caller ids)
+  P.nlvl = 0;
+  for (int v = 0; v < V; ++v) P.nlvl = std::max(P.nlvl, P.level[v] + 1);
+  P.lvl_ptr.assign(P.nlvl + 1, 0);
+  for (int v = 0; v < V; ++v) P.lvl_ptr[P.level[v] + 1]++;
+  for (int l = 0; l < P.nlvl; ++l) P.lvl_ptr[l + 1] += P.lvl_ptr[l];
+  P.lvl_nodes.resize(V);
+  {
+    std::vector<int32_t> f(P.lvl_ptr.begin(), P.lvl_ptr.end() - 1);
+    for (int v = 0; v < V; ++v) P.lvl_nodes[f[P.level[v]]++] = v;
+  }
+
+  // segments: contiguous internal nodes of one class, sized so that the per-node
+  // kernels launch about target_blocks blocks over all restart groups
+  int RB = 1;
+  while (RB < p->B && RB < 32) RB <<= 1;
+  int G = (p->B + RB - 1) / RB;
+  long want = std::max(1L, (long)target_blocks / G);
+  int seglen = (int)std::max(1L, ((long)V + want - 1) / want);
+  // keep a segment to a handful of rows per thread at least
+  seglen = std::max(seglen, std::max(1, kThreads / RB));
+  P.cls_seg_ptr.assign(C + 1, 0);
+  int i0 = 0;
+  for (int c = 0; c < C; ++c) {
+    int i1 = i0;
+    while (i1 < V && P.cls[i1] == c) ++i1;
+    for (int s = i0; s < i1; s += seglen) {
+      P.seg.push_back(s);
+      P.seg.push_back(std::min(i1, s + seglen));
+      P.seg.push_back(c);
+    }
+    P.cls_seg_ptr[c + 1] = (int)P.seg.size() / 3;
+    i0 = i1;
+  }
+  P.nseg = (int)P.seg.size() / 3;
+  return GAUS_OK;
+}
+
+}  // namespace gaus

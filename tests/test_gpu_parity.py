@@ -1,0 +1,205 @@
+"""GPU path (through the C ABI) against the fp64 oracle on the same seeded inputs.
+
+Tolerances (the fp32 reading of "within 1e-4 relative"):
+  * loss and every term value, per restart: |d| <= 1e-4 |ref| + 1e-5;
+  * gradients, per restart: max|d| <= 1e-4 max|ref| (+ 1e-7), and every
+    component with |ref| >= 1e-2 max|ref| within 1e-4 |ref| (+ 1e-7);
+  * schedules, legalization status and verifier reports: bit-exact.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def g():
+    import paper_2602_20427_gb300 as g
+    g.build()
+    g.lib()
+    return g
+
+
+def _ohp(hp, terms):
+    return oracle.hparams(tau=hp.tau, rho=hp.rho, alpha=hp.alpha, w_res=hp.w_res, w_mem=hp.w_mem,
+                          terms=terms)
+
+
+def check_loss_grad(p, g, B, mu, sg, lam, hp, restarts=None, rtol=1e-4):
+    """Run gaus_loss_grad on all B restarts; compare the listed restarts with the oracle."""
+    ctx = g.Gaus(p, B, hp)
+    dmu, dsg = torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda()
+    dlam = torch.from_numpy(lam.astype(np.float32)).cuda()
+    out = ctx.loss_grad(dmu, dsg, dlam)
+    torch.cuda.synchronize()
+    ctx.close()
+    rs = list(range(B)) if restarts is None else list(restarts)
+    op = oracle.OracleProblem(p)
+    loss, terms, gm, gs = oracle.loss_grad(op, _ohp(hp, hp.terms), mu[:, rs].astype(np.float64),
+                                           sg[:, rs].astype(np.float64), lam[rs].astype(np.float64))
+    o_loss = out["loss"].cpu().numpy()[rs]
+    o_terms = out["terms"].cpu().numpy()[rs]
+    o_gm = out["grad_mu"].cpu().numpy()[:, rs]
+    o_gs = out["grad_sigma"].cpu().numpy()[:, rs]
+    assert np.all(out["status"].cpu().numpy() == 0)
+    np.testing.assert_allclose(o_loss, loss, rtol=rtol, atol=1e-5)
+    np.testing.assert_allclose(o_terms, terms, rtol=rtol, atol=1e-5)
+    for ref, got in ((gm, o_gm), (gs, o_gs)):
+        for k in range(len(rs)):
+            r, x = ref[:, k], got[:, k]
+            scale = np.max(np.abs(r))
+            err = np.abs(x - r)
+            assert np.max(err) <= rtol * scale + 1e-7, (k, np.max(err), scale)
+            big = np.abs(r) >= 1e-2 * scale
+            assert np.all(err[big] <= rtol * np.abs(r[big]) + 1e-7), (k, np.max(err[big] / np.abs(r[big])))
+    return out
+
+
+def _lam(B, rng):
+    return rng.uniform(0.0, 2.0, size=(B, 3)).astype(np.float32)
+
+
+@pytest.mark.parametrize("B", [1, 4])
+def test_tiny_layered(g, B):
+    p = W.tiny_layered(1)
+    mu, sg = W.init_state(p, B, 1, mu_jitter="uniform01", sigma0=1.0)
+    hp = g.default_hparams(terms=p.terms, tau=0.05, rho=0.01)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, np.random.default_rng(0)), hp)
+
+
+def test_random_layered_b64(g):
+    p = W.random_layered(1)
+    mu, sg = W.init_state(p, 64, 2)
+    hp = g.default_hparams(terms=p.terms)
+    check_loss_grad(p, g, 64, mu, sg, _lam(64, np.random.default_rng(1)), hp, restarts=range(0, 64, 9))
+
+
+def test_logic_small_all_terms(g):
+    p = W.logic_network(2, V=2000, depth=40)
+    mu, sg = W.init_state(p, 32, 3)
+    hp = g.default_hparams(terms=p.terms, alpha=0.7, w_res=1.3, rho=1e-3)
+    check_loss_grad(p, g, 32, mu, sg, _lam(32, np.random.default_rng(2)), hp, restarts=range(0, 32, 5))
+
+
+def test_modulo_with_recurrences(g):
+    p = W.modulo_loop(3, V=400, levels=20, n_back=20)
+    terms = W.DEP | W.RES_OBJ | W.RES_VIOL | W.REC
+    p.terms = terms
+    mu, sg = W.init_state(p, 8, 4)
+    hp = g.default_hparams(terms=terms, rho=1e-3)
+    check_loss_grad(p, g, 8, mu, sg, _lam(8, np.random.default_rng(3)), hp)
+
+
+@pytest.mark.parametrize("B", [3, 40])
+def test_ragged_restart_counts(g, B):
+    p = W.random_layered(5)
+    p.terms = W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL
+    mu, sg = W.init_state(p, B, 5)
+    hp = g.default_hparams(terms=p.terms)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, np.random.default_rng(4)), hp,
+                    restarts=sorted({0, B // 2, B - 1}))
+
+
+def test_edge_cases_windows_and_bounds(g):
+    # mu far outside [0, D), sigma at sigma_min, windows longer than the 32-point
+    # cache, zero-latency (chaining) edges, an unlimited class, a high fan-out node
+    rng = np.random.default_rng(9)
+    V = 80
+    src, dst = [], []
+    for v in range(1, 65):            # node 0 feeds 64 consumers
+        src.append(0); dst.append(v)
+    for v in range(65, V):
+        for u in rng.choice(v, size=2, replace=False):
+            src.append(int(u)); dst.append(v)
+    lat = rng.integers(0, 3, size=V)
+    lat[0] = 0
+    p = W._finish("edge_cases", V, src, dst, lat, rng.integers(0, 3, size=V), 3, [4.0, np.inf, 2.0], rng,
+                  D=120, demand=rng.integers(1, 3, size=V), bits=np.ones(V),
+                  terms=W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL)
+    B = 8
+    mu = (p.start[:, None] + rng.normal(0, 3, size=(V, B))).astype(np.float32)
+    sg = rng.uniform(0.3, 2.0, size=(V, B)).astype(np.float32)
+    mu[3, 0], mu[4, 1], mu[5, 2] = -50.0, 170.0, 119.49999
+    sg[6, :] = 0.05
+    sg[7:12, 3] = 9.0                 # windows of ~109 points
+    sg[0, 4] = 12.0
+    hp = g.default_hparams(terms=p.terms, tau=0.1, rho=0.01)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, rng), hp)
+
+
+def test_single_bin_horizon(g):
+    p = W.random_small(3, V=6, D=1, p_edge=0.4, max_lat=0)
+    p.terms = W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL
+    mu = np.random.default_rng(1).normal(0, 1, size=(6, 2)).astype(np.float32)
+    sg = np.full((6, 2), 1.0, np.float32)
+    hp = g.default_hparams(terms=p.terms, tau=0.2)
+    check_loss_grad(p, g, 2, mu, sg, _lam(2, np.random.default_rng(1)), hp)
+
+
+def test_fold_with_ii_equal_to_d(g):
+    p = W.modulo_loop(4, V=300, levels=15, n_back=10)
+    p.D = p.II = max(p.cp, p.II)
+    p.terms = W.DEP | W.RES_OBJ | W.RES_VIOL | W.REC
+    mu, sg = W.init_state(p, 4, 6)
+    hp = g.default_hparams(terms=p.terms, rho=1e-3)
+    check_loss_grad(p, g, 4, mu, sg, _lam(4, np.random.default_rng(6)), hp)
+
+
+def test_logic_network_full_size_sampled(g):
+    # the headline workload at its full size, in the launch configuration the
+    # benchmark uses (V = 10,000, B = 64); the oracle checks two restarts
+    p = W.logic_network(1)
+    mu, sg = W.init_state(p, 64, 1)
+    hp = g.default_hparams(terms=p.terms)
+    lam = np.full((64, 3), 1e-6, np.float32)
+    check_loss_grad(p, g, 64, mu, sg, lam, hp, restarts=[0, 37])
+
+
+def test_nonfinite_restart_is_isolated(g):
+    p = W.random_layered(2)
+    B = 8
+    mu, sg = W.init_state(p, B, 8)
+    hp = g.default_hparams(terms=p.terms)
+    lam = torch.full((B, 3), 1e-6, device="cuda")
+    ctx = g.Gaus(p, B, hp)
+    clean = ctx.loss_grad(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), lam)
+    clean = {k: v.clone() for k, v in clean.items()}
+    mu2, sg2 = mu.copy(), sg.copy()
+    mu2[10, 2] = np.nan
+    sg2[20, 5] = -1.0
+    out = ctx.loss_grad(torch.from_numpy(mu2).cuda(), torch.from_numpy(sg2).cuda(), lam)
+    torch.cuda.synchronize()
+    st = out["status"].cpu().numpy()
+    assert st[2] == 6 and st[5] == 6 and np.all(np.delete(st, [2, 5]) == 0)
+    keep = [b for b in range(B) if b not in (2, 5)]
+    for k in ("loss", "grad_mu", "grad_sigma"):
+        a, c = out[k].cpu().numpy(), clean[k].cpu().numpy()
+        if a.ndim == 1:
+            np.testing.assert_array_equal(a[keep], c[keep])
+        else:
+            np.testing.assert_array_equal(a[:, keep], c[:, keep])
+    # a later clean call on the same context reports OK again
+    out = ctx.loss_grad(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), lam)
+    torch.cuda.synchronize()
+    assert np.all(out["status"].cpu().numpy() == 0)
+    ctx.close()
+
+
+def test_run_to_run_determinism(g):
+    p = W.logic_network(3, V=3000, depth=50)
+    B = 32
+    mu, sg = W.init_state(p, B, 9)
+    hp = g.default_hparams(terms=p.terms)
+    lam = torch.full((B, 3), 1e-6, device="cuda")
+    ctx = g.Gaus(p, B, hp)
+    a = {k: v.clone() for k, v in ctx.loss_grad(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), lam).items()}
+    b = ctx.loss_grad(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), lam)
+    torch.cuda.synchronize()
+    for k in a:
+        assert torch.equal(a[k], b[k]), k
+    ctx.close()
