@@ -61,6 +61,7 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   IterArgs A;
   A.mu = mu; A.sg = sg;
   A.V = P.V; A.B = P.B; A.D = P.D; A.II = P.II; A.Dh = P.Dh; A.C = P.C; A.RB = ctx->RB; A.G = ctx->G;
+  A.kc = ctx->kc;
   A.k_win = ctx->hp.window_k; A.alpha = ctx->hp.alpha;
   A.perm = ctx->d_perm; A.w = ctx->d_w; A.lat = ctx->d_lat;
   A.in_ptr = ctx->d_in_ptr; A.in_src = ctx->d_in_src; A.in_lat = ctx->d_in_lat;
@@ -97,12 +98,17 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   const unsigned on = ctx->hp.terms;
   IterArgs A = iter_args(ctx, mu, sg);
   FwdKernel kf = pick_fwd(on, P.II);
-  kf<<<ctx->nblk, kThreads, ctx->smem_fwd, st>>>(A);
+  kf<<<ctx->nblk, kFwdThreads, ctx->smem_fwd, st>>>(A);
   CK(cudaGetLastError(), "k_fwd launch");
+  RedArgs R;
+  R.B = P.B; R.C = P.C; R.Dh = P.Dh; R.RB = ctx->RB; R.G = ctx->G;
+  R.cls_seg_ptr = ctx->d_cls_seg_ptr; R.hpart = ctx->d_hpart; R.hspan = ctx->d_hspan; R.U = ctx->d_U;
+  k_reduce<<<ctx->red_blocks, 256, 0, st>>>(R);
+  CK(cudaGetLastError(), "k_reduce launch");
   if (ev) CK(cudaEventRecord(ev[1], st), "event");
 
   FinArgs F;
-  F.B = P.B; F.C = P.C; F.Dh = P.Dh; F.RB = ctx->RB; F.G = ctx->G;
+  F.B = P.B; F.C = P.C; F.Dh = P.Dh; F.RB = ctx->RB; F.G = ctx->G; F.Ug = ctx->d_U;
   F.terms = on; F.tau = ctx->hp.tau; F.rho = ctx->hp.rho; F.alpha = ctx->hp.alpha;
   F.w_res = ctx->hp.w_res; F.w_mem = ctx->hp.w_mem;
   F.cls_seg_ptr = ctx->d_cls_seg_ptr; F.limit = ctx->d_limit;
@@ -161,7 +167,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   const bool have_dev = cudaGetDevice(&dev) == cudaSuccess &&
                         cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess;
   std::string err;
-  gaus_status st = plan_problem(prob, 4 * nsm, &ctx->plan, &err);
+  gaus_status st = plan_problem(prob, 8 * nsm, &ctx->plan, &err);
   if (st != GAUS_OK) { ctx->err = err; return st; }
   Plan &P = ctx->plan;
   if ((ctx->hp.terms & GAUS_REC) && P.II <= 0) { ctx->err = "GAUS_REC needs II > 0"; return GAUS_EINVAL; }
@@ -175,13 +181,28 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   while (ctx->RB < P.B && ctx->RB < 32) ctx->RB <<= 1;
   ctx->G = (P.B + ctx->RB - 1) / ctx->RB;
   ctx->nblk = P.nseg * ctx->G;
-  ctx->smem_fwd = (size_t)ctx->RB * P.Dh * sizeof(long long) + 3 * (size_t)kCache * kThreads * sizeof(float);
+  {
+    const int per = 256 / ctx->RB;
+    ctx->red_blocks = ctx->G * P.C * ((P.Dh + per - 1) / per);
+  }
+  // k_fwd shared memory: the two histogram halves plus the own-window cache,
+  // sized for two resident blocks per SM when the histogram allows it.
+  const size_t hist = 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned);
+  const size_t per_pt = 3 * (size_t)kFwdThreads * sizeof(float);
+  const size_t budget2 = kMaxSmem / 2 - 1024, budget1 = kMaxSmem - 1024;
+  int kc = 0;
+  if (hist + 16 * per_pt <= budget2) kc = (int)std::min<size_t>(kCacheMax, (budget2 - hist) / per_pt);
+  else if (hist + 4 * per_pt <= budget1) kc = (int)std::min<size_t>(kCacheMax, (budget1 - hist) / per_pt);
+  if (kc < 4) {
+    ctx->err = "usage histogram of this horizon/II does not fit in shared memory";
+    return GAUS_EINVAL;
+  }
+  ctx->kc = kc;
+  ctx->smem_fwd = hist + (size_t)kc * per_pt;
   ctx->smem_upd = (size_t)ctx->RB * P.Dh * sizeof(float);
   ctx->smem_fin = (size_t)P.C * P.Dh * sizeof(double);
   ctx->smem_ver = ((size_t)P.C * P.Dh + (P.D + 1) + P.Dh) * sizeof(long long);
-  const size_t static_fwd = 3 * kThreads * sizeof(double) + 64;
-  if (ctx->smem_fwd + static_fwd > kMaxSmem || ctx->smem_upd > kMaxSmem || ctx->smem_fin > kMaxSmem ||
-      ctx->smem_ver > kMaxSmem) {
+  if (ctx->smem_upd > kMaxSmem || ctx->smem_fin > kMaxSmem || ctx->smem_ver > kMaxSmem) {
     ctx->err = "histogram of this horizon/II does not fit in shared memory";
     return GAUS_EINVAL;
   }
@@ -229,6 +250,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
 
   const size_t VB = (size_t)P.V * P.B;
   TRY(scratch(ctx, &ctx->d_hpart, (size_t)ctx->nblk * ctx->RB * P.Dh));
+  TRY(scratch(ctx, &ctx->d_U, (size_t)P.B * P.C * P.Dh));
   TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
   TRY(scratch(ctx, &ctx->d_fwd, (size_t)ctx->nblk * ctx->RB * 3));
   TRY(scratch(ctx, &ctx->d_gpart, 6 * VB));

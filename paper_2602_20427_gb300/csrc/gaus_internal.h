@@ -11,10 +11,11 @@
 
 namespace gaus {
 
-// Threads per block of the per-(node, restart) kernels.
+// Threads per block of the node/edge pass and of the update kernel.
+constexpr int kFwdThreads = 256;
 constexpr int kThreads = 128;
-// Own-window points cached in shared memory per thread (longer windows recompute).
-constexpr int kCache = 32;
+// Most own-window points cached in shared memory per thread (longer windows recompute).
+constexpr int kCacheMax = 32;
 // Fixed-point scale of the usage histograms: P * 2^32 accumulated in int64.
 constexpr float kFix = 4294967296.0f;
 constexpr double kInvFix = 1.0 / 4294967296.0;
@@ -68,6 +69,8 @@ struct gaus_ctx {
   cudaStream_t stream = nullptr;
   std::string err;
   int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per pass
+  int kc = 0;                    // own-window points cached per thread in k_fwd
+  int red_blocks = 0;
   size_t smem_fwd = 0, smem_upd = 0, smem_fin = 0, smem_ver = 0;
   // device graph
   int32_t *d_perm = nullptr;
@@ -87,9 +90,10 @@ struct gaus_ctx {
   int32_t *d_b_src = nullptr, *d_b_dst = nullptr, *d_b_dist = nullptr;
   int32_t *d_asap = nullptr, *d_alap = nullptr;
   // scratch
-  long long *d_hpart = nullptr;  // nblk * RB * Dh fixed-point usage partials
+  long long *d_hpart = nullptr;  // nblk * Dh * RB fixed-point usage partials
   int2 *d_hspan = nullptr;       // nblk folded bin span written by each block
   double *d_fwd = nullptr;       // nblk * RB * 3 forward sums (dep, com, rec)
+  double *d_U = nullptr;         // B * C * Dh usage (k_reduce)
   float *d_gpart = nullptr;      // 6 * V * B partial gradient sums (internal index)
   float *d_H = nullptr;          // B * C * Dh usage adjoint dL/dU
   float *d_coef = nullptr;       // B * 4 (c_dep, c_rec)

@@ -27,7 +27,7 @@ namespace gaus {
 
 struct IterArgs {
   const float *mu, *sg;  // (V, B) caller order
-  int V, B, D, II, Dh, C, RB, G;
+  int V, B, D, II, Dh, C, RB, G, kc;
   float k_win, alpha;
   const int32_t *perm;
   const float *w;
@@ -44,8 +44,17 @@ struct IterArgs {
   int32_t *nonfinite;
 };
 
+struct RedArgs {
+  int B, C, Dh, RB, G;
+  const int32_t *cls_seg_ptr;
+  const long long *hpart;
+  const int2 *hspan;
+  double *U;
+};
+
 struct FinArgs {
   int B, C, Dh, RB, G;
+  const double *Ug;   // (B, C, Dh) usage from k_reduce
   unsigned terms;
   float tau, rho, alpha, w_res, w_mem;
   const int32_t *cls_seg_ptr;
@@ -103,80 +112,102 @@ constexpr float kInvSqrt2Pi = 0.3989422804014327f;
 constexpr float kInvSqrt2 = 0.7071067811865476f;
 
 template <bool kDep, bool kCom, bool kRec>
-__global__ void __launch_bounds__(kThreads) k_fwd(const IterArgs A) {
+__global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
+  // Shared memory: usage histogram as two u32 halves [bin][restart] (conflict-free
+  // for any bins the lanes of a warp touch), then the own-window cache.
   extern __shared__ __align__(16) unsigned char smem[];
-  const int tid = threadIdx.x, RB = A.RB, Dh = A.Dh;
-  long long *hist = reinterpret_cast<long long *>(smem);
-  float *cC = reinterpret_cast<float *>(hist + (size_t)RB * Dh);
-  float *cF = cC + kCache * kThreads;
-  float *cZ = cF + kCache * kThreads;
+  constexpr int T = kFwdThreads;
+  const int tid = threadIdx.x, RB = A.RB, Dh = A.Dh, kc = A.kc;
+  unsigned *hlo = reinterpret_cast<unsigned *>(smem);
+  unsigned *hhi = hlo + (size_t)Dh * RB;
+  float *cC = reinterpret_cast<float *>(hhi + (size_t)Dh * RB);
+  float *cF = cC + (size_t)kc * T;
+  float *cZ = cF + (size_t)kc * T;
   __shared__ int s_lo, s_hi;
-  __shared__ double s_red[3][kThreads];
 
   const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
   const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1];
-  for (int i = tid; i < RB * Dh; i += kThreads) hist[i] = 0;
+  for (int i = tid; i < 2 * RB * Dh; i += T) hlo[i] = 0u;
   if (tid == 0) { s_lo = INT_MAX; s_hi = INT_MIN; }
   __syncthreads();
 
-  const int r = tid % RB, b = g * RB + r, rows = kThreads / RB;
+  const int r = tid % RB, b = g * RB + r, rows = T / RB;
   const bool bok = b < A.B;
   const size_t VB = (size_t)A.V * A.B;
+  constexpr unsigned FULL = 0xffffffffu;
   float fdep = 0.f, fcom = 0.f, frec = 0.f;
   int lo = INT_MAX, hi = INT_MIN;
+  // Control flow is kept warp-uniform: every lane runs the same item count and
+  // every loop runs to the warp's maximum trip count with a per-lane predicate,
+  // so the warp never splits around the shared-memory atomics.
+  const int n_items = (s1 - s0 + rows - 1) / rows;
 
-  for (int vi = s0 + tid / RB; vi < s1; vi += rows) {
-    if (!bok) continue;
-    const int vc = A.perm[vi];
-    const size_t gi = (size_t)vi * A.B + b;
-    const float mu = A.mu[(size_t)vc * A.B + b], sg = A.sg[(size_t)vc * A.B + b];
-    if (!usable(mu, sg)) {
+  for (int it = 0; it < n_items; ++it) {
+    const int vi = s0 + tid / RB + it * rows;
+    bool valid = bok && vi < s1;
+    const int vcl = valid ? vi : s0;
+    const int vc = A.perm[vcl];
+    const size_t gi = (size_t)vcl * A.B + (bok ? b : 0);
+    const float mu = valid ? A.mu[(size_t)vc * A.B + b] : 0.f;
+    const float sg = valid ? A.sg[(size_t)vc * A.B + b] : 1.f;
+    if (valid && !usable(mu, sg)) {
       A.nonfinite[b] = 1;
       for (int k = 0; k < 6; ++k) A.gpart[k * VB + gi] = 0.f;
-      continue;
+      valid = false;
     }
-    const float inv_s = 1.0f / sg, wv = A.w[vi];
-    int a, bw;
-    window(mu, sg, A.k_win, A.D, a, bw);
-    const int n = bw - a + 1;
+    const float inv_s = valid ? 1.0f / sg : 1.0f, wv = A.w[vcl];
+    int a = 0, bw = -2;
+    if (valid) window(mu, sg, A.k_win, A.D, a, bw);
+    const int n = bw - a + 1;                      // points; -1 for an idle lane
+    const int nmax = __reduce_max_sync(FULL, n);
 
     // ---- own points: cache C, phi, z*phi; bin masses into the usage histogram ----
     // P(d) for d in [a, b+1] from Q(|z|) = Phi(-|z|) so that both tails keep
-    // relative accuracy: C = Q when z <= 0, 1 - Q otherwise.
+    // relative accuracy: C = Q when z <= 0, 1 - Q otherwise.  Each mass enters
+    // the histogram as round(w P 2^32), split into 16-bit halves (exact sums).
     float zp = 0.f, qp = 0.f;
-    for (int j = 0; j <= n; ++j) {
-      float zc = 0.f, qc = 0.f, P;
-      if (j < n) {
-        zc = ((float)(a + j) + 0.5f - mu) * inv_s;
-        qc = 0.5f * erfcf(fabsf(zc) * kInvSqrt2);
-        if (j < kCache) {
-          const float f = kInvSqrt2Pi * expf(-0.5f * zc * zc);
-          cC[j * kThreads + tid] = zc <= 0.f ? qc : 1.0f - qc;
-          cF[j * kThreads + tid] = f;
-          cZ[j * kThreads + tid] = zc * f;
-        }
+    for (int j = 0; j <= nmax; ++j) {
+      const bool pt = j < n;                       // point a+j exists
+      const float zc = ((float)(a + j) + 0.5f - mu) * inv_s;
+      const float qc = pt ? 0.5f * erfcf(fabsf(zc) * kInvSqrt2) : 0.f;
+      if (pt && j < kc) {
+        const float f = kInvSqrt2Pi * expf(-0.5f * zc * zc);
+        cC[j * T + tid] = zc <= 0.f ? qc : 1.0f - qc;
+        cF[j * T + tid] = f;
+        cZ[j * T + tid] = zc * f;
       }
-      if (n == 0) P = 1.0f;
-      else if (j == 0) P = zc <= 0.f ? qc : 1.0f - qc;
-      else if (j == n) P = zp <= 0.f ? 1.0f - qp : qp;
-      else if (zc <= 0.f) P = qc - qp;
-      else if (zp > 0.f) P = qp - qc;
-      else P = (0.5f - qc) + (0.5f - qp);
-      const long long q = __float2ll_rn(wv * P * kFix);
-      atomicAdd(reinterpret_cast<unsigned long long *>(&hist[r * Dh + fold_bin(a + j, A.II)]),
-                (unsigned long long)q);
+      // branch-free selection of the bin-mass formula
+      const float c_cur = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;       // C(a+j), 1 past the window
+      const float c_prev = j == 0 ? 0.0f : (zp <= 0.f ? qp : 1.0f - qp);  // C(a+j-1)
+      float P = c_cur - c_prev;
+      P = (pt && j > 0 && zc <= 0.f) ? qc - qp : P;
+      P = (pt && j > 0 && zp > 0.f) ? qp - qc : P;
+      P = (pt && j > 0 && zp <= 0.f && zc > 0.f) ? (0.5f - qc) + (0.5f - qp) : P;
+      P = (!pt && j > 0 && zp > 0.f) ? qp : P;     // top bin: upper tail Q directly
+      if (j <= n) {
+        // round(x 2^32) = hi 2^16 + lo with hi = floor(x 2^16) and lo = round(frac 2^16),
+        // using 32-bit conversions only (64-bit ones run at the FP64 rate)
+        const float xs = fmaxf(wv * P, 0.0f) * 65536.0f;
+        const float fh = floorf(xs);
+        const int cell = fold_bin(a + j, A.II) * RB + r;
+        atomicAdd(&hlo[cell], __float2uint_rn((xs - fh) * 65536.0f));
+        atomicAdd(&hhi[cell], (unsigned)fh);
+      }
       zp = zc;
       qp = qc;
     }
-    lo = min(lo, a);
-    hi = max(hi, bw + 1);
+    __syncwarp();
+    if (valid) {
+      lo = min(lo, a);
+      hi = max(hi, bw + 1);
+    }
 
     // own point j: C, phi, z*phi (recomputed beyond the cache)
     auto own = [&](int j, float &C, float &f, float &zf) {
-      if (j < kCache) {
-        C = cC[j * kThreads + tid];
-        f = cF[j * kThreads + tid];
-        zf = cZ[j * kThreads + tid];
+      if (j < kc) {
+        C = cC[j * T + tid];
+        f = cF[j * T + tid];
+        zf = cZ[j * T + tid];
       } else {
         const float z = ((float)(a + j) + 0.5f - mu) * inv_s;
         const float q = 0.5f * erfcf(fabsf(z) * kInvSqrt2);
@@ -192,132 +223,176 @@ __global__ void __launch_bounds__(kThreads) k_fwd(const IterArgs A) {
     // dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
     // dL_com,e/dC_v(t) = -C_u(t)
     if (kDep || kCom) {
-      for (int e = A.in_ptr[vi]; e < A.in_ptr[vi + 1]; ++e) {
-        const int uc = A.in_src[e], L = A.in_lat[e];
-        const float mu_u = A.mu[(size_t)uc * A.B + b], sg_u = A.sg[(size_t)uc * A.B + b];
-        if (!usable(mu_u, sg_u)) continue;
-        const float inv_u = 1.0f / sg_u;
-        int au, bu;
-        window(mu_u, sg_u, A.k_win, A.D, au, bu);
+      const int e0 = A.in_ptr[vcl], deg = valid ? A.in_ptr[vcl + 1] - e0 : 0;
+      const int dmax = __reduce_max_sync(FULL, deg);
+      for (int q = 0; q < dmax; ++q) {
+        const bool eon = q < deg;
+        const int uc = eon ? A.in_src[e0 + q] : 0, L = eon ? A.in_lat[e0 + q] : 0;
+        const float mu_u = eon ? A.mu[(size_t)uc * A.B + b] : 0.f;
+        const float sg_u = eon ? A.sg[(size_t)uc * A.B + b] : 1.f;
+        const bool ok = eon && usable(mu_u, sg_u);
+        const float inv_u = ok ? 1.0f / sg_u : 1.0f;
+        int au = 0, bu = -1;
+        if (ok) window(mu_u, sg_u, A.k_win, A.D, au, bu);
+        const int m = ok ? n : 0;
+        const int mmax = __reduce_max_sync(FULL, m);
         float c_lo = cdf_at(a - L, mu_u, inv_u, au, bu);
-        for (int j = 0; j < n; ++j) {
-          const int t = a + j;
-          const float c_hi = cdf_at(t + 1 - L, mu_u, inv_u, au, bu);
-          const float p = c_hi - c_lo;
-          float Cv, f, zf;
-          own(j, Cv, f, zf);
-          if (kDep) {
-            fdep += Cv * p;
-            Ad += p * f;
-            Bd += p * zf;
+        for (int j = 0; j < mmax; ++j) {
+          if (j < m) {
+            const int t = a + j;
+            const float c_hi = cdf_at(t + 1 - L, mu_u, inv_u, au, bu);
+            const float p = c_hi - c_lo;
+            float Cv, f, zf;
+            own(j, Cv, f, zf);
+            if (kDep) {
+              fdep += Cv * p;
+              Ad += p * f;
+              Bd += p * zf;
+            }
+            if (kCom) {
+              const float cu = (L == 1) ? c_hi : cdf_at(t, mu_u, inv_u, au, bu);
+              fcom += cu * (1.0f - Cv);
+              Ao -= A.alpha * cu * f;
+              Bo -= A.alpha * cu * zf;
+            }
+            c_lo = c_hi;
           }
-          if (kCom) {
-            const float cu = (L == 1) ? c_hi : cdf_at(t, mu_u, inv_u, au, bu);
-            fcom += cu * (1.0f - Cv);
-            Ao -= A.alpha * cu * f;
-            Bo -= A.alpha * cu * zf;
-          }
-          c_lo = c_hi;
         }
-        if (kDep) fdep += 1.0f - c_lo;
+        __syncwarp();
+        if (kDep && ok) fdep += 1.0f - c_lo;
       }
     }
     // ---- out-edges v -> w (own = producer), latency L = Lat(v) ----
     // dV_e/dC_v(x) = -P_w(x + L);  dL_com,e/dC_v(x) = 1 - C_w(x)
     // L_com,e part = sum_{x in own, x < a_w} C_v(x) + max(0, a_w - 1 - b_v)
     if (kDep || kCom) {
-      const int L = A.lat[vi];
-      for (int e = A.out_ptr[vi]; e < A.out_ptr[vi + 1]; ++e) {
-        const int wc = A.out_dst[e];
-        const float mu_w = A.mu[(size_t)wc * A.B + b], sg_w = A.sg[(size_t)wc * A.B + b];
-        if (!usable(mu_w, sg_w)) continue;
-        const float inv_w = 1.0f / sg_w;
-        int aw, bw2;
-        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
+      const int L = A.lat[vcl];
+      const int e0 = A.out_ptr[vcl], deg = valid ? A.out_ptr[vcl + 1] - e0 : 0;
+      const int dmax = __reduce_max_sync(FULL, deg);
+      for (int q = 0; q < dmax; ++q) {
+        const bool eon = q < deg;
+        const int wc = eon ? A.out_dst[e0 + q] : 0;
+        const float mu_w = eon ? A.mu[(size_t)wc * A.B + b] : 0.f;
+        const float sg_w = eon ? A.sg[(size_t)wc * A.B + b] : 1.f;
+        const bool ok = eon && usable(mu_w, sg_w);
+        const float inv_w = ok ? 1.0f / sg_w : 1.0f;
+        int aw = 0, bw2 = -1;
+        if (ok) window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
+        const int m = ok ? n : 0;
+        const int mmax = __reduce_max_sync(FULL, m);
         float c_lo = cdf_at(a + L - 1, mu_w, inv_w, aw, bw2);
-        for (int j = 0; j < n; ++j) {
-          const int x = a + j;
-          const float c_hi = cdf_at(x + L, mu_w, inv_w, aw, bw2);
-          float Cv, f, zf;
-          own(j, Cv, f, zf);
-          if (kDep) {
-            const float p = c_hi - c_lo;
-            Ad -= p * f;
-            Bd -= p * zf;
+        for (int j = 0; j < mmax; ++j) {
+          if (j < m) {
+            const int x = a + j;
+            const float c_hi = cdf_at(x + L, mu_w, inv_w, aw, bw2);
+            float Cv, f, zf;
+            own(j, Cv, f, zf);
+            if (kDep) {
+              const float p = c_hi - c_lo;
+              Ad -= p * f;
+              Bd -= p * zf;
+            }
+            if (kCom) {
+              const float cw = (L == 1) ? c_lo : cdf_at(x, mu_w, inv_w, aw, bw2);
+              Ao += A.alpha * (1.0f - cw) * f;
+              Bo += A.alpha * (1.0f - cw) * zf;
+              if (x < aw) fcom += Cv;
+            }
+            c_lo = c_hi;
           }
-          if (kCom) {
-            const float cw = (L == 1) ? c_lo : cdf_at(x, mu_w, inv_w, aw, bw2);
-            Ao += A.alpha * (1.0f - cw) * f;
-            Bo += A.alpha * (1.0f - cw) * zf;
-            if (x < aw) fcom += Cv;
-          }
-          c_lo = c_hi;
         }
-        if (kCom) fcom += (float)max(0, aw - 1 - bw);
+        __syncwarp();
+        if (kCom && ok) fcom += (float)max(0, aw - 1 - bw);
       }
     }
     // ---- back edges (App. B.3): a dependency with latency Lat(j) - k II ----
     if (kRec) {
-      for (int e = A.bin_ptr[vi]; e < A.bin_ptr[vi + 1]; ++e) {  // own = consumer i
-        const int jc = A.bin_src[e], L = A.bin_shift[e];
-        const float mu_u = A.mu[(size_t)jc * A.B + b], sg_u = A.sg[(size_t)jc * A.B + b];
-        if (!usable(mu_u, sg_u)) continue;
-        const float inv_u = 1.0f / sg_u;
-        int au, bu;
-        window(mu_u, sg_u, A.k_win, A.D, au, bu);
-        float c_lo = cdf_at(a - L, mu_u, inv_u, au, bu);
-        for (int j = 0; j < n; ++j) {
-          const float c_hi = cdf_at(a + j + 1 - L, mu_u, inv_u, au, bu);
-          const float p = c_hi - c_lo;
-          float Cv, f, zf;
-          own(j, Cv, f, zf);
-          frec += Cv * p;
-          Ar += p * f;
-          Br += p * zf;
-          c_lo = c_hi;
+      {  // own = consumer i
+        const int e0 = A.bin_ptr[vcl], deg = valid ? A.bin_ptr[vcl + 1] - e0 : 0;
+        const int dmax = __reduce_max_sync(FULL, deg);
+        for (int q = 0; q < dmax; ++q) {
+          const bool eon = q < deg;
+          const int jc = eon ? A.bin_src[e0 + q] : 0, L = eon ? A.bin_shift[e0 + q] : 0;
+          const float mu_u = eon ? A.mu[(size_t)jc * A.B + b] : 0.f;
+          const float sg_u = eon ? A.sg[(size_t)jc * A.B + b] : 1.f;
+          const bool ok = eon && usable(mu_u, sg_u);
+          const float inv_u = ok ? 1.0f / sg_u : 1.0f;
+          int au = 0, bu = -1;
+          if (ok) window(mu_u, sg_u, A.k_win, A.D, au, bu);
+          const int m = ok ? n : 0;
+          const int mmax = __reduce_max_sync(FULL, m);
+          float c_lo = cdf_at(a - L, mu_u, inv_u, au, bu);
+          for (int j = 0; j < mmax; ++j) {
+            if (j < m) {
+              const float c_hi = cdf_at(a + j + 1 - L, mu_u, inv_u, au, bu);
+              const float p = c_hi - c_lo;
+              float Cv, f, zf;
+              own(j, Cv, f, zf);
+              frec += Cv * p;
+              Ar += p * f;
+              Br += p * zf;
+              c_lo = c_hi;
+            }
+          }
+          __syncwarp();
+          if (ok) frec += 1.0f - c_lo;
         }
-        frec += 1.0f - c_lo;
       }
-      for (int e = A.bout_ptr[vi]; e < A.bout_ptr[vi + 1]; ++e) {  // own = producer j
-        const int ic = A.bout_dst[e], L = A.bout_shift[e];
-        const float mu_w = A.mu[(size_t)ic * A.B + b], sg_w = A.sg[(size_t)ic * A.B + b];
-        if (!usable(mu_w, sg_w)) continue;
-        const float inv_w = 1.0f / sg_w;
-        int aw, bw2;
-        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
-        float c_lo = cdf_at(a + L - 1, mu_w, inv_w, aw, bw2);
-        for (int j = 0; j < n; ++j) {
-          const float c_hi = cdf_at(a + j + L, mu_w, inv_w, aw, bw2);
-          const float p = c_hi - c_lo;
-          float Cv, f, zf;
-          own(j, Cv, f, zf);
-          Ar -= p * f;
-          Br -= p * zf;
-          c_lo = c_hi;
+      {  // own = producer j
+        const int e0 = A.bout_ptr[vcl], deg = valid ? A.bout_ptr[vcl + 1] - e0 : 0;
+        const int dmax = __reduce_max_sync(FULL, deg);
+        for (int q = 0; q < dmax; ++q) {
+          const bool eon = q < deg;
+          const int ic = eon ? A.bout_dst[e0 + q] : 0, L = eon ? A.bout_shift[e0 + q] : 0;
+          const float mu_w = eon ? A.mu[(size_t)ic * A.B + b] : 0.f;
+          const float sg_w = eon ? A.sg[(size_t)ic * A.B + b] : 1.f;
+          const bool ok = eon && usable(mu_w, sg_w);
+          const float inv_w = ok ? 1.0f / sg_w : 1.0f;
+          int aw = 0, bw2 = -1;
+          if (ok) window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
+          const int m = ok ? n : 0;
+          const int mmax = __reduce_max_sync(FULL, m);
+          float c_lo = cdf_at(a + L - 1, mu_w, inv_w, aw, bw2);
+          for (int j = 0; j < mmax; ++j) {
+            if (j < m) {
+              const float c_hi = cdf_at(a + j + L, mu_w, inv_w, aw, bw2);
+              const float p = c_hi - c_lo;
+              float Cv, f, zf;
+              own(j, Cv, f, zf);
+              Ar -= p * f;
+              Br -= p * zf;
+              c_lo = c_hi;
+            }
+          }
+          __syncwarp();
         }
       }
     }
-    A.gpart[0 * VB + gi] = Ad;
-    A.gpart[1 * VB + gi] = Bd;
-    A.gpart[2 * VB + gi] = Ao;
-    A.gpart[3 * VB + gi] = Bo;
-    A.gpart[4 * VB + gi] = Ar;
-    A.gpart[5 * VB + gi] = Br;
+    if (valid) {
+      A.gpart[0 * VB + gi] = Ad;
+      A.gpart[1 * VB + gi] = Bd;
+      A.gpart[2 * VB + gi] = Ao;
+      A.gpart[3 * VB + gi] = Bo;
+      A.gpart[4 * VB + gi] = Ar;
+      A.gpart[5 * VB + gi] = Br;
+    }
   }
 
-  // ---- per-restart forward sums of this block (fixed order) ----
-  s_red[0][tid] = fdep;
-  s_red[1][tid] = fcom;
-  s_red[2][tid] = frec;
+  // ---- per-restart forward sums of this block (fixed order), reusing the cache ----
   if (lo <= hi) {
     atomicMin(&s_lo, lo);
     atomicMax(&s_hi, hi);
   }
   __syncthreads();
+  double *red = reinterpret_cast<double *>(cC);
+  red[0 * T + tid] = fdep;
+  red[1 * T + tid] = fcom;
+  red[2 * T + tid] = frec;
+  __syncthreads();
   if (tid < RB) {
     double acc[3] = {0.0, 0.0, 0.0};
     for (int row = 0; row < rows; ++row)
-      for (int k = 0; k < 3; ++k) acc[k] += s_red[k][row * RB + tid];
+      for (int k = 0; k < 3; ++k) acc[k] += red[k * T + row * RB + tid];
     for (int k = 0; k < 3; ++k) A.fwd[((size_t)blk * RB + tid) * 3 + k] = acc[k];
   }
   // ---- histogram rows restricted to the folded span the block touched ----
@@ -336,11 +411,34 @@ __global__ void __launch_bounds__(kThreads) k_fwd(const IterArgs A) {
   }
   if (tid == 0) A.hspan[blk] = make_int2(flo, fhi);
   const int len = fhi - flo + 1;
-  if (len > 0)
-    for (int i = tid; i < RB * len; i += kThreads) {
-      const int rr = i / len, d = flo + i % len;
-      A.hpart[((size_t)blk * RB + rr) * Dh + d] = hist[rr * Dh + d];
+  if (len > 0) {
+    // partials laid out [block][bin][restart]
+    long long *dst = A.hpart + (size_t)blk * Dh * RB;
+    for (int i = tid; i < RB * len; i += T) {
+      const int cell = flo * RB + i;
+      dst[cell] = (long long)(((unsigned long long)hhi[cell] << 16) + (unsigned long long)hlo[cell]);
     }
+  }
+}
+
+// Usage per (restart, class, bin) from the partials of every block of the class
+// (fixed order over segments; exact int64 sums).  Block = (group g, class c,
+// tile of 256/RB bins); threads = restarts x bins, coalesced over restarts.
+__global__ void __launch_bounds__(256) k_reduce(const RedArgs A) {
+  const int RB = A.RB, Dh = A.Dh, per = 256 / RB;
+  const int tiles = (Dh + per - 1) / per;
+  int x = blockIdx.x;
+  const int tile = x % tiles; x /= tiles;
+  const int c = x % A.C, g = x / A.C;
+  const int r = threadIdx.x % RB, d = tile * per + threadIdx.x / RB, b = g * RB + r;
+  if (d >= Dh || b >= A.B) return;
+  long long acc = 0;
+  for (int s = A.cls_seg_ptr[c]; s < A.cls_seg_ptr[c + 1]; ++s) {
+    const int blk = s * A.G + g;
+    const int2 sp = A.hspan[blk];
+    if (d >= sp.x && d <= sp.y) acc += A.hpart[((size_t)blk * Dh + d) * RB + r];
+  }
+  A.U[((size_t)b * A.C + c) * Dh + d] = (double)acc * kInvFix;
 }
 
 // Deterministic block reduction (blockDim.x == 256).
@@ -377,16 +475,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   __shared__ double s_m[kMaxClasses], s_s[kMaxClasses];
   const int b = blockIdx.x, g = b / A.RB, r = b % A.RB, tid = threadIdx.x, Dh = A.Dh;
 
-  for (int c = 0; c < A.C; ++c)
-    for (int t = tid; t < Dh; t += 256) {
-      long long acc = 0;
-      for (int s = A.cls_seg_ptr[c]; s < A.cls_seg_ptr[c + 1]; ++s) {
-        const int blk = s * A.G + g;
-        const int2 sp = A.hspan[blk];
-        if (t >= sp.x && t <= sp.y) acc += A.hpart[((size_t)blk * A.RB + r) * Dh + t];
-      }
-      U[c * Dh + t] = (double)acc * kInvFix;
-    }
+  for (int i = tid; i < A.C * Dh; i += 256) U[i] = A.Ug[(size_t)b * A.C * Dh + i];
   __syncthreads();
 
   // forward sums of the edge terms over every block of this restart group

@@ -233,8 +233,15 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
   int G = (p->B + RB - 1) / RB;
   long want = std::max(1L, (long)target_blocks / G);
   int seglen = (int)std::max(1L, ((long)V + want - 1) / want);
-  // keep a segment to a handful of rows per thread at least
-  seglen = std::max(seglen, std::max(1, kThreads / RB));
+  // at least one row of nodes per block pass; and few enough nodes that the
+  // 16-bit halves of the shared-memory usage histogram cannot overflow:
+  // segment length * max demand * ceil(D / Dh) * 2^16 < 2^32
+  seglen = std::max(seglen, std::max(1, kFwdThreads / RB));
+  int maxw = 1;
+  for (int v = 0; v < V; ++v) maxw = std::max(maxw, P.c_dem[v]);
+  const long folds = (p->D + P.Dh - 1) / P.Dh;
+  const long cap = std::max(1L, 32768L / ((long)maxw * folds));
+  seglen = (int)std::max(1L, std::min<long>(seglen, cap));
   P.cls_seg_ptr.assign(C + 1, 0);
   int i0 = 0;
   for (int c = 0; c < C; ++c) {
