@@ -22,6 +22,7 @@
 #include <stdint.h>
 
 #include "gaus_internal.h"
+#include "mills_ratio.h"
 
 namespace gaus {
 
@@ -93,11 +94,23 @@ __device__ __forceinline__ void window(float mu, float sg, float k, int D, int &
   b = (int)hi;
 }
 
+// Phi(z) from the Mills ratio: the upper tail Q(|z|) = exp(-z^2/2) P(|z|)/Q(|z|)
+// (rational fit of mills_ratio.h, |z| <= 12), absolute error ~1e-6.  Used for
+// the neighbour values of the edge terms, which only need absolute accuracy.
+__device__ __forceinline__ float cdf_fast(float z) {
+  const float x = fabsf(z);
+  const float e = __expf(-0.5f * z * z);
+  const float num = (((kMillsP[4] * x + kMillsP[3]) * x + kMillsP[2]) * x + kMillsP[1]) * x + kMillsP[0];
+  const float den = ((((kMillsQ[5] * x + kMillsQ[4]) * x + kMillsQ[3]) * x + kMillsQ[2]) * x + kMillsQ[1]) * x + 1.0f;
+  const float q = e * __fdividef(num, den);
+  return z <= 0.f ? q : 1.0f - q;
+}
+
 // Windowed CDF of a neighbour at integer point x.
 __device__ __forceinline__ float cdf_at(int x, float mu, float inv_s, int a, int b) {
   if (x < a) return 0.0f;
   if (x > b) return 1.0f;
-  return normcdff(((float)x + 0.5f - mu) * inv_s);
+  return cdf_fast(((float)x + 0.5f - mu) * inv_s);
 }
 
 __device__ __forceinline__ int fold_bin(int d, int II) { return II > 0 ? d % II : d; }
@@ -110,6 +123,136 @@ __device__ __forceinline__ bool usable(float mu, float sg) {
 
 constexpr float kInvSqrt2Pi = 0.3989422804014327f;
 constexpr float kInvSqrt2 = 0.7071067811865476f;
+
+// Bin mass of bin p of a window from the tail values (z, q = Q(|z|)) of points p
+// and p - 1: P = C(a+p) - C(a+p-1), with C = 0 below the window and 1 above it,
+// choosing the subtraction that keeps both tails relatively accurate.
+__device__ __forceinline__ float bin_mass(bool pt, bool first, float zc, float qc, float zp, float qp) {
+  const float c_cur = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;
+  const float c_prev = first ? 0.0f : (zp <= 0.f ? qp : 1.0f - qp);
+  float P = c_cur - c_prev;
+  P = (pt && !first && zc <= 0.f) ? qc - qp : P;
+  P = (pt && !first && zp > 0.f) ? qp - qc : P;
+  P = (pt && !first && zp <= 0.f && zc > 0.f) ? (0.5f - qc) + (0.5f - qp) : P;
+  P = (!pt && !first && zp > 0.f) ? qp : P;  // top bin: upper tail Q directly
+  return P;
+}
+
+// Adds round(w P 2^32) to a histogram cell as two exact 16-bit halves, using
+// 32-bit conversions only (float -> 64-bit integer conversion runs at the FP64 rate).
+__device__ __forceinline__ void hist_add(unsigned *hlo, unsigned *hhi, int cell, float wP) {
+  const float xs = fmaxf(wP, 0.0f) * 65536.0f;
+  const float fh = floorf(xs);
+  atomicAdd(&hlo[cell], __float2uint_rn((xs - fh) * 65536.0f));
+  atomicAdd(&hhi[cell], (unsigned)fh);
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// One (node, restart) item whose window is long, processed by the whole warp with
+// lanes over its points (32 at a time).  Same terms and formulas as the per-lane
+// path; the warp-reduced sums are returned in out[0..8] on every lane:
+// Ad, Bd, Ao, Bo, Ar, Br, fdep, fcom, frec.
+template <bool kDep, bool kCom, bool kRec>
+__device__ void coop_item(const IterArgs &A, int vcl, int b, int r, int RB, float mu, float inv_s, int a, int bw,
+                          float wv, unsigned *hlo, unsigned *hhi, float out[9]) {
+  constexpr unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31, n = bw - a + 1;
+  float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f, fdep = 0.f, fcom = 0.f, frec = 0.f;
+  float z_carry = 0.f, q_carry = 0.f;
+  for (int base = 0; base <= n; base += 32) {
+    const int pidx = base + lane;
+    const bool pt = pidx < n;
+    const int t = a + pidx;
+    const float z = ((float)t + 0.5f - mu) * inv_s;
+    const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
+    const float Cv = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
+    const float f = pt ? kInvSqrt2Pi * expf(-0.5f * z * z) : 0.f;
+    const float zf = z * f;
+    float zp = __shfl_up_sync(FULL, z, 1), qp = __shfl_up_sync(FULL, q, 1);
+    if (lane == 0) { zp = z_carry; qp = q_carry; }
+    if (pidx <= n) hist_add(hlo, hhi, fold_bin(t, A.II) * RB + r, wv * bin_mass(pt, pidx == 0, z, q, zp, qp));
+    z_carry = __shfl_sync(FULL, z, 31);
+    q_carry = __shfl_sync(FULL, q, 31);
+    if (kDep || kCom) {
+      for (int e = A.in_ptr[vcl]; e < A.in_ptr[vcl + 1]; ++e) {  // own = consumer
+        const int uc = A.in_src[e], L = A.in_lat[e];
+        const float mu_u = A.mu[(size_t)uc * A.B + b], sg_u = A.sg[(size_t)uc * A.B + b];
+        if (!usable(mu_u, sg_u)) continue;
+        const float inv_u = 1.0f / sg_u;
+        int au, bu;
+        window(mu_u, sg_u, A.k_win, A.D, au, bu);
+        if (pt) {
+          const float c_hi = cdf_at(t + 1 - L, mu_u, inv_u, au, bu);
+          const float p = c_hi - cdf_at(t - L, mu_u, inv_u, au, bu);
+          if (kDep) { fdep += Cv * p; Ad += p * f; Bd += p * zf; }
+          if (kCom) {
+            const float cu = (L == 1) ? c_hi : cdf_at(t, mu_u, inv_u, au, bu);
+            fcom += cu * (1.0f - Cv);
+            Ao -= A.alpha * cu * f;
+            Bo -= A.alpha * cu * zf;
+          }
+        }
+        if (kDep && base == 0 && lane == 0) fdep += 1.0f - cdf_at(bw + 1 - L, mu_u, inv_u, au, bu);
+      }
+      const int L = A.lat[vcl];
+      for (int e = A.out_ptr[vcl]; e < A.out_ptr[vcl + 1]; ++e) {  // own = producer
+        const int wc = A.out_dst[e];
+        const float mu_w = A.mu[(size_t)wc * A.B + b], sg_w = A.sg[(size_t)wc * A.B + b];
+        if (!usable(mu_w, sg_w)) continue;
+        const float inv_w = 1.0f / sg_w;
+        int aw, bw2;
+        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
+        if (pt) {
+          const float c_hi = cdf_at(t + L, mu_w, inv_w, aw, bw2);
+          const float c_lo = cdf_at(t + L - 1, mu_w, inv_w, aw, bw2);
+          if (kDep) { const float p = c_hi - c_lo; Ad -= p * f; Bd -= p * zf; }
+          if (kCom) {
+            const float cw = (L == 1) ? c_lo : cdf_at(t, mu_w, inv_w, aw, bw2);
+            Ao += A.alpha * (1.0f - cw) * f;
+            Bo += A.alpha * (1.0f - cw) * zf;
+            if (t < aw) fcom += Cv;
+          }
+        }
+        if (kCom && base == 0 && lane == 0) fcom += (float)max(0, aw - 1 - bw);
+      }
+    }
+    if (kRec) {
+      for (int e = A.bin_ptr[vcl]; e < A.bin_ptr[vcl + 1]; ++e) {  // own = consumer i
+        const int jc = A.bin_src[e], L = A.bin_shift[e];
+        const float mu_u = A.mu[(size_t)jc * A.B + b], sg_u = A.sg[(size_t)jc * A.B + b];
+        if (!usable(mu_u, sg_u)) continue;
+        const float inv_u = 1.0f / sg_u;
+        int au, bu;
+        window(mu_u, sg_u, A.k_win, A.D, au, bu);
+        if (pt) {
+          const float p = cdf_at(t + 1 - L, mu_u, inv_u, au, bu) - cdf_at(t - L, mu_u, inv_u, au, bu);
+          frec += Cv * p; Ar += p * f; Br += p * zf;
+        }
+        if (base == 0 && lane == 0) frec += 1.0f - cdf_at(bw + 1 - L, mu_u, inv_u, au, bu);
+      }
+      for (int e = A.bout_ptr[vcl]; e < A.bout_ptr[vcl + 1]; ++e) {  // own = producer j
+        const int ic = A.bout_dst[e], L = A.bout_shift[e];
+        const float mu_w = A.mu[(size_t)ic * A.B + b], sg_w = A.sg[(size_t)ic * A.B + b];
+        if (!usable(mu_w, sg_w)) continue;
+        const float inv_w = 1.0f / sg_w;
+        int aw, bw2;
+        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
+        if (pt) {
+          const float p = cdf_at(t + L, mu_w, inv_w, aw, bw2) - cdf_at(t + L - 1, mu_w, inv_w, aw, bw2);
+          Ar -= p * f; Br -= p * zf;
+        }
+      }
+    }
+  }
+  __syncwarp();
+  out[0] = warp_sum(Ad); out[1] = warp_sum(Bd); out[2] = warp_sum(Ao); out[3] = warp_sum(Bo);
+  out[4] = warp_sum(Ar); out[5] = warp_sum(Br);
+  out[6] = warp_sum(fdep); out[7] = warp_sum(fcom); out[8] = warp_sum(frec);
+}
 
 template <bool kDep, bool kCom, bool kRec>
 __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
@@ -158,7 +301,14 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     const float inv_s = valid ? 1.0f / sg : 1.0f, wv = A.w[vcl];
     int a = 0, bw = -2;
     if (valid) window(mu, sg, A.k_win, A.D, a, bw);
-    const int n = bw - a + 1;                      // points; -1 for an idle lane
+    const int nfull = bw - a + 1;                  // points; -1 for an idle lane
+    // Windows much longer than the warp's typical one (or than the cache) go to
+    // the cooperative path after this per-lane pass.
+    const int nact = __popc(__ballot_sync(FULL, valid));
+    const int mean = nact ? __reduce_add_sync(FULL, max(nfull, 0)) / nact : 0;
+    const bool is_long = valid && nfull > min(kc, max(8, 3 * mean + 8));
+    const int n = is_long ? -1 : nfull;            // per-lane points
+    const bool vs = valid && !is_long;
     const int nmax = __reduce_max_sync(FULL, n);
 
     // ---- own points: cache C, phi, z*phi; bin masses into the usage histogram ----
@@ -176,23 +326,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
         cF[j * T + tid] = f;
         cZ[j * T + tid] = zc * f;
       }
-      // branch-free selection of the bin-mass formula
-      const float c_cur = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;       // C(a+j), 1 past the window
-      const float c_prev = j == 0 ? 0.0f : (zp <= 0.f ? qp : 1.0f - qp);  // C(a+j-1)
-      float P = c_cur - c_prev;
-      P = (pt && j > 0 && zc <= 0.f) ? qc - qp : P;
-      P = (pt && j > 0 && zp > 0.f) ? qp - qc : P;
-      P = (pt && j > 0 && zp <= 0.f && zc > 0.f) ? (0.5f - qc) + (0.5f - qp) : P;
-      P = (!pt && j > 0 && zp > 0.f) ? qp : P;     // top bin: upper tail Q directly
-      if (j <= n) {
-        // round(x 2^32) = hi 2^16 + lo with hi = floor(x 2^16) and lo = round(frac 2^16),
-        // using 32-bit conversions only (64-bit ones run at the FP64 rate)
-        const float xs = fmaxf(wv * P, 0.0f) * 65536.0f;
-        const float fh = floorf(xs);
-        const int cell = fold_bin(a + j, A.II) * RB + r;
-        atomicAdd(&hlo[cell], __float2uint_rn((xs - fh) * 65536.0f));
-        atomicAdd(&hhi[cell], (unsigned)fh);
-      }
+      if (j <= n) hist_add(hlo, hhi, fold_bin(a + j, A.II) * RB + r, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
       zp = zc;
       qp = qc;
     }
@@ -223,7 +357,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     // dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
     // dL_com,e/dC_v(t) = -C_u(t)
     if (kDep || kCom) {
-      const int e0 = A.in_ptr[vcl], deg = valid ? A.in_ptr[vcl + 1] - e0 : 0;
+      const int e0 = A.in_ptr[vcl], deg = vs ? A.in_ptr[vcl + 1] - e0 : 0;
       const int dmax = __reduce_max_sync(FULL, deg);
       for (int q = 0; q < dmax; ++q) {
         const bool eon = q < deg;
@@ -267,7 +401,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     // L_com,e part = sum_{x in own, x < a_w} C_v(x) + max(0, a_w - 1 - b_v)
     if (kDep || kCom) {
       const int L = A.lat[vcl];
-      const int e0 = A.out_ptr[vcl], deg = valid ? A.out_ptr[vcl + 1] - e0 : 0;
+      const int e0 = A.out_ptr[vcl], deg = vs ? A.out_ptr[vcl + 1] - e0 : 0;
       const int dmax = __reduce_max_sync(FULL, deg);
       for (int q = 0; q < dmax; ++q) {
         const bool eon = q < deg;
@@ -308,7 +442,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     // ---- back edges (App. B.3): a dependency with latency Lat(j) - k II ----
     if (kRec) {
       {  // own = consumer i
-        const int e0 = A.bin_ptr[vcl], deg = valid ? A.bin_ptr[vcl + 1] - e0 : 0;
+        const int e0 = A.bin_ptr[vcl], deg = vs ? A.bin_ptr[vcl + 1] - e0 : 0;
         const int dmax = __reduce_max_sync(FULL, deg);
         for (int q = 0; q < dmax; ++q) {
           const bool eon = q < deg;
@@ -339,7 +473,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
         }
       }
       {  // own = producer j
-        const int e0 = A.bout_ptr[vcl], deg = valid ? A.bout_ptr[vcl + 1] - e0 : 0;
+        const int e0 = A.bout_ptr[vcl], deg = vs ? A.bout_ptr[vcl + 1] - e0 : 0;
         const int dmax = __reduce_max_sync(FULL, deg);
         for (int q = 0; q < dmax; ++q) {
           const bool eon = q < deg;
@@ -366,6 +500,23 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
           }
           __syncwarp();
         }
+      }
+    }
+    // ---- cooperative pass over the long windows of this warp ----
+    unsigned longmask = __ballot_sync(FULL, is_long);
+    while (longmask) {
+      const int src = __ffs(longmask) - 1;
+      longmask &= longmask - 1;
+      const int l_v = __shfl_sync(FULL, vcl, src), l_b = __shfl_sync(FULL, b, src);
+      const int l_r = __shfl_sync(FULL, r, src), l_a = __shfl_sync(FULL, a, src);
+      const int l_bw = __shfl_sync(FULL, bw, src);
+      const float l_mu = __shfl_sync(FULL, mu, src), l_inv = __shfl_sync(FULL, inv_s, src);
+      const float l_w = __shfl_sync(FULL, wv, src);
+      float sums[9];
+      coop_item<kDep, kCom, kRec>(A, l_v, l_b, l_r, RB, l_mu, l_inv, l_a, l_bw, l_w, hlo, hhi, sums);
+      if ((threadIdx.x & 31) == src) {
+        Ad = sums[0]; Bd = sums[1]; Ao = sums[2]; Bo = sums[3]; Ar = sums[4]; Br = sums[5];
+        fdep += sums[6]; fcom += sums[7]; frec += sums[8];
       }
     }
     if (valid) {

@@ -203,3 +203,15 @@ def test_run_to_run_determinism(g):
     for k in a:
         assert torch.equal(a[k], b[k]), k
     ctx.close()
+
+
+def test_mixed_window_lengths_short_and_cooperative_paths(g):
+    # sigma spread over two orders of magnitude inside every warp: most windows
+    # take the per-lane path, the long ones the warp-cooperative path
+    p = W.logic_network(6, V=1500, depth=30)
+    B = 32
+    rng = np.random.default_rng(12)
+    mu = (p.start[:, None] + rng.normal(0, 2, size=(p.V, B))).astype(np.float32)
+    sg = np.exp(rng.uniform(np.log(0.05), np.log(6.0), size=(p.V, B))).astype(np.float32)
+    hp = g.default_hparams(terms=p.terms, rho=1e-3)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, rng), hp, restarts=range(0, 32, 4))
