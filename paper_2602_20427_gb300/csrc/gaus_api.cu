@@ -69,7 +69,7 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   A.bin_ptr = ctx->d_bin_ptr; A.bin_src = ctx->d_bin_src; A.bin_shift = ctx->d_bin_shift;
   A.bout_ptr = ctx->d_bout_ptr; A.bout_dst = ctx->d_bout_dst; A.bout_shift = ctx->d_bout_shift;
   A.seg = ctx->d_seg; A.hpart = ctx->d_hpart; A.hspan = ctx->d_hspan; A.fwd = ctx->d_fwd;
-  A.gpart = ctx->d_gpart; A.nonfinite = ctx->d_nonfinite;
+  A.gpart = ctx->d_gpart; A.nonfinite = ctx->d_nonfinite; A.win = ctx->d_win;
   return A;
 }
 
@@ -97,6 +97,12 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   const Plan &P = ctx->plan;
   const unsigned on = ctx->hp.terms;
   IterArgs A = iter_args(ctx, mu, sg);
+  {
+    const size_t n = (size_t)P.V * P.B;
+    k_windows<<<(int)std::min<size_t>((n + 255) / 256, 8 * 152), 256, 0, st>>>(mu, sg, ctx->d_win, n,
+                                                                          ctx->hp.window_k, P.D);
+    CK(cudaGetLastError(), "k_windows launch");
+  }
   FwdKernel kf = pick_fwd(on, P.II);
   kf<<<ctx->nblk, kFwdThreads, ctx->smem_fwd, st>>>(A);
   CK(cudaGetLastError(), "k_fwd launch");
@@ -254,6 +260,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
   TRY(scratch(ctx, &ctx->d_fwd, (size_t)ctx->nblk * ctx->RB * 3));
   TRY(scratch(ctx, &ctx->d_gpart, 6 * VB));
+  TRY(scratch(ctx, &ctx->d_win, VB));
   TRY(scratch(ctx, &ctx->d_H, (size_t)P.B * P.C * P.Dh));
   TRY(scratch(ctx, &ctx->d_coef, (size_t)P.B * 4));
   TRY(scratch(ctx, &ctx->d_nonfinite, (size_t)P.B));

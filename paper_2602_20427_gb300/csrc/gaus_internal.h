@@ -95,6 +95,7 @@ struct gaus_ctx {
   double *d_fwd = nullptr;       // nblk * RB * 3 forward sums (dep, com, rec)
   double *d_U = nullptr;         // B * C * Dh usage (k_reduce)
   float *d_gpart = nullptr;      // 6 * V * B partial gradient sums (internal index)
+  unsigned *d_win = nullptr;     // V * B packed windows (caller order)
   float *d_H = nullptr;          // B * C * Dh usage adjoint dL/dU
   float *d_coef = nullptr;       // B * 4 (c_dep, c_rec)
   int32_t *d_nonfinite = nullptr;  // B flags

@@ -43,6 +43,7 @@ struct IterArgs {
   double *fwd;
   float *gpart;
   int32_t *nonfinite;
+  const unsigned *win;  // (V, B) packed windows: a | (b + 1) << 16
 };
 
 struct RedArgs {
@@ -266,12 +267,12 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
   float *cC = reinterpret_cast<float *>(hhi + (size_t)Dh * RB);
   float *cF = cC + (size_t)kc * T;
   float *cZ = cF + (size_t)kc * T;
-  __shared__ int s_lo, s_hi;
+  __shared__ int s_lo, s_hi, s_next;
 
   const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
   const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1];
   for (int i = tid; i < 2 * RB * Dh; i += T) hlo[i] = 0u;
-  if (tid == 0) { s_lo = INT_MAX; s_hi = INT_MIN; }
+  if (tid == 0) { s_lo = INT_MAX; s_hi = INT_MIN; s_next = 0; }
   __syncthreads();
 
   const int r = tid % RB, b = g * RB + r, rows = T / RB;
@@ -280,13 +281,17 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
   constexpr unsigned FULL = 0xffffffffu;
   float fdep = 0.f, fcom = 0.f, frec = 0.f;
   int lo = INT_MAX, hi = INT_MIN;
-  // Control flow is kept warp-uniform: every lane runs the same item count and
-  // every loop runs to the warp's maximum trip count with a per-lane predicate,
-  // so the warp never splits around the shared-memory atomics.
-  const int n_items = (s1 - s0 + rows - 1) / rows;
-
-  for (int it = 0; it < n_items; ++it) {
-    const int vi = s0 + tid / RB + it * rows;
+  // Control flow is kept warp-uniform: each warp claims the next group of
+  // 32 / RB nodes of the segment from a shared counter (so warps finish
+  // together), and every loop runs to the warp's maximum trip count with a
+  // per-lane predicate, so the warp never splits around the shared atomics.
+  const int npw = 32 / RB;
+  for (;;) {
+    int base = 0;
+    if ((tid & 31) == 0) base = atomicAdd(&s_next, npw);
+    base = __shfl_sync(FULL, base, 0);
+    if (base >= s1 - s0) break;
+    const int vi = s0 + base + (tid & 31) / RB;
     bool valid = bok && vi < s1;
     const int vcl = valid ? vi : s0;
     const int vc = A.perm[vcl];
@@ -352,28 +357,35 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     };
 
     float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f;
-    // ---- in-edges u -> v (own = consumer), latency L = Lat(u) ----
-    // V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
-    // dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
-    // dL_com,e/dC_v(t) = -C_u(t)
+    // ---- edges: every edge term is a dot product of the own window with the
+    // neighbour's CDF shifted by a latency; only the own points where the
+    // neighbour's values vary (or, for communication, are a constant 1) are
+    // visited, and the neighbour's mean and sigma are read only then. ----
+    // in-edges u -> v (own = consumer), latency L = Lat(u):
+    //   V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
+    //   dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
+    //   dL_com,e/dC_v(t) = -C_u(t)
     if (kDep || kCom) {
       const int e0 = A.in_ptr[vcl], deg = vs ? A.in_ptr[vcl + 1] - e0 : 0;
       const int dmax = __reduce_max_sync(FULL, deg);
       for (int q = 0; q < dmax; ++q) {
         const bool eon = q < deg;
         const int uc = eon ? A.in_src[e0 + q] : 0, L = eon ? A.in_lat[e0 + q] : 0;
-        const float mu_u = eon ? A.mu[(size_t)uc * A.B + b] : 0.f;
-        const float sg_u = eon ? A.sg[(size_t)uc * A.B + b] : 1.f;
-        const bool ok = eon && usable(mu_u, sg_u);
-        const float inv_u = ok ? 1.0f / sg_u : 1.0f;
-        int au = 0, bu = -1;
-        if (ok) window(mu_u, sg_u, A.k_win, A.D, au, bu);
-        const int m = ok ? n : 0;
-        const int mmax = __reduce_max_sync(FULL, m);
-        float c_lo = cdf_at(a - L, mu_u, inv_u, au, bu);
-        for (int j = 0; j < mmax; ++j) {
-          if (j < m) {
-            const int t = a + j;
+        const unsigned wm = eon ? A.win[(size_t)uc * A.B + b] : 0u;
+        const int au = (int)(wm & 0xFFFFu), bu = (int)(wm >> 16) - 1;
+        // P_u(t+1-L) != 0 for t in [au+L-1, bu+L]; C_u(t) != 0 for t >= au
+        const int jlo = max(0, au + min(kDep ? L - 1 : 0, 0) - a);
+        const int jhi = kCom ? n - 1 : min(n - 1, bu + L - a);
+        const int x0 = bw + 1 - L;
+        const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
+        const bool need = cnt > 0 || (kDep && eon && x0 >= au && x0 <= bu);
+        const float mu_u = need ? A.mu[(size_t)uc * A.B + b] : 0.f;
+        const float inv_u = need ? 1.0f / A.sg[(size_t)uc * A.B + b] : 1.f;
+        const int cmax = __reduce_max_sync(FULL, cnt);
+        float c_lo = cnt ? cdf_at(a + jlo - L, mu_u, inv_u, au, bu) : 0.f;
+        for (int k2 = 0; k2 < cmax; ++k2) {
+          if (k2 < cnt) {
+            const int j = jlo + k2, t = a + j;
             const float c_hi = cdf_at(t + 1 - L, mu_u, inv_u, au, bu);
             const float p = c_hi - c_lo;
             float Cv, f, zf;
@@ -393,12 +405,13 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
           }
         }
         __syncwarp();
-        if (kDep && ok) fdep += 1.0f - c_lo;
+        if (kDep && eon) fdep += 1.0f - cdf_at(x0, mu_u, inv_u, au, bu);
       }
     }
-    // ---- out-edges v -> w (own = producer), latency L = Lat(v) ----
-    // dV_e/dC_v(x) = -P_w(x + L);  dL_com,e/dC_v(x) = 1 - C_w(x)
-    // L_com,e part = sum_{x in own, x < a_w} C_v(x) + max(0, a_w - 1 - b_v)
+    // out-edges v -> w (own = producer), latency L = Lat(v):
+    //   dV_e/dC_v(x) = -P_w(x + L), nonzero for x in [aw-L, bw+1-L]
+    //   dL_com,e/dC_v(x) = 1 - C_w(x), nonzero for x <= bw
+    //   L_com,e part = sum_{x in own, x < a_w} C_v(x) + max(0, a_w - 1 - b_v)
     if (kDep || kCom) {
       const int L = A.lat[vcl];
       const int e0 = A.out_ptr[vcl], deg = vs ? A.out_ptr[vcl + 1] - e0 : 0;
@@ -406,18 +419,21 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
       for (int q = 0; q < dmax; ++q) {
         const bool eon = q < deg;
         const int wc = eon ? A.out_dst[e0 + q] : 0;
-        const float mu_w = eon ? A.mu[(size_t)wc * A.B + b] : 0.f;
-        const float sg_w = eon ? A.sg[(size_t)wc * A.B + b] : 1.f;
-        const bool ok = eon && usable(mu_w, sg_w);
-        const float inv_w = ok ? 1.0f / sg_w : 1.0f;
-        int aw = 0, bw2 = -1;
-        if (ok) window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
-        const int m = ok ? n : 0;
-        const int mmax = __reduce_max_sync(FULL, m);
-        float c_lo = cdf_at(a + L - 1, mu_w, inv_w, aw, bw2);
-        for (int j = 0; j < mmax; ++j) {
-          if (j < m) {
-            const int x = a + j;
+        const unsigned wm = eon ? A.win[(size_t)wc * A.B + b] : 0u;
+        const int aw = (int)(wm & 0xFFFFu), bw2 = (int)(wm >> 16) - 1;
+        int jlo = max(0, aw - L - a), jhi = min(n - 1, bw2 + 1 - L - a);
+        if (kCom) {
+          jlo = 0;
+          jhi = max(jhi, min(n - 1, bw2 - a));
+        }
+        const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
+        const float mu_w = cnt ? A.mu[(size_t)wc * A.B + b] : 0.f;
+        const float inv_w = cnt ? 1.0f / A.sg[(size_t)wc * A.B + b] : 1.f;
+        const int cmax = __reduce_max_sync(FULL, cnt);
+        float c_lo = cnt ? cdf_at(a + jlo + L - 1, mu_w, inv_w, aw, bw2) : 0.f;
+        for (int k2 = 0; k2 < cmax; ++k2) {
+          if (k2 < cnt) {
+            const int j = jlo + k2, x = a + j;
             const float c_hi = cdf_at(x + L, mu_w, inv_w, aw, bw2);
             float Cv, f, zf;
             own(j, Cv, f, zf);
@@ -436,10 +452,10 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
           }
         }
         __syncwarp();
-        if (kCom && ok) fcom += (float)max(0, aw - 1 - bw);
+        if (kCom && eon) fcom += (float)max(0, aw - 1 - bw);
       }
     }
-    // ---- back edges (App. B.3): a dependency with latency Lat(j) - k II ----
+    // back edges (App. B.3): a dependency with latency Lat(j) - k II
     if (kRec) {
       {  // own = consumer i
         const int e0 = A.bin_ptr[vcl], deg = vs ? A.bin_ptr[vcl + 1] - e0 : 0;
@@ -447,17 +463,19 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
         for (int q = 0; q < dmax; ++q) {
           const bool eon = q < deg;
           const int jc = eon ? A.bin_src[e0 + q] : 0, L = eon ? A.bin_shift[e0 + q] : 0;
-          const float mu_u = eon ? A.mu[(size_t)jc * A.B + b] : 0.f;
-          const float sg_u = eon ? A.sg[(size_t)jc * A.B + b] : 1.f;
-          const bool ok = eon && usable(mu_u, sg_u);
-          const float inv_u = ok ? 1.0f / sg_u : 1.0f;
-          int au = 0, bu = -1;
-          if (ok) window(mu_u, sg_u, A.k_win, A.D, au, bu);
-          const int m = ok ? n : 0;
-          const int mmax = __reduce_max_sync(FULL, m);
-          float c_lo = cdf_at(a - L, mu_u, inv_u, au, bu);
-          for (int j = 0; j < mmax; ++j) {
-            if (j < m) {
+          const unsigned wm = eon ? A.win[(size_t)jc * A.B + b] : 0u;
+          const int au = (int)(wm & 0xFFFFu), bu = (int)(wm >> 16) - 1;
+          const int jlo = max(0, au + L - 1 - a), jhi = min(n - 1, bu + L - a);
+          const int x0 = bw + 1 - L;
+          const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
+          const bool need = cnt > 0 || (eon && x0 >= au && x0 <= bu);
+          const float mu_u = need ? A.mu[(size_t)jc * A.B + b] : 0.f;
+          const float inv_u = need ? 1.0f / A.sg[(size_t)jc * A.B + b] : 1.f;
+          const int cmax = __reduce_max_sync(FULL, cnt);
+          float c_lo = cnt ? cdf_at(a + jlo - L, mu_u, inv_u, au, bu) : 0.f;
+          for (int k2 = 0; k2 < cmax; ++k2) {
+            if (k2 < cnt) {
+              const int j = jlo + k2;
               const float c_hi = cdf_at(a + j + 1 - L, mu_u, inv_u, au, bu);
               const float p = c_hi - c_lo;
               float Cv, f, zf;
@@ -469,7 +487,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
             }
           }
           __syncwarp();
-          if (ok) frec += 1.0f - c_lo;
+          if (eon) frec += 1.0f - cdf_at(x0, mu_u, inv_u, au, bu);
         }
       }
       {  // own = producer j
@@ -478,17 +496,17 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
         for (int q = 0; q < dmax; ++q) {
           const bool eon = q < deg;
           const int ic = eon ? A.bout_dst[e0 + q] : 0, L = eon ? A.bout_shift[e0 + q] : 0;
-          const float mu_w = eon ? A.mu[(size_t)ic * A.B + b] : 0.f;
-          const float sg_w = eon ? A.sg[(size_t)ic * A.B + b] : 1.f;
-          const bool ok = eon && usable(mu_w, sg_w);
-          const float inv_w = ok ? 1.0f / sg_w : 1.0f;
-          int aw = 0, bw2 = -1;
-          if (ok) window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
-          const int m = ok ? n : 0;
-          const int mmax = __reduce_max_sync(FULL, m);
-          float c_lo = cdf_at(a + L - 1, mu_w, inv_w, aw, bw2);
-          for (int j = 0; j < mmax; ++j) {
-            if (j < m) {
+          const unsigned wm = eon ? A.win[(size_t)ic * A.B + b] : 0u;
+          const int aw = (int)(wm & 0xFFFFu), bw2 = (int)(wm >> 16) - 1;
+          const int jlo = max(0, aw - L - a), jhi = min(n - 1, bw2 + 1 - L - a);
+          const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
+          const float mu_w = cnt ? A.mu[(size_t)ic * A.B + b] : 0.f;
+          const float inv_w = cnt ? 1.0f / A.sg[(size_t)ic * A.B + b] : 1.f;
+          const int cmax = __reduce_max_sync(FULL, cnt);
+          float c_lo = cnt ? cdf_at(a + jlo + L - 1, mu_w, inv_w, aw, bw2) : 0.f;
+          for (int k2 = 0; k2 < cmax; ++k2) {
+            if (k2 < cnt) {
+              const int j = jlo + k2;
               const float c_hi = cdf_at(a + j + L, mu_w, inv_w, aw, bw2);
               const float p = c_hi - c_lo;
               float Cv, f, zf;
@@ -590,6 +608,17 @@ __global__ void __launch_bounds__(256) k_reduce(const RedArgs A) {
     if (d >= sp.x && d <= sp.y) acc += A.hpart[((size_t)blk * Dh + d) * RB + r];
   }
   A.U[((size_t)b * A.C + c) * Dh + d] = (double)acc * kInvFix;
+}
+
+// Window of every (node, restart): a | (b + 1) << 16 with the points [a, b] of
+// window(); an unusable mean/sigma gets the empty window at the horizon start.
+__global__ void k_windows(const float *mu, const float *sg, unsigned *win, size_t n, float k, int D) {
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+    int a = 0, b = -1;
+    const float m = mu[i], s = sg[i];
+    if (usable(m, s)) window(m, s, k, D, a, b);
+    win[i] = (unsigned)a | ((unsigned)(b + 1) << 16);
+  }
 }
 
 // Deterministic block reduction (blockDim.x == 256).

@@ -242,6 +242,10 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
   const long folds = (p->D + P.Dh - 1) / P.Dh;
   const long cap = std::max(1L, 32768L / ((long)maxw * folds));
   seglen = (int)std::max(1L, std::min<long>(seglen, cap));
+  // whole rows of the block: warps then claim equal shares
+  const int rows = kFwdThreads / RB;
+  if (seglen > rows) seglen = (seglen + rows - 1) / rows * rows;
+  if (seglen > cap) seglen = (int)std::max(1L, cap >= rows ? cap - cap % rows : cap);
   P.cls_seg_ptr.assign(C + 1, 0);
   int i0 = 0;
   for (int c = 0; c < C; ++c) {
