@@ -21,8 +21,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "gaus_device.cuh"
 #include "gaus_internal.h"
-#include "mills_ratio.h"
 
 namespace gaus {
 
@@ -85,68 +85,6 @@ struct UpdArgs {
   const int32_t *step_dev;                   // per-restart step (Adam mode, iterate)
   float lr, beta1, beta2, eps, sigma_min;
 };
-
-// Points t with |t + 1/2 - mu| <= k sigma, clipped to [0, D-2]; a = b + 1 when empty.
-__device__ __forceinline__ void window(float mu, float sg, float k, int D, int &a, int &b) {
-  float lo = ceilf(mu - k * sg - 0.5f), hi = floorf(mu + k * sg - 0.5f);
-  lo = fminf(fmaxf(lo, 0.0f), (float)(D - 1));
-  hi = fminf(fmaxf(hi, -1.0f), (float)(D - 2));
-  a = (int)lo;
-  b = (int)hi;
-}
-
-// Phi(z) from the Mills ratio: the upper tail Q(|z|) = exp(-z^2/2) P(|z|)/Q(|z|)
-// (rational fit of mills_ratio.h, |z| <= 12), absolute error ~1e-6.  Used for
-// the neighbour values of the edge terms, which only need absolute accuracy.
-__device__ __forceinline__ float cdf_fast(float z) {
-  const float x = fabsf(z);
-  const float e = __expf(-0.5f * z * z);
-  const float num = (((kMillsP[4] * x + kMillsP[3]) * x + kMillsP[2]) * x + kMillsP[1]) * x + kMillsP[0];
-  const float den = ((((kMillsQ[5] * x + kMillsQ[4]) * x + kMillsQ[3]) * x + kMillsQ[2]) * x + kMillsQ[1]) * x + 1.0f;
-  const float q = e * __fdividef(num, den);
-  return z <= 0.f ? q : 1.0f - q;
-}
-
-// Windowed CDF of a neighbour at integer point x.
-__device__ __forceinline__ float cdf_at(int x, float mu, float inv_s, int a, int b) {
-  if (x < a) return 0.0f;
-  if (x > b) return 1.0f;
-  return cdf_fast(((float)x + 0.5f - mu) * inv_s);
-}
-
-__device__ __forceinline__ int fold_bin(int d, int II) { return II > 0 ? d % II : d; }
-
-// A restart's (mu, sigma) is usable when both are finite and sigma >= 1e-30, so
-// that 1/sigma is finite.
-__device__ __forceinline__ bool usable(float mu, float sg) {
-  return isfinite(mu) && isfinite(sg) && sg >= 1e-30f;
-}
-
-constexpr float kInvSqrt2Pi = 0.3989422804014327f;
-constexpr float kInvSqrt2 = 0.7071067811865476f;
-
-// Bin mass of bin p of a window from the tail values (z, q = Q(|z|)) of points p
-// and p - 1: P = C(a+p) - C(a+p-1), with C = 0 below the window and 1 above it,
-// choosing the subtraction that keeps both tails relatively accurate.
-__device__ __forceinline__ float bin_mass(bool pt, bool first, float zc, float qc, float zp, float qp) {
-  const float c_cur = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;
-  const float c_prev = first ? 0.0f : (zp <= 0.f ? qp : 1.0f - qp);
-  float P = c_cur - c_prev;
-  P = (pt && !first && zc <= 0.f) ? qc - qp : P;
-  P = (pt && !first && zp > 0.f) ? qp - qc : P;
-  P = (pt && !first && zp <= 0.f && zc > 0.f) ? (0.5f - qc) + (0.5f - qp) : P;
-  P = (!pt && !first && zp > 0.f) ? qp : P;  // top bin: upper tail Q directly
-  return P;
-}
-
-// Adds round(w P 2^32) to a histogram cell as two exact 16-bit halves, using
-// 32-bit conversions only (float -> 64-bit integer conversion runs at the FP64 rate).
-__device__ __forceinline__ void hist_add(unsigned *hlo, unsigned *hhi, int cell, float wP) {
-  const float xs = fmaxf(wP, 0.0f) * 65536.0f;
-  const float fh = floorf(xs);
-  atomicAdd(&hlo[cell], __float2uint_rn((xs - fh) * 65536.0f));
-  atomicAdd(&hhi[cell], (unsigned)fh);
-}
 
 __device__ __forceinline__ float warp_sum(float x) {
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
