@@ -201,8 +201,40 @@ gaus_status gaus_round(gaus_ctx *ctx, const float *mu, int32_t *sched);
  * of gaus_report, written.  Integer arithmetic only. */
 gaus_status gaus_verify(gaus_ctx *ctx, const int32_t *sched, gaus_report *rep);
 
+/* Expected usage per resource class without allocating device memory.
+ *
+ * For callers that cannot call cudaMalloc -- code that runs inside a memory pool
+ * or arena owned by another framework, allocation-free real-time loops, or hosts
+ * whose device memory is budgeted before this library is used.  It needs no
+ * context: the caller passes device arrays it already owns, and the only working
+ * memory is a fixed 16 MiB array that the library keeps in device globals on every
+ * GPU that loads it, until the process exits.  The paper has no counterpart; this
+ * is the usage reduction of gaus_loss_grad offered on its own.
+ *
+ *   usage[b, c, t] = sum over nodes v of class c of demand[v] * P_v^d, summed over the
+ *   bins d with d mod II = t (t < II) when II > 0, else d = t (t < D),
+ * with P the bin masses of Eq. round truncated to +-window_k * sigma, exactly as
+ * gaus_loss_grad computes them (exact fixed-point sums, deterministic).
+ *   mu, sigma (V, B) fp32, res_class (V) int32 in 0..C-1, demand (V) int32 in
+ *   0..64 or NULL (= 1): DEVICE pointers, read only.
+ *   usage (B, C, II or D) fp64 DEVICE pointer, written.
+ *   cuda_stream: cudaStream_t of the work (NULL = legacy default stream).
+ * Limits: (II or D) * min(B, 32) <= 25,600; at most 1,024 (restart group, class)
+ * pairs with groups of 32 restarts; the partial histograms of all blocks must fit
+ * in the 16 MiB array (EINVAL with a message otherwise, nothing enqueued).  A
+ * restart whose mean or sigma is non-finite (or sigma < 1e-30) contributes nothing.
+ * The first call on a device looks up the array's device address and sets the
+ * kernel's shared-memory limit; make that first call before any stream capture.
+ * Every call shares the array: calls whose work overlaps on the GPU race and give
+ * undefined results.  No cudaMalloc, cudaFree or allocating library routine is
+ * called.  Errors: EINVAL, ECUDA (message in gaus_last_error(NULL)). */
+gaus_status gaus_expected_usage_noalloc(const float *mu, const float *sigma, const int32_t *res_class,
+                                        const int32_t *demand, int32_t V, int32_t B, int32_t C, int32_t D,
+                                        int32_t II, float window_k, double *usage, void *cuda_stream);
+
 /* Message of the last error on this context ("" if none), or with ctx = NULL the
- * message of this thread's last failed gaus_create.  Valid until the next call. */
+ * message of this thread's last failed gaus_create or gaus_expected_usage_noalloc.
+ * Valid until the next call. */
 const char *gaus_last_error(const gaus_ctx *ctx);
 
 /* Release the context and its device memory (synchronises its stream). */

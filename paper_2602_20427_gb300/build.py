@@ -12,7 +12,7 @@ CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libgaus.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["gaus_api.cu", "gaus_plan.cpp"]
+SOURCES = ["gaus_api.cu", "gaus_plan.cpp", "gaus_noalloc.cu"]
 
 
 def _nvcc() -> str:

@@ -290,6 +290,11 @@ void drop_graph(gaus_ctx *ctx) {
 
 }  // namespace
 
+namespace gaus {
+// Message for gaus_last_error(NULL) from entry points that have no context.
+void set_thread_error(const std::string &msg) { g_create_error = msg; }
+}  // namespace gaus
+
 extern "C" {
 
 gaus_status gaus_default_hparams(gaus_hparams *hp) {
