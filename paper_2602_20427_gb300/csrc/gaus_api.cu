@@ -106,6 +106,21 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   FwdKernel kf = pick_fwd(on, P.II);
   kf<<<ctx->nblk, kFwdThreads, ctx->smem_fwd, st>>>(A);
   CK(cudaGetLastError(), "k_fwd launch");
+  const bool reg = on & GAUS_REG_OBJ;
+  RegArgs RA;
+  if (reg) {
+    RA.mu = mu; RA.sg = sg;
+    RA.V = P.V; RA.B = P.B; RA.D = P.D; RA.II = P.II; RA.Dh = P.Dh; RA.RB = ctx->RBr; RA.G = ctx->Gr;
+    RA.k_win = ctx->hp.window_k; RA.perm = ctx->d_perm; RA.bits = ctx->d_bits;
+    RA.out_ptr = ctx->d_out_ptr; RA.out_dst = ctx->d_out_dst; RA.seg = ctx->d_seg; RA.win = ctx->d_win;
+    RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gpart = ctx->d_gpart; RA.eslot = ctx->d_eslot;
+    k_reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
+    CK(cudaGetLastError(), "k_reg_fwd launch");
+    const int per = 256 / ctx->RBr;
+    k_reduce_reg<<<ctx->Gr * ((P.Dh + per - 1) / per), 256, 0, st>>>(ctx->d_rpart, ctx->d_Ureg, P.B, P.Dh,
+                                                                     ctx->RBr, ctx->Gr, P.nseg);
+    CK(cudaGetLastError(), "k_reduce_reg launch");
+  }
   RedArgs R;
   R.B = P.B; R.C = P.C; R.Dh = P.Dh; R.RB = ctx->RB; R.G = ctx->G;
   R.cls_seg_ptr = ctx->d_cls_seg_ptr; R.hpart = ctx->d_hpart; R.hspan = ctx->d_hspan; R.U = ctx->d_U;
@@ -115,6 +130,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
 
   FinArgs F;
   F.B = P.B; F.C = P.C; F.Dh = P.Dh; F.RB = ctx->RB; F.G = ctx->G; F.Ug = ctx->d_U;
+  F.Ureg = reg ? ctx->d_Ureg : nullptr; F.Hreg = ctx->d_Hreg;
   F.terms = on; F.tau = ctx->hp.tau; F.rho = ctx->hp.rho; F.alpha = ctx->hp.alpha;
   F.w_res = ctx->hp.w_res; F.w_mem = ctx->hp.w_mem;
   F.cls_seg_ptr = ctx->d_cls_seg_ptr; F.limit = ctx->d_limit;
@@ -124,9 +140,14 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   F.status = status; F.nonfinite = ctx->d_nonfinite;
   k_finalize<<<P.B, 256, ctx->smem_fin, st>>>(F);
   CK(cudaGetLastError(), "k_finalize launch");
+  if (reg) {
+    k_reg_bwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rbwd, st>>>(RA);
+    CK(cudaGetLastError(), "k_reg_bwd launch");
+  }
   if (ev) CK(cudaEventRecord(ev[2], st), "event");
 
   UpdArgs U;
+  U.in_ptr = ctx->d_in_ptr; U.in_eslot = ctx->d_in_eslot; U.eslot = reg ? ctx->d_eslot : nullptr;
   U.mu = const_cast<float *>(mu); U.sg = const_cast<float *>(sg);
   U.V = P.V; U.B = P.B; U.D = P.D; U.II = P.II; U.Dh = P.Dh; U.C = P.C; U.RB = ctx->RB; U.G = ctx->G;
   U.k_win = ctx->hp.window_k; U.perm = ctx->d_perm; U.w = ctx->d_w; U.seg = ctx->d_seg;
@@ -162,10 +183,16 @@ gaus_status set_smem_attrs(gaus_ctx *ctx) {
     CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_upd), "smem attr upd");
   CK(cudaFuncSetAttribute((const void *)k_finalize, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fin),
      "smem attr fin");
+  CK(cudaFuncSetAttribute((const void *)k_reg_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_rfwd),
+     "smem attr reg fwd");
+  CK(cudaFuncSetAttribute((const void *)k_reg_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_rbwd),
+     "smem attr reg bwd");
   CK(cudaFuncSetAttribute((const void *)k_verify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_ver),
      "smem attr ver");
   return GAUS_OK;
 }
+
+gaus_status alloc_storage_scratch(gaus_ctx *ctx);
 
 gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   // Validate and plan on the host first: argument and graph errors never touch CUDA.
@@ -177,7 +204,6 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   if (st != GAUS_OK) { ctx->err = err; return st; }
   Plan &P = ctx->plan;
   if ((ctx->hp.terms & GAUS_REC) && P.II <= 0) { ctx->err = "GAUS_REC needs II > 0"; return GAUS_EINVAL; }
-  if (ctx->hp.terms & GAUS_REG_OBJ) { ctx->err = "GAUS_REG_OBJ is not available in this build"; return GAUS_EINVAL; }
   if (!have_dev) {
     cudaGetLastError();
     ctx->err = "no CUDA device";
@@ -204,9 +230,24 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     return GAUS_EINVAL;
   }
   ctx->kc = kc;
+  // storage-term kernels: their own restarts-per-row so that the storage histogram
+  // (two u32 halves), its difference array and constants fit in shared memory
+  ctx->RBr = ctx->RB;
+  auto rfwd_bytes = [&](int rb) {
+    return (2 * (size_t)P.Dh * rb + (size_t)(P.Dh + 1) * rb + rb) * sizeof(unsigned);
+  };
+  while (ctx->RBr > 1 && rfwd_bytes(ctx->RBr) > kMaxSmem - 1024) ctx->RBr >>= 1;
+  if (rfwd_bytes(ctx->RBr) > kMaxSmem - 1024) {
+    ctx->err = "storage histogram of this horizon/II does not fit in shared memory";
+    return GAUS_EINVAL;
+  }
+  ctx->Gr = (P.B + ctx->RBr - 1) / ctx->RBr;
+  ctx->nblk_r = P.nseg * ctx->Gr;
+  ctx->smem_rfwd = rfwd_bytes(ctx->RBr);
+  ctx->smem_rbwd = (size_t)P.Dh * ctx->RBr * sizeof(float);
   ctx->smem_fwd = hist + (size_t)kc * per_pt;
   ctx->smem_upd = (size_t)ctx->RB * P.Dh * sizeof(float);
-  ctx->smem_fin = (size_t)P.C * P.Dh * sizeof(double);
+  ctx->smem_fin = (size_t)(P.C + 1) * P.Dh * sizeof(double);
   ctx->smem_ver = ((size_t)P.C * P.Dh + (P.D + 1) + P.Dh) * sizeof(long long);
   if (ctx->smem_upd > kMaxSmem || ctx->smem_fin > kMaxSmem || ctx->smem_ver > kMaxSmem) {
     ctx->err = "histogram of this horizon/II does not fit in shared memory";
@@ -225,6 +266,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(upload(ctx, &ctx->d_in_lat, P.in_lat));
   TRY(upload(ctx, &ctx->d_out_ptr, P.out_ptr));
   TRY(upload(ctx, &ctx->d_out_dst, P.out_dst));
+  TRY(upload(ctx, &ctx->d_in_eslot, P.in_eslot));
   TRY(upload(ctx, &ctx->d_bin_ptr, P.bin_ptr));
   TRY(upload(ctx, &ctx->d_bin_src, P.bin_src));
   TRY(upload(ctx, &ctx->d_bin_shift, P.bin_shift));
@@ -257,6 +299,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   const size_t VB = (size_t)P.V * P.B;
   TRY(scratch(ctx, &ctx->d_hpart, (size_t)ctx->nblk * ctx->RB * P.Dh));
   TRY(scratch(ctx, &ctx->d_U, (size_t)P.B * P.C * P.Dh));
+  if (ctx->hp.terms & GAUS_REG_OBJ) TRY(alloc_storage_scratch(ctx));
   TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
   TRY(scratch(ctx, &ctx->d_fwd, (size_t)ctx->nblk * ctx->RB * 3));
   TRY(scratch(ctx, &ctx->d_gpart, 6 * VB));
@@ -268,6 +311,17 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_loss_tmp, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_terms_tmp, (size_t)P.B * GAUS_NT));
   CK(cudaDeviceSynchronize(), "setup sync");
+  return GAUS_OK;
+}
+
+// Scratch of the storage term (also allocated when the term is switched on later).
+gaus_status alloc_storage_scratch(gaus_ctx *ctx) {
+  if (ctx->d_rpart) return GAUS_OK;
+  const Plan &P = ctx->plan;
+  TRY(scratch(ctx, &ctx->d_rpart, (size_t)ctx->nblk_r * P.Dh * ctx->RBr));
+  TRY(scratch(ctx, &ctx->d_Ureg, (size_t)P.B * P.Dh));
+  TRY(scratch(ctx, &ctx->d_Hreg, (size_t)P.B * P.Dh));
+  TRY(scratch(ctx, &ctx->d_eslot, (size_t)std::max(1, P.E) * P.B));
   return GAUS_OK;
 }
 
@@ -343,7 +397,10 @@ gaus_status gaus_set_hparams(gaus_ctx *ctx, const gaus_hparams *hp) {
   gaus_status st = check_hparams(hp, &ctx->err);
   if (st != GAUS_OK) return st;
   if ((hp->terms & GAUS_REC) && ctx->plan.II <= 0) { ctx->err = "GAUS_REC needs II > 0"; return GAUS_EINVAL; }
-  if (hp->terms & GAUS_REG_OBJ) { ctx->err = "GAUS_REG_OBJ is not available in this build"; return GAUS_EINVAL; }
+  if (hp->terms & GAUS_REG_OBJ) {
+    gaus_status st2 = alloc_storage_scratch(ctx);
+    if (st2 != GAUS_OK) return st2;
+  }
   ctx->hp = *hp;
   drop_graph(ctx);
   return GAUS_OK;

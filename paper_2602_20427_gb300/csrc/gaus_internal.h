@@ -36,6 +36,8 @@ struct Plan {
   std::vector<int32_t> in_ptr, in_src, in_lat;
   // CSR of internal producers: consumer caller id
   std::vector<int32_t> out_ptr, out_dst;
+  // CSR position of each internal in-edge (CSC order)
+  std::vector<int32_t> in_eslot;
   // back edges grouped by internal consumer i: producer caller id j, shift Lat(j) - k II
   std::vector<int32_t> bin_ptr, bin_src, bin_shift;
   // back edges grouped by internal producer j: consumer caller id i, same shift
@@ -71,6 +73,8 @@ struct gaus_ctx {
   int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per pass
   int kc = 0;                    // own-window points cached per thread in k_fwd
   int red_blocks = 0;
+  int RBr = 32, Gr = 1, nblk_r = 0;  // storage-term kernels: restarts per row, groups, blocks
+  size_t smem_rfwd = 0, smem_rbwd = 0;
   size_t smem_fwd = 0, smem_upd = 0, smem_fin = 0, smem_ver = 0;
   // device graph
   int32_t *d_perm = nullptr;
@@ -94,6 +98,11 @@ struct gaus_ctx {
   int2 *d_hspan = nullptr;       // nblk folded bin span written by each block
   double *d_fwd = nullptr;       // nblk * RB * 3 forward sums (dep, com, rec)
   double *d_U = nullptr;         // B * C * Dh usage (k_reduce)
+  long long *d_rpart = nullptr;  // nblk_r * Dh * RBr storage partials
+  double *d_Ureg = nullptr;      // B * Dh expected (folded) storage
+  float *d_Hreg = nullptr;       // B * Dh storage adjoint
+  float2 *d_eslot = nullptr;     // E * B successor shares of the storage gradient
+  int32_t *d_in_eslot = nullptr; // E
   float *d_gpart = nullptr;      // 6 * V * B partial gradient sums (internal index)
   unsigned *d_win = nullptr;     // V * B packed windows (caller order)
   float *d_H = nullptr;          // B * C * Dh usage adjoint dL/dU

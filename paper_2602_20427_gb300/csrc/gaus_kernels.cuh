@@ -23,6 +23,7 @@
 
 #include "gaus_device.cuh"
 #include "gaus_internal.h"
+#include "gaus_reg.cuh"
 
 namespace gaus {
 
@@ -57,6 +58,8 @@ struct RedArgs {
 struct FinArgs {
   int B, C, Dh, RB, G;
   const double *Ug;   // (B, C, Dh) usage from k_reduce
+  const double *Ureg; // (B, Dh) storage, or NULL when the storage term is off
+  float *Hreg;        // (B, Dh) storage adjoint
   unsigned terms;
   float tau, rho, alpha, w_res, w_mem;
   const int32_t *cls_seg_ptr;
@@ -72,6 +75,8 @@ struct FinArgs {
 };
 
 struct UpdArgs {
+  const int32_t *in_ptr, *in_eslot;  // storage term: successor shares gathered per in-edge
+  const float2 *eslot;               // NULL when the storage term is off
   float *mu, *sg;  // caller order; written when adam
   int V, B, D, II, Dh, C, RB, G;
   float k_win;
@@ -627,6 +632,25 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   }
   __syncthreads();
 
+  // LogSumExp of the (folded) expected storage, Eq. max over Eq. active
+  double reg_lse = 0.0, reg_m = 0.0, reg_s = 1.0;
+  if (A.Ureg) {
+    double *R = U + (size_t)A.C * Dh;
+    for (int t = tid; t < Dh; t += 256) R[t] = A.Ureg[(size_t)b * Dh + t];
+    __syncthreads();
+    double m = -1e300;
+    for (int t = tid; t < Dh; t += 256) m = fmax(m, R[t]);
+    m = block_max(m, buf);
+    double sacc = 0.0;
+    for (int t = tid; t < Dh; t += 256) sacc += (double)expf((float)((R[t] - m) / A.tau));
+    sacc = block_sum(sacc, buf);
+    reg_m = m;
+    reg_s = sacc;
+    reg_lse = m + (double)A.tau * log(sacc);
+    for (int t = tid; t < Dh; t += 256)
+      A.Hreg[(size_t)b * Dh + t] = (float)((double)A.w_mem * (double)expf((float)((R[t] - m) / A.tau)) / sacc);
+  }
+
   const bool on_dep = A.terms & GAUS_DEP, on_com = A.terms & GAUS_COM;
   const bool on_robj = A.terms & GAUS_RES_OBJ, on_rv = A.terms & GAUS_RES_VIOL;
   const bool on_rec = A.terms & GAUS_REC;
@@ -636,6 +660,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
     double L = 0.0;
     if (on_robj) L += (double)A.w_res * lse_sum;
     if (on_com) L += (double)A.alpha * lcom;
+    if (A.Ureg) L += (double)A.w_mem * reg_lse;
     const double Vk[3] = {on_dep ? vdep : 0.0, on_rv ? vres : 0.0, on_rec ? vrec : 0.0};
     const bool act[3] = {on_dep, on_rv, on_rec};
     for (int k = 0; k < 3; ++k)
@@ -643,7 +668,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
     float *T = A.terms_out + (size_t)b * GAUS_NT;
     T[GAUS_T_RES] = on_robj ? (float)lse_sum : 0.f;
     T[GAUS_T_COM] = on_com ? (float)lcom : 0.f;
-    T[GAUS_T_REG] = 0.f;
+    T[GAUS_T_REG] = A.Ureg ? (float)reg_lse : 0.f;
     T[GAUS_T_VDEP] = (float)Vk[0];
     T[GAUS_T_VRES] = (float)Vk[1];
     T[GAUS_T_VREC] = (float)Vk[2];
@@ -708,8 +733,14 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
         Bh += gh * z * f;
       }
     }
-    const float Asum = c_dep * A.gpart[0 * VB + gi] + A.gpart[2 * VB + gi] + c_rec * A.gpart[4 * VB + gi] + Ah;
-    const float Bsum = c_dep * A.gpart[1 * VB + gi] + A.gpart[3 * VB + gi] + c_rec * A.gpart[5 * VB + gi] + Bh;
+    float Asum = c_dep * A.gpart[0 * VB + gi] + A.gpart[2 * VB + gi] + c_rec * A.gpart[4 * VB + gi] + Ah;
+    float Bsum = c_dep * A.gpart[1 * VB + gi] + A.gpart[3 * VB + gi] + c_rec * A.gpart[5 * VB + gi] + Bh;
+    if (A.eslot && ok)
+      for (int e = A.in_ptr[vi]; e < A.in_ptr[vi + 1]; ++e) {
+        const float2 sh = A.eslot[(size_t)A.in_eslot[e] * A.B + b];
+        Asum += sh.x;
+        Bsum += sh.y;
+      }
     // dC/dmu = -phi/sigma, dC/dsigma = -z phi/sigma
     const float gm = ok ? -Asum / sg : 0.f, gs = ok ? -Bsum / sg : 0.f;
     if (!kAdam) {

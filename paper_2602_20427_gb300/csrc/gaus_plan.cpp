@@ -177,6 +177,31 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
     o = P.out_ptr[i];
     for (int q = p->succ_ptr[v]; q < p->succ_ptr[v + 1]; ++q, ++o) P.out_dst[o] = p->succ_idx[q];
   }
+  // CSC position of every in-edge -> CSR position of the same edge in its
+  // producer's out-list (per-edge slots written by producers, read by consumers)
+  {
+    std::vector<int64_t> key(E);
+    std::vector<int32_t> pos(E);
+    for (int i = 0; i < V; ++i)
+      for (int o = P.out_ptr[i]; o < P.out_ptr[i + 1]; ++o) {
+        key[o] = (int64_t)P.perm[i] * V + P.out_dst[o];
+        pos[o] = o;
+      }
+    std::vector<int32_t> idx(E);
+    std::iota(idx.begin(), idx.end(), 0);
+    std::sort(idx.begin(), idx.end(), [&](int x, int y) { return key[x] < key[y]; });
+    P.in_eslot.resize(E);
+    for (int i = 0; i < V; ++i)
+      for (int e = P.in_ptr[i]; e < P.in_ptr[i + 1]; ++e) {
+        const int64_t k = (int64_t)P.in_src[e] * V + P.perm[i];
+        int lo = 0, hi = E - 1;
+        while (lo < hi) {
+          const int mid = (lo + hi) / 2;
+          if (key[idx[mid]] < k) lo = mid + 1; else hi = mid;
+        }
+        P.in_eslot[e] = pos[idx[lo]];
+      }
+  }
   // back edges: shift = Lat(j) - k II (a back edge acts as a dependency with that latency)
   P.bin_ptr.assign(V + 1, 0);
   P.bout_ptr.assign(V + 1, 0);

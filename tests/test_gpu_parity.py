@@ -215,3 +215,44 @@ def test_mixed_window_lengths_short_and_cooperative_paths(g):
     sg = np.exp(rng.uniform(np.log(0.05), np.log(6.0), size=(p.V, B))).astype(np.float32)
     hp = g.default_hparams(terms=p.terms, rho=1e-3)
     check_loss_grad(p, g, B, mu, sg, _lam(B, rng), hp, restarts=range(0, 32, 4))
+
+
+# ---------------------------------------------------------------- storage term (Eq. active)
+def test_storage_term_regular_small(g):
+    p = W.random_small(31, V=40, D=30, C=2, max_lat=2, p_edge=0.12)
+    p.terms = W.DEP | W.REG_OBJ
+    rng = np.random.default_rng(31)
+    B = 8
+    mu = (p.start[:, None] + rng.normal(0, 2, size=(p.V, B))).astype(np.float32)
+    sg = rng.uniform(0.3, 2.5, size=(p.V, B)).astype(np.float32)
+    hp = g.default_hparams(terms=p.terms, tau=0.3, w_mem=1.7)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, rng), hp)
+
+
+def test_storage_term_wide_layered_small(g):
+    p = W.wide_layered(4, width=60, levels=12)
+    B = 16
+    mu, sg = W.init_state(p, B, 11)
+    hp = g.default_hparams(terms=p.terms, rho=1e-3)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, np.random.default_rng(11)), hp, restarts=[0, 7, 15])
+
+
+@pytest.mark.parametrize("factor", [1.0, 1.5])
+def test_formulation_c_modulo_storage(g, factor):
+    p = W.modulo_loop(7, ii_factor=factor, V=300, levels=15, n_back=15)
+    p.terms = W.DEP | W.RES_VIOL | W.REG_OBJ | W.REC
+    B = 8
+    mu, sg = W.init_state(p, B, 12)
+    hp = g.default_hparams(terms=p.terms, rho=1e-3)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, np.random.default_rng(12)), hp, restarts=[0, 3, 7])
+
+
+def test_wide_layered_full_size_sampled_storage(g):
+    # the wide workload at its full size (V = 50,000, B = 16) with the storage and
+    # usage terms; the oracle checks two restarts
+    p = W.wide_layered(1)
+    p.terms = W.RES_OBJ | W.RES_VIOL | W.REG_OBJ
+    mu, sg = W.init_state(p, 16, 1)
+    hp = g.default_hparams(terms=p.terms)
+    lam = np.full((16, 3), 1e-6, np.float32)
+    check_loss_grad(p, g, 16, mu, sg, lam, hp, restarts=[0, 9])
