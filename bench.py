@@ -1,12 +1,13 @@
 #!/usr/bin/env python
 """GauS hot-path benchmark: fused loss + gradient + Adam iterations/s x B restarts.
 
-One step = `--inner` fused iterations (gaus_iterate: loss, gradient, Adam,
-multiplier update; Sec. 3.3, Alg. GauS) followed by one round + legalize
-(App. A) and one verify (Sec. 2.1) of all B restarts -- one outer period of
-Alg. GauS.  The default run (20 steps of 100 iterations) is the 2,000-iteration
-trajectory of the logic-network workload (V = 10,000, B = 64) from its seeded
-initial state.
+One step = one complete batched solve of Alg. GauS on the logic-network
+workload (V = 10,000, B = 64 restarts) from its seeded initial state: the state
+is initialised (means and deviations copied in, Adam moments and step zeroed,
+multipliers set to lambda_0), then `--iters` fused iterations (gaus_iterate:
+loss, gradient, Adam, multiplier update; Sec. 3.3) run, with a round + legalize
+(App. A) and a verify (Sec. 2.1) of all B restarts every `--period` iterations.
+Every step does the same work, so the number does not depend on --steps.
 
 Prints one JSON line.  `--impl reference` times the fp64 CPU oracle on the same
 workload and metric (bounded sample per step).
@@ -40,9 +41,10 @@ SM_MAX_MHZ = 2070.0
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--inner", type=int, default=100, help="fused iterations per step")
+    ap.add_argument("--iters", type=int, default=2000, help="fused iterations per solve (one step)")
+    ap.add_argument("--period", type=int, default=100, help="iterations between legalize + verify")
     ap.add_argument("--impl", default="gaus", choices=["gaus", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -56,11 +58,12 @@ def workload(rank=0):
     return p, B, mu, sg
 
 
-def describe(p, B, iters):
+def describe(p, B, iters, period=None):
     return {"workload": f"{p.name}: AND/INV logic network, V={p.V}, E={p.E}, depth 120, "
                         f"D={p.D}, 2 classes (AND limit 64, INV unlimited), unit latency, "
                         f"Formulation A terms (Res LSE + ReLU, Com, Dep)",
             "B": B, "V": p.V, "E": p.E, "D": p.D, "iterations_per_step": iters,
+            "legalize_verify_every": period,
             "init": "mu = ASAP + N(0, 2), sigma = 1.5 (seeded)", "tau": 1e-2, "rho": 1e-4, "lr": 1e-2,
             "window_k": 6.0}
 
@@ -166,27 +169,39 @@ def gpu_arm(args):
     p, B, mu0, sg0 = workload(rank)
     hp = g.default_hparams(terms=p.terms)
     ctx = g.Gaus(p, B, hp)
-    inner = args.inner
+    iters, period = args.iters, args.period
+    assert iters % period == 0, "--iters must be a multiple of --period"
     dmu0, dsg0 = torch.from_numpy(mu0).cuda(), torch.from_numpy(sg0).cuda()
     st = ctx.new_state(dmu0, dsg0, hp.lambda0)
     sched = torch.empty((p.V, B), dtype=torch.int32, device="cuda")
     lstat = torch.empty(B, dtype=torch.int32, device="cuda")
     rep = torch.empty(B * 200, dtype=torch.uint8, device="cuda")
+    reg = bool(p.terms & W.REG_OBJ)
+    launches_per_iter = 5 + (3 if reg else 0)   # windows, fwd, [reg fwd, reg reduce], reduce, finalize, [reg bwd], update
+    launches_per_step = iters * launches_per_iter + (iters // period) * 2
 
-    def reset():
-        fresh = ctx.new_state(dmu0, dsg0, hp.lambda0)
-        for kk, v in fresh.items():
-            st[kk].copy_(v)
+    def init_state(mu_src, sg_src):
+        st["mu"].copy_(mu_src, non_blocking=True)
+        st["sigma"].copy_(sg_src, non_blocking=True)
+        for kk in ("m_mu", "v_mu", "m_sigma", "v_sigma", "loss", "terms"):
+            st[kk].zero_()
+        st["step"].zero_()
+        st["status"].zero_()
+        st["lambda_"].fill_(hp.lambda0)
+
+    def solve():
+        for _ in range(iters // period):
+            ctx.iterate(period, st)
+            ctx.legalize(st["mu"], sched, lstat)
+            ctx.verify_raw(sched, rep)
 
     def step():
-        ctx.iterate(inner, st)
-        ctx.legalize(st["mu"], sched, lstat)
-        ctx.verify_raw(sched, rep)
+        init_state(dmu0, dsg0)
+        solve()
 
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
-    reset()
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device="cuda")
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     gpu_id = None
@@ -210,41 +225,79 @@ def gpu_arm(args):
     torch.cuda.synchronize()
     wall = time.perf_counter() - wall0
     clocks = sampler.stop() if sampler else None
-    ms = sum(a.elapsed_time(b) for a, b in evs)
+    step_ms = [a.elapsed_time(b) for a, b in evs]
+    ms = sum(step_ms)
     if world > 1:
         dist.barrier()
         t = torch.tensor([ms], dtype=torch.float64, device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     status_ok = bool(int(st["status"].abs().sum()) == 0)
-    units = args.steps * inner * B * world
+    feasible = int((lstat == 0).sum())
+    units = args.steps * iters * B * world
     value = units / (ms / 1e3)
 
-    # ---- kernel-level timing and algorithmic work along the same trajectory
-    reset()
+    # ---- legalize + verify alone (part of every step above; reported separately)
+    lv = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    lv[0].record()
+    for _ in range(10):
+        ctx.legalize(st["mu"], sched, lstat)
+        ctx.verify_raw(sched, rep)
+    lv[1].record()
+    torch.cuda.synchronize()
+    legalize_verify_ms = lv[0].elapsed_time(lv[1]) / 10
+
+    # ---- phase timing and algorithmic work along one solve (no graph, events between phases)
+    init_state(dmu0, dsg0)
     src = torch.from_numpy(np.asarray(p.src, np.int64)).cuda()
     dst = torch.from_numpy(np.asarray(p.dst, np.int64)).cuda()
-    k_ms = np.zeros(3)
+    ph_ms = np.zeros(4)
     flops_total, t_fwd_total, npt_total, neb_total = 0.0, 0.0, 0.0, 0.0
-    for k in range(args.steps):
+    fwd_first = fwd_last = None
+    nchunk = iters // period
+    for k in range(nchunk):
         f0, n0, e0 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
-        kms = np.array(ctx.profile_iterate(inner, st))
+        kms = np.array(ctx.profile_iterate(period, st))
         f1, n1, e1 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
-        k_ms += kms / args.steps
-        flops_total += inner * 0.5 * (f0 + f1)
-        npt_total += inner * 0.5 * (n0 + n1)
-        neb_total += inner * 0.5 * (e0 + e1)
-        t_fwd_total += inner * kms[0] * 1e-3
+        ph_ms += kms / nchunk
+        flops_total += period * 0.5 * (f0 + f1)
+        npt_total += period * 0.5 * (n0 + n1)
+        neb_total += period * 0.5 * (e0 + e1)
+        t_fwd_total += period * kms[1] * 1e-3
+        fwd_first = kms[1] if fwd_first is None else fwd_first
+        fwd_last = kms[1]
     achieved = flops_total / t_fwd_total / 1e12
     peak = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
     traffic = profiled_traffic()
 
+    # ---- steady state at fixed sigma: the initial state with lr = 1e-20 (an Adam step is
+    # at most ~lr, far below one ulp of mu or sigma, so the windows never shrink)
+    hp0 = g.default_hparams(terms=p.terms, lr=1e-20)
+    ctx0 = g.Gaus(p, B, hp0)
+    st0 = ctx0.new_state(dmu0, dsg0, hp0.lambda0)
+    ctx0.iterate(20, st0)
+    ev0 = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    n_fixed = 200
+    torch.cuda.synchronize()
+    ev0[0].record()
+    ctx0.iterate(n_fixed, st0)
+    ev0[1].record()
+    torch.cuda.synchronize()
+    fixed_ms = ev0[0].elapsed_time(ev0[1]) / n_fixed
+    fixed_ph = ctx0.profile_iterate(20, st0)
+    ctx0.close()
+    steady = {"value": B / (fixed_ms / 1e3), "unit": UNIT, "sigma": 1.5, "ms_per_iteration": fixed_ms,
+              "k_fwd_ms": fixed_ph[1],
+              "note": "initial state of the same workload with lr = 1e-20, so every iteration has the "
+                      "initial +-6 sigma windows (the most expensive point of the run)"}
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        reset()
         h_mu = torch.from_numpy(mu0.copy()).pin_memory()
         h_sg = torch.from_numpy(sg0.copy()).pin_memory()
+        h_mu_out = torch.empty_like(h_mu).pin_memory()
+        h_sg_out = torch.empty_like(h_sg).pin_memory()
         h_sched = torch.empty((p.V, B), dtype=torch.int32).pin_memory()
         h_rep = torch.empty(B * 200, dtype=torch.uint8).pin_memory()
         h_loss = torch.empty(B, dtype=torch.float32).pin_memory()
@@ -253,11 +306,10 @@ def gpu_arm(args):
         for k in range(args.steps):
             flush.fill_(k & 255)
             eev[k][0].record()
-            st["mu"].copy_(h_mu, non_blocking=True)
-            st["sigma"].copy_(h_sg, non_blocking=True)
-            step()
-            h_mu.copy_(st["mu"], non_blocking=True)
-            h_sg.copy_(st["sigma"], non_blocking=True)
+            init_state(h_mu, h_sg)                   # host -> device copies of the solve's inputs
+            solve()
+            h_mu_out.copy_(st["mu"], non_blocking=True)
+            h_sg_out.copy_(st["sigma"], non_blocking=True)
             h_sched.copy_(sched, non_blocking=True)
             h_rep.copy_(rep, non_blocking=True)
             h_loss.copy_(st["loss"], non_blocking=True)
@@ -282,18 +334,23 @@ def gpu_arm(args):
                 "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f32",
                 "data": "synthetic (seeded logic-network DAG and initial means)",
-                "config": dict(describe(p, B, inner), l2="flushed between steps (256 MB write)",
+                "config": dict(describe(p, B, iters, period), l2="flushed between steps (256 MB write)",
                                parallelism=f"restarts sharded, {world} replica(s)"),
-                "e2e": e2e, "gpu_launches": args.steps * (3 * inner + 2),
+                "e2e": e2e, "gpu_launches": args.steps * launches_per_step,
                 "clocks": clocks,
                 "roofline": {"bound": "alu", "kernel": "k_fwd (node + edge pass)", "achieved": achieved,
                              "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
                              "peak_note": "FP32: 152 SM x 128 lanes x 2 flop x 2070 MHz (max SM clock)",
                              "cost_model": "20 flop per CDF point + 8 flop per edge-bin",
-                             "points_per_iter": npt_total / (args.steps * inner),
-                             "edge_bins_per_iter": neb_total / (args.steps * inner)},
-                "kernel_ms": {"k_fwd": k_ms[0], "k_finalize": k_ms[1], "k_update": k_ms[2]},
-                "status_ok": status_ok, "wall_s": wall,
+                             "points_per_iter": npt_total / iters,
+                             "edge_bins_per_iter": neb_total / iters},
+                "phase_ms_per_iteration": {"k_windows": ph_ms[0], "k_fwd": ph_ms[1],
+                                           "reduce_finalize": ph_ms[2], "k_update": ph_ms[3],
+                                           "k_fwd_first_period": fwd_first, "k_fwd_last_period": fwd_last},
+                "legalize_verify_ms": legalize_verify_ms,
+                "steady_fixed_sigma": steady,
+                "step_ms": step_ms,
+                "status_ok": status_ok, "legalized_ok": feasible, "wall_s": wall,
                 "cpu_baseline": cpu}
         print(json.dumps(line))
     if world > 1:
@@ -368,7 +425,7 @@ def reference_arm(args):
                       "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
                       "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
                       "data": "synthetic (seeded logic-network DAG and initial means)",
-                      "config": dict(describe(p, B, 1), sample=sample),
+                      "config": dict(describe(p, B, args.iters, args.period), sample=sample),
                       "cpu_baseline": {"value": value, "unit": UNIT, "cores": int(os.environ["OMP_NUM_THREADS"]),
                                        "kind": "oracle", "sample": sample},
                       "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))

@@ -179,11 +179,12 @@ gaus_status gaus_adam_step(gaus_ctx *ctx, float *mu, float *sigma, const float *
 gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st);
 
 /* Kernel-level timing of gaus_iterate: runs n_iters iterations exactly as
- * gaus_iterate does, but launched one kernel at a time with a CUDA event
- * between kernels, and adds the mean duration in milliseconds of the three
- * kernels of an iteration to ms_out[0..2] (host array: node/edge pass,
- * per-restart finalize, gradient + Adam).  Synchronises the context's stream.
- * Library feature for measurement; not on the hot path. */
+ * gaus_iterate does, but launched without a graph and with CUDA events between
+ * the phases, and adds the mean duration in milliseconds of each phase of an
+ * iteration to ms_out[0..3] (host array of 4): [0] window table, [1] node/edge
+ * pass (k_fwd alone), [2] storage pass + usage reduction + per-restart finalize,
+ * [3] gradient gather + Adam.  Synchronises the context's stream.  Library
+ * feature for measurement; not on the hot path. */
 gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st, double *ms_out);
 
 /* Round every mean to s = floor(mu + 1/2) (Sec. 3.3 Sampling; exact for every

@@ -229,7 +229,8 @@ class Gaus:
         self._check(lib().gaus_iterate(self._ctx, C.c_int32(n), C.byref(s)))
 
     def profile_iterate(self, n, state):
-        """Mean per-kernel durations (ms) of n iterations: [node/edge, finalize, update]."""
+        """Mean per-phase durations (ms) of n iterations:
+        [window table, node/edge pass, reductions + finalize, gradient + Adam]."""
         torch = self.torch
         VB, f32 = (self.V, self.B), torch.float32
         s = State(*(self._dev(state[k], f32, VB).value for k in ("mu", "sigma", "m_mu", "v_mu", "m_sigma",
@@ -239,9 +240,9 @@ class Gaus:
                   self._dev(state["loss"], f32, (self.B,)).value,
                   self._dev(state["terms"], f32, (self.B, NT)).value,
                   self._dev(state["status"], torch.int32, (self.B,)).value)
-        ms = (C.c_double * 3)(0.0, 0.0, 0.0)
+        ms = (C.c_double * 4)(0.0, 0.0, 0.0, 0.0)
         self._check(lib().gaus_profile_iterate(self._ctx, C.c_int32(n), C.byref(s), ms))
-        return [ms[0], ms[1], ms[2]]
+        return list(ms)
 
     def round(self, mu, sched=None):
         torch = self.torch

@@ -103,9 +103,11 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
                                                                           ctx->hp.window_k, P.D);
     CK(cudaGetLastError(), "k_windows launch");
   }
+  if (ev) CK(cudaEventRecord(ev[1], st), "event");
   FwdKernel kf = pick_fwd(on, P.II);
   kf<<<ctx->nblk, kFwdThreads, ctx->smem_fwd, st>>>(A);
   CK(cudaGetLastError(), "k_fwd launch");
+  if (ev) CK(cudaEventRecord(ev[2], st), "event");
   const bool reg = on & GAUS_REG_OBJ;
   RegArgs RA;
   if (reg) {
@@ -116,9 +118,8 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
     RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gpart = ctx->d_gpart; RA.eslot = ctx->d_eslot;
     k_reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_fwd launch");
-    const int per = 256 / ctx->RBr;
-    k_reduce_reg<<<ctx->Gr * ((P.Dh + per - 1) / per), 256, 0, st>>>(ctx->d_rpart, ctx->d_Ureg, P.B, P.Dh,
-                                                                     ctx->RBr, ctx->Gr, P.nseg);
+    k_reduce_reg<<<ctx->Gr * P.Dh, 256, 0, st>>>(ctx->d_rpart, ctx->d_Ureg, P.B, P.Dh, ctx->RBr, ctx->Gr,
+                                                 P.nseg);
     CK(cudaGetLastError(), "k_reduce_reg launch");
   }
   RedArgs R;
@@ -126,7 +127,6 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   R.cls_seg_ptr = ctx->d_cls_seg_ptr; R.hpart = ctx->d_hpart; R.hspan = ctx->d_hspan; R.U = ctx->d_U;
   k_reduce<<<ctx->red_blocks, 256, 0, st>>>(R);
   CK(cudaGetLastError(), "k_reduce launch");
-  if (ev) CK(cudaEventRecord(ev[1], st), "event");
 
   FinArgs F;
   F.B = P.B; F.C = P.C; F.Dh = P.Dh; F.RB = ctx->RB; F.G = ctx->G; F.Ug = ctx->d_U;
@@ -136,6 +136,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   F.cls_seg_ptr = ctx->d_cls_seg_ptr; F.limit = ctx->d_limit;
   F.hpart = ctx->d_hpart; F.hspan = ctx->d_hspan; F.fwd = ctx->d_fwd;
   F.lambda = lambda; F.update_lambda = adam ? 1 : 0; F.step = adam ? S->step : nullptr;
+  F.beta1 = ctx->hp.beta1; F.beta2 = ctx->hp.beta2;
   F.H = ctx->d_H; F.coef = ctx->d_coef; F.loss = loss; F.terms_out = terms;
   F.status = status; F.nonfinite = ctx->d_nonfinite;
   k_finalize<<<P.B, 256, ctx->smem_fin, st>>>(F);
@@ -144,13 +145,13 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
     k_reg_bwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rbwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_bwd launch");
   }
-  if (ev) CK(cudaEventRecord(ev[2], st), "event");
+  if (ev) CK(cudaEventRecord(ev[3], st), "event");
 
   UpdArgs U;
   U.in_ptr = ctx->d_in_ptr; U.in_eslot = ctx->d_in_eslot; U.eslot = reg ? ctx->d_eslot : nullptr;
   U.mu = const_cast<float *>(mu); U.sg = const_cast<float *>(sg);
   U.V = P.V; U.B = P.B; U.D = P.D; U.II = P.II; U.Dh = P.Dh; U.C = P.C; U.RB = ctx->RB; U.G = ctx->G;
-  U.k_win = ctx->hp.window_k; U.perm = ctx->d_perm; U.w = ctx->d_w; U.seg = ctx->d_seg;
+  U.k_win = ctx->hp.window_k; U.perm = ctx->d_perm; U.win = ctx->d_win; U.w = ctx->d_w; U.seg = ctx->d_seg;
   U.gpart = ctx->d_gpart; U.H = ctx->d_H; U.coef = ctx->d_coef;
   U.grad_mu = grad_mu; U.grad_sg = grad_sg;
   U.m_mu = adam ? S->m_mu : nullptr; U.v_mu = adam ? S->v_mu : nullptr;
@@ -160,14 +161,14 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   U.sigma_min = ctx->hp.sigma_min;
   const bool hist = on & (GAUS_RES_OBJ | GAUS_RES_VIOL);
   if (adam) {
-    if (hist) k_update<true, true><<<ctx->nblk, kThreads, ctx->smem_upd, st>>>(U);
+    if (hist) k_update<true, true><<<ctx->nblk, kThreads, 0, st>>>(U);
     else k_update<true, false><<<ctx->nblk, kThreads, 0, st>>>(U);
   } else {
-    if (hist) k_update<false, true><<<ctx->nblk, kThreads, ctx->smem_upd, st>>>(U);
+    if (hist) k_update<false, true><<<ctx->nblk, kThreads, 0, st>>>(U);
     else k_update<false, false><<<ctx->nblk, kThreads, 0, st>>>(U);
   }
   CK(cudaGetLastError(), "k_update launch");
-  if (ev) CK(cudaEventRecord(ev[3], st), "event");
+  if (ev) CK(cudaEventRecord(ev[4], st), "event");
   return GAUS_OK;
 }
 
@@ -178,9 +179,6 @@ gaus_status set_smem_attrs(gaus_ctx *ctx) {
                        (const void *)k_fwd<false, false, true>, (const void *)k_fwd<false, false, false>};
   for (const void *f : fwd)
     CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fwd), "smem attr fwd");
-  const void *upd[] = {(const void *)k_update<true, true>, (const void *)k_update<false, true>};
-  for (const void *f : upd)
-    CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_upd), "smem attr upd");
   CK(cudaFuncSetAttribute((const void *)k_finalize, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fin),
      "smem attr fin");
   CK(cudaFuncSetAttribute((const void *)k_reg_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_rfwd),
@@ -213,10 +211,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   while (ctx->RB < P.B && ctx->RB < 32) ctx->RB <<= 1;
   ctx->G = (P.B + ctx->RB - 1) / ctx->RB;
   ctx->nblk = P.nseg * ctx->G;
-  {
-    const int per = 256 / ctx->RB;
-    ctx->red_blocks = ctx->G * P.C * ((P.Dh + per - 1) / per);
-  }
+  ctx->red_blocks = ctx->G * P.C * P.Dh;
   // k_fwd shared memory: the two histogram halves plus the own-window cache,
   // sized for two resident blocks per SM when the histogram allows it.
   const size_t hist = 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned);
@@ -493,24 +488,25 @@ gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_stat
     ctx->err = "gaus_profile_iterate: NULL pointer or n_iters < 0";
     return GAUS_EINVAL;
   }
-  std::vector<cudaEvent_t> ev(4 * (size_t)n_iters);
+  constexpr int kEv = 5;  // before k_windows, before / after k_fwd, after finalize, after update
+  std::vector<cudaEvent_t> ev(kEv * (size_t)n_iters);
   for (auto &e : ev) CK(cudaEventCreate(&e), "event create");
   gaus_status st = GAUS_OK;
   for (int i = 0; i < n_iters && st == GAUS_OK; ++i)
     st = enqueue_iteration(ctx, ctx->stream, S->mu, S->sigma, S->lambda, true, nullptr, nullptr, S->loss,
-                           S->terms, S->status, S, &ev[4 * (size_t)i]);
+                           S->terms, S->status, S, &ev[kEv * (size_t)i]);
   cudaError_t e = cudaStreamSynchronize(ctx->stream);
-  double acc[3] = {0, 0, 0};
+  double acc[kEv - 1] = {0, 0, 0, 0};
   for (int i = 0; i < n_iters && st == GAUS_OK && e == cudaSuccess; ++i)
-    for (int k = 0; k < 3; ++k) {
+    for (int k = 0; k < kEv - 1; ++k) {
       float ms = 0.f;
-      cudaEventElapsedTime(&ms, ev[4 * (size_t)i + k], ev[4 * (size_t)i + k + 1]);
+      cudaEventElapsedTime(&ms, ev[kEv * (size_t)i + k], ev[kEv * (size_t)i + k + 1]);
       acc[k] += ms;
     }
   for (auto &x : ev) cudaEventDestroy(x);
   if (st != GAUS_OK) return st;
   if (e != cudaSuccess) return cuda_fail(ctx, e, "profile sync");
-  for (int k = 0; k < 3; ++k) ms_out[k] += n_iters ? acc[k] / n_iters : 0.0;
+  for (int k = 0; k < kEv - 1; ++k) ms_out[k] += n_iters ? acc[k] / n_iters : 0.0;
   return GAUS_OK;
 }
 

@@ -96,10 +96,10 @@ struct gaus_ctx {
   // scratch
   long long *d_hpart = nullptr;  // nblk * Dh * RB fixed-point usage partials
   int2 *d_hspan = nullptr;       // nblk folded bin span written by each block
-  double *d_fwd = nullptr;       // nblk * RB * 3 forward sums (dep, com, rec)
-  double *d_U = nullptr;         // B * C * Dh usage (k_reduce)
+  long long *d_fwd = nullptr;    // nblk * RB * 3 forward sums (dep, com, rec), 2^32 fixed point
+  long long *d_U = nullptr;      // B * C * Dh usage (k_reduce), 2^32 fixed point
   long long *d_rpart = nullptr;  // nblk_r * Dh * RBr storage partials
-  double *d_Ureg = nullptr;      // B * Dh expected (folded) storage
+  long long *d_Ureg = nullptr;   // B * Dh expected (folded) storage, 2^32 fixed point
   float *d_Hreg = nullptr;       // B * Dh storage adjoint
   float2 *d_eslot = nullptr;     // E * B successor shares of the storage gradient
   int32_t *d_in_eslot = nullptr; // E

@@ -41,7 +41,7 @@ struct IterArgs {
   const int32_t *seg;
   long long *hpart;
   int2 *hspan;
-  double *fwd;
+  long long *fwd;
   float *gpart;
   int32_t *nonfinite;
   const unsigned *win;  // (V, B) packed windows: a | (b + 1) << 16
@@ -52,13 +52,13 @@ struct RedArgs {
   const int32_t *cls_seg_ptr;
   const long long *hpart;
   const int2 *hspan;
-  double *U;
+  long long *U;       // (B, C, Dh) usage, 2^32 fixed point
 };
 
 struct FinArgs {
   int B, C, Dh, RB, G;
-  const double *Ug;   // (B, C, Dh) usage from k_reduce
-  const double *Ureg; // (B, Dh) storage, or NULL when the storage term is off
+  const long long *Ug;   // (B, C, Dh) usage from k_reduce, 2^32 fixed point
+  const long long *Ureg; // (B, Dh) storage, or NULL when the storage term is off
   float *Hreg;        // (B, Dh) storage adjoint
   unsigned terms;
   float tau, rho, alpha, w_res, w_mem;
@@ -66,10 +66,11 @@ struct FinArgs {
   const float *limit;
   const long long *hpart;
   const int2 *hspan;
-  const double *fwd;
+  const long long *fwd;
   float *lambda;      // read; updated in place when update_lambda
   int update_lambda;
   int32_t *step;      // incremented when not NULL
+  float beta1, beta2; // Adam, for the bias corrections written to coef[2], coef[3]
   float *H, *coef, *loss, *terms_out;
   int32_t *status, *nonfinite;
 };
@@ -81,6 +82,7 @@ struct UpdArgs {
   int V, B, D, II, Dh, C, RB, G;
   float k_win;
   const int32_t *perm;
+  const unsigned *win;  // (V, B) packed windows of the state being updated
   const float *w;
   const int32_t *seg;
   const float *gpart;
@@ -90,6 +92,36 @@ struct UpdArgs {
   const int32_t *step_dev;                   // per-restart step (Adam mode, iterate)
   float lr, beta1, beta2, eps, sigma_min;
 };
+
+// round(x 2^32) for a forward sum x >= 0 of one item, with 32-bit conversions only.
+__device__ __forceinline__ long long to_fix(float x) {
+  const float xs = fmaxf(x, 0.0f) * 65536.0f;
+  const float fh = floorf(xs);
+  return ((long long)(unsigned)fh << 16) + (long long)__float2uint_rn((xs - fh) * 65536.0f);
+}
+
+// Mean window length (points) of restart b over the nodes s0..s1 of a segment,
+// from the windows table; rows threads per restart.  It sees restart b's data
+// only, so the split of items between the per-lane and the cooperative path --
+// and with it every rounding -- does not depend on the other restarts.  The
+// caller zeroes s_sum / s_cnt and synchronises before the call.
+__device__ __forceinline__ int seg_mean_window(const unsigned *win, const int32_t *perm, int s0, int s1, int b,
+                                               bool bok, int B, int tid, int RB, int rows, int *s_sum, int *s_cnt) {
+  int sum = 0, cnt = 0;
+  if (bok)
+    for (int vi = s0 + tid / RB; vi < s1; vi += rows) {
+      const unsigned w = win[(size_t)perm[vi] * B + b];
+      const int n = (int)(w >> 16) - (int)(w & 0xffffu);
+      if (n > 0) { sum += min(n, 4096); ++cnt; }
+    }
+  if (cnt) {
+    atomicAdd(&s_sum[tid % RB], sum);
+    atomicAdd(&s_cnt[tid % RB], cnt);
+  }
+  __syncthreads();
+  const int c = s_cnt[tid % RB];
+  return c ? s_sum[tid % RB] / c : 0;
+}
 
 __device__ __forceinline__ float warp_sum(float x) {
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
@@ -210,19 +242,23 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
   float *cC = reinterpret_cast<float *>(hhi + (size_t)Dh * RB);
   float *cF = cC + (size_t)kc * T;
   float *cZ = cF + (size_t)kc * T;
-  __shared__ int s_lo, s_hi, s_next;
+  __shared__ int s_lo, s_hi, s_next, s_wsum[32], s_wcnt[32];
 
   const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
   const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1];
   for (int i = tid; i < 2 * RB * Dh; i += T) hlo[i] = 0u;
   if (tid == 0) { s_lo = INT_MAX; s_hi = INT_MIN; s_next = 0; }
+  if (tid < 32) { s_wsum[tid] = 0; s_wcnt[tid] = 0; }
   __syncthreads();
 
   const int r = tid % RB, b = g * RB + r, rows = T / RB;
   const bool bok = b < A.B;
+  // long-window threshold of this restart in this segment
+  const int long_min = min(kc, max(8, 3 * seg_mean_window(A.win, A.perm, s0, s1, b, bok, A.B, tid, RB, rows,
+                                                           s_wsum, s_wcnt) + 8));
   const size_t VB = (size_t)A.V * A.B;
   constexpr unsigned FULL = 0xffffffffu;
-  float fdep = 0.f, fcom = 0.f, frec = 0.f;
+  long long xdep = 0, xcom = 0, xrec = 0;  // forward sums, exact (order-free) fixed point
   int lo = INT_MAX, hi = INT_MIN;
   // Control flow is kept warp-uniform: each warp claims the next group of
   // 32 / RB nodes of the segment from a shared counter (so warps finish
@@ -235,6 +271,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     base = __shfl_sync(FULL, base, 0);
     if (base >= s1 - s0) break;
     const int vi = s0 + base + (tid & 31) / RB;
+    float fdep = 0.f, fcom = 0.f, frec = 0.f;  // this item's forward sums
     bool valid = bok && vi < s1;
     const int vcl = valid ? vi : s0;
     const int vc = A.perm[vcl];
@@ -250,11 +287,9 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     int a = 0, bw = -2;
     if (valid) window(mu, sg, A.k_win, A.D, a, bw);
     const int nfull = bw - a + 1;                  // points; -1 for an idle lane
-    // Windows much longer than the warp's typical one (or than the cache) go to
-    // the cooperative path after this per-lane pass.
-    const int nact = __popc(__ballot_sync(FULL, valid));
-    const int mean = nact ? __reduce_add_sync(FULL, max(nfull, 0)) / nact : 0;
-    const bool is_long = valid && nfull > min(kc, max(8, 3 * mean + 8));
+    // Windows much longer than this restart's typical one in the segment (or
+    // than the cache) go to the cooperative path after this per-lane pass.
+    const bool is_long = valid && nfull > long_min;
     const int n = is_long ? -1 : nfull;            // per-lane points
     const bool vs = valid && !is_long;
     const int nmax = __reduce_max_sync(FULL, n);
@@ -480,6 +515,9 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
         fdep += sums[6]; fcom += sums[7]; frec += sums[8];
       }
     }
+    xdep += to_fix(fdep);
+    xcom += to_fix(fcom);
+    xrec += to_fix(frec);
     if (valid) {
       A.gpart[0 * VB + gi] = Ad;
       A.gpart[1 * VB + gi] = Bd;
@@ -496,13 +534,13 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
     atomicMax(&s_hi, hi);
   }
   __syncthreads();
-  double *red = reinterpret_cast<double *>(cC);
-  red[0 * T + tid] = fdep;
-  red[1 * T + tid] = fcom;
-  red[2 * T + tid] = frec;
+  long long *red = reinterpret_cast<long long *>(cC);
+  red[0 * T + tid] = xdep;
+  red[1 * T + tid] = xcom;
+  red[2 * T + tid] = xrec;
   __syncthreads();
   if (tid < RB) {
-    double acc[3] = {0.0, 0.0, 0.0};
+    long long acc[3] = {0, 0, 0};
     for (int row = 0; row < rows; ++row)
       for (int k = 0; k < 3; ++k) acc[k] += red[k * T + row * RB + tid];
     for (int k = 0; k < 3; ++k) A.fwd[((size_t)blk * RB + tid) * 3 + k] = acc[k];
@@ -533,24 +571,40 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
   }
 }
 
-// Usage per (restart, class, bin) from the partials of every block of the class
-// (fixed order over segments; exact int64 sums).  Block = (group g, class c,
-// tile of 256/RB bins); threads = restarts x bins, coalesced over restarts.
+// Usage per (restart, class, bin) from the partials of every block of the class:
+// block = (group g, class c, bin d); threads = restarts x slices of the segment
+// list (four independent loads in flight per thread); slices are combined in a
+// fixed order (exact int64 sums, kept in 2^32 fixed point).
 __global__ void __launch_bounds__(256) k_reduce(const RedArgs A) {
-  const int RB = A.RB, Dh = A.Dh, per = 256 / RB;
-  const int tiles = (Dh + per - 1) / per;
+  __shared__ long long part[256];
+  const int RB = A.RB, Dh = A.Dh, nsl = 256 / RB;
   int x = blockIdx.x;
-  const int tile = x % tiles; x /= tiles;
+  const int d = x % Dh; x /= Dh;
   const int c = x % A.C, g = x / A.C;
-  const int r = threadIdx.x % RB, d = tile * per + threadIdx.x / RB, b = g * RB + r;
-  if (d >= Dh || b >= A.B) return;
+  const int r = threadIdx.x % RB, sl = threadIdx.x / RB, b = g * RB + r;
+  const int s_end = A.cls_seg_ptr[c + 1];
   long long acc = 0;
-  for (int s = A.cls_seg_ptr[c]; s < A.cls_seg_ptr[c + 1]; ++s) {
-    const int blk = s * A.G + g;
-    const int2 sp = A.hspan[blk];
-    if (d >= sp.x && d <= sp.y) acc += A.hpart[((size_t)blk * Dh + d) * RB + r];
+  for (int s = A.cls_seg_ptr[c] + sl; s < s_end; s += 4 * nsl) {
+    long long v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int ss = s + u * nsl;
+      v[u] = 0;
+      if (ss < s_end) {
+        const int blk = ss * A.G + g;
+        const int2 sp = A.hspan[blk];
+        if (d >= sp.x && d <= sp.y) v[u] = A.hpart[((size_t)blk * Dh + d) * RB + r];
+      }
+    }
+    acc += v[0] + v[1] + v[2] + v[3];
   }
-  A.U[((size_t)b * A.C + c) * Dh + d] = (double)acc * kInvFix;
+  part[threadIdx.x] = acc;
+  __syncthreads();
+  if (sl == 0 && b < A.B) {
+    long long tot = 0;
+    for (int k = 0; k < nsl; ++k) tot += part[k * RB + r];
+    A.U[((size_t)b * A.C + c) * Dh + d] = tot;
+  }
 }
 
 // Window of every (node, restart): a | (b + 1) << 16 with the points [a, b] of
@@ -564,117 +618,127 @@ __global__ void k_windows(const float *mu, const float *sg, unsigned *win, size_
   }
 }
 
-// Deterministic block reduction (blockDim.x == 256).
-__device__ __forceinline__ double block_sum(double x, double *buf) {
-  const int tid = threadIdx.x;
-  buf[tid] = x;
-  __syncthreads();
-  for (int s = 128; s > 0; s >>= 1) {
-    if (tid < s) buf[tid] += buf[tid + s];
-    __syncthreads();
-  }
-  const double r = buf[0];
-  __syncthreads();
-  return r;
-}
-__device__ __forceinline__ double block_max(double x, double *buf) {
-  const int tid = threadIdx.x;
-  buf[tid] = x;
-  __syncthreads();
-  for (int s = 128; s > 0; s >>= 1) {
-    if (tid < s) buf[tid] = fmax(buf[tid], buf[tid + s]);
-    __syncthreads();
-  }
-  const double r = buf[0];
-  __syncthreads();
-  return r;
+// x * 2^-32 of a 2^32 fixed-point value as float, through two 32-bit halves
+// (64-bit integer to floating-point conversions run at the FP64 rate).
+__device__ __forceinline__ float fix_to_float(long long x) {
+  const int hi = (int)(x >> 32);
+  const unsigned lo = (unsigned)((unsigned long long)x & 0xffffffffull);
+  return (float)hi + (float)lo * 2.3283064365386963e-10f;
 }
 
-// One block (256 threads) per restart.
+// Deterministic block reductions over 256 threads: a fixed xor-shuffle tree per
+// warp, then the 8 warp results in order.
+__device__ __forceinline__ float block_sum_f(float x, float *sh) {
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = x;
+  __syncthreads();
+  float t = 0.f;
+  for (int w = 0; w < 8; ++w) t += sh[w];
+  __syncthreads();
+  return t;
+}
+__device__ __forceinline__ long long block_sum_i64(long long x, long long *sh) {
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = x;
+  __syncthreads();
+  long long t = 0;
+  for (int w = 0; w < 8; ++w) t += sh[w];
+  __syncthreads();
+  return t;
+}
+__device__ __forceinline__ long long block_max_ll(long long x, long long *sh) {
+  for (int o = 16; o > 0; o >>= 1) x = max(x, (long long)__shfl_xor_sync(0xffffffffu, x, o));
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = x;
+  __syncthreads();
+  long long t = sh[0];
+  for (int w = 1; w < 8; ++w) t = max(t, sh[w]);
+  __syncthreads();
+  return t;
+}
+
+// One block (256 threads) per restart.  Usage and storage stay exact 2^32 fixed
+// point (max and ReLU excess in integers); the softmax runs in fp32 on exact
+// differences from the max, and only thread 0 assembles the loss in fp64.
 __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   extern __shared__ __align__(16) unsigned char smem_f[];
-  double *U = reinterpret_cast<double *>(smem_f);  // C * Dh
-  __shared__ double buf[256];
-  __shared__ double s_m[kMaxClasses], s_s[kMaxClasses];
+  long long *U = reinterpret_cast<long long *>(smem_f);  // (C + 1) * Dh
+  __shared__ long long shl[8];
+  __shared__ float shf[8];
+  __shared__ long long s_m[kMaxClasses + 1], s_R[kMaxClasses];
+  __shared__ float s_s[kMaxClasses + 1];
   const int b = blockIdx.x, g = b / A.RB, r = b % A.RB, tid = threadIdx.x, Dh = A.Dh;
+  const float kInvFixF = 2.3283064365386963e-10f;
 
   for (int i = tid; i < A.C * Dh; i += 256) U[i] = A.Ug[(size_t)b * A.C * Dh + i];
+  if (A.Ureg)
+    for (int t = tid; t < Dh; t += 256) U[A.C * Dh + t] = A.Ureg[(size_t)b * Dh + t];
+  if (tid < A.C) {
+    const float R = A.limit[tid];
+    // limits in fixed point; an infinite or huge limit never binds
+    s_R[tid] = (isfinite(R) && R < 1.0e9f) ? (long long)R * 4294967296LL +
+                                                   (long long)((R - floorf(R)) * 4294967296.0f)
+                                           : LLONG_MAX;
+  }
   __syncthreads();
 
   // forward sums of the edge terms over every block of this restart group
-  double f3[3] = {0.0, 0.0, 0.0};
+  long long f3[3] = {0, 0, 0};
   const int nseg = A.cls_seg_ptr[A.C];
   for (int s = tid; s < nseg; s += 256)
     for (int k = 0; k < 3; ++k) f3[k] += A.fwd[((size_t)(s * A.G + g) * A.RB + r) * 3 + k];
-  const double vdep = block_sum(f3[0], buf);
-  const double lcom = block_sum(f3[1], buf);
-  const double vrec = block_sum(f3[2], buf);
+  const float vdep = (float)((double)block_sum_i64(f3[0], shl) * kInvFix);
+  const float lcom = (float)((double)block_sum_i64(f3[1], shl) * kInvFix);
+  const float vrec = (float)((double)block_sum_i64(f3[2], shl) * kInvFix);
 
-  // ReLU excess over finite limits (Eq. relu)
-  double ex = 0.0;
+  // ReLU excess over finite limits (Eq. relu), exact
+  long long ex = 0;
   for (int i = tid; i < A.C * Dh; i += 256) {
-    const float R = A.limit[i / Dh];
-    if (isfinite(R) && U[i] > (double)R) ex += U[i] - (double)R;
+    const long long R = s_R[i / Dh];
+    if (R != LLONG_MAX && U[i] > R) ex += U[i] - R;
   }
-  const double vres = block_sum(ex, buf);
+  ex = block_sum_i64(ex, shl);
 
-  // LogSumExp per class (Eq. max), max shifted out
-  double lse_sum = 0.0;
-  for (int c = 0; c < A.C; ++c) {
-    double m = -1e300;
-    for (int t = tid; t < Dh; t += 256) m = fmax(m, U[c * Dh + t]);
-    m = block_max(m, buf);
-    double s = 0.0;
-    for (int t = tid; t < Dh; t += 256) s += (double)expf((float)((U[c * Dh + t] - m) / A.tau));
-    s = block_sum(s, buf);
-    if (tid == 0) { s_m[c] = m; s_s[c] = s; }
-    lse_sum += m + (double)A.tau * log(s);
+  // LogSumExp per class (Eq. max) and of the storage, max shifted out
+  const int nh = A.C + (A.Ureg ? 1 : 0);
+  for (int c = 0; c < nh; ++c) {
+    long long m = LLONG_MIN;
+    for (int t = tid; t < Dh; t += 256) m = max(m, U[c * Dh + t]);
+    m = block_max_ll(m, shl);
+    float sacc = 0.f;
+    for (int t = tid; t < Dh; t += 256) sacc += expf(fix_to_float(U[c * Dh + t] - m) / A.tau);
+    sacc = block_sum_f(sacc, shf);
+    if (tid == 0) { s_m[c] = m; s_s[c] = sacc; }
   }
   __syncthreads();
-
-  // LogSumExp of the (folded) expected storage, Eq. max over Eq. active
-  double reg_lse = 0.0, reg_m = 0.0, reg_s = 1.0;
-  if (A.Ureg) {
-    double *R = U + (size_t)A.C * Dh;
-    for (int t = tid; t < Dh; t += 256) R[t] = A.Ureg[(size_t)b * Dh + t];
-    __syncthreads();
-    double m = -1e300;
-    for (int t = tid; t < Dh; t += 256) m = fmax(m, R[t]);
-    m = block_max(m, buf);
-    double sacc = 0.0;
-    for (int t = tid; t < Dh; t += 256) sacc += (double)expf((float)((R[t] - m) / A.tau));
-    sacc = block_sum(sacc, buf);
-    reg_m = m;
-    reg_s = sacc;
-    reg_lse = m + (double)A.tau * log(sacc);
-    for (int t = tid; t < Dh; t += 256)
-      A.Hreg[(size_t)b * Dh + t] = (float)((double)A.w_mem * (double)expf((float)((R[t] - m) / A.tau)) / sacc);
-  }
 
   const bool on_dep = A.terms & GAUS_DEP, on_com = A.terms & GAUS_COM;
   const bool on_robj = A.terms & GAUS_RES_OBJ, on_rv = A.terms & GAUS_RES_VIOL;
   const bool on_rec = A.terms & GAUS_REC;
   const float *lam = A.lambda + (size_t)b * GAUS_K;
-  const double c_res = on_rv ? (double)lam[GAUS_K_RES] + (double)A.rho * vres : 0.0;
+  const double vres = (double)ex * kInvFix;
+  const float c_res = on_rv ? (float)((double)lam[GAUS_K_RES] + (double)A.rho * vres) : 0.f;
   if (tid == 0) {
+    double lse_sum = 0.0;
+    for (int c = 0; c < A.C; ++c) lse_sum += (double)s_m[c] * kInvFix + (double)A.tau * (double)logf(s_s[c]);
+    const double reg_lse = A.Ureg ? (double)s_m[A.C] * kInvFix + (double)A.tau * (double)logf(s_s[A.C]) : 0.0;
     double L = 0.0;
     if (on_robj) L += (double)A.w_res * lse_sum;
-    if (on_com) L += (double)A.alpha * lcom;
+    if (on_com) L += (double)A.alpha * (double)lcom;
     if (A.Ureg) L += (double)A.w_mem * reg_lse;
-    const double Vk[3] = {on_dep ? vdep : 0.0, on_rv ? vres : 0.0, on_rec ? vrec : 0.0};
+    const double Vk[3] = {on_dep ? (double)vdep : 0.0, on_rv ? vres : 0.0, on_rec ? (double)vrec : 0.0};
     const bool act[3] = {on_dep, on_rv, on_rec};
     for (int k = 0; k < 3; ++k)
       if (act[k]) L += (double)lam[k] * Vk[k] + 0.5 * (double)A.rho * Vk[k] * Vk[k];
     float *T = A.terms_out + (size_t)b * GAUS_NT;
     T[GAUS_T_RES] = on_robj ? (float)lse_sum : 0.f;
-    T[GAUS_T_COM] = on_com ? (float)lcom : 0.f;
+    T[GAUS_T_COM] = on_com ? lcom : 0.f;
     T[GAUS_T_REG] = A.Ureg ? (float)reg_lse : 0.f;
     T[GAUS_T_VDEP] = (float)Vk[0];
     T[GAUS_T_VRES] = (float)Vk[1];
     T[GAUS_T_VREC] = (float)Vk[2];
     A.loss[b] = (float)L;
-    A.coef[b * 4 + 0] = on_dep ? (float)((double)lam[GAUS_K_DEP] + (double)A.rho * vdep) : 0.f;
-    A.coef[b * 4 + 1] = on_rec ? (float)((double)lam[GAUS_K_REC] + (double)A.rho * vrec) : 0.f;
+    A.coef[b * 4 + 0] = on_dep ? (float)((double)lam[GAUS_K_DEP] + (double)A.rho * Vk[0]) : 0.f;
+    A.coef[b * 4 + 1] = on_rec ? (float)((double)lam[GAUS_K_REC] + (double)A.rho * Vk[2]) : 0.f;
     const int bad = A.nonfinite[b];
     if (A.status) A.status[b] = bad ? GAUS_ENONFINITE : GAUS_OK;
     A.nonfinite[b] = 0;
@@ -683,56 +747,106 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
       for (int k = 0; k < 3; ++k)
         if (act[k]) lw[k] = (float)((double)lw[k] + (double)A.rho * Vk[k]);
     }
-    if (A.step) A.step[b] += 1;
+    if (A.step) {
+      const int st = A.step[b] + 1;
+      A.step[b] = st;
+      // Adam bias corrections of this step (torch.optim.Adam)
+      A.coef[b * 4 + 2] = 1.0f - powf(A.beta1, (float)st);
+      A.coef[b * 4 + 3] = 1.0f - powf(A.beta2, (float)st);
+    }
   }
-  // usage adjoint dL/dU_c(t) = w_res softmax_c(t) + c_res [U_c(t) > R_c]
+  // usage adjoint dL/dU_c(t) = w_res softmax_c(t) + c_res [U_c(t) > R_c], [class][bin][restart]
   for (int i = tid; i < A.C * Dh; i += 256) {
     const int c = i / Dh;
-    double h = 0.0;
-    if (on_robj) h += (double)A.w_res * (double)expf((float)((U[i] - s_m[c]) / A.tau)) / s_s[c];
-    const float R = A.limit[c];
-    if (on_rv && isfinite(R) && U[i] > (double)R) h += c_res;
-    A.H[(size_t)b * A.C * Dh + i] = (float)h;
+    float h = 0.f;
+    if (on_robj) h += A.w_res * expf(fix_to_float(U[i] - s_m[c]) / A.tau) / s_s[c];
+    if (on_rv && s_R[c] != LLONG_MAX && U[i] > s_R[c]) h += c_res;
+    A.H[(size_t)i * A.B + b] = h;
   }
+  if (A.Ureg)
+    for (int t = tid; t < Dh; t += 256)
+      A.Hreg[(size_t)b * Dh + t] = A.w_mem * expf(fix_to_float(U[A.C * Dh + t] - s_m[A.C]) / A.tau) / s_s[A.C];
+  (void)kInvFixF;
 }
 
 template <bool kAdam, bool kHist>
 __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
-  extern __shared__ __align__(16) unsigned char smem_u[];
-  float *Hs = reinterpret_cast<float *>(smem_u);  // Dh * RB
+  constexpr unsigned FULL = 0xffffffffu;
   const int tid = threadIdx.x, RB = A.RB, Dh = A.Dh;
   const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
   const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1], c = A.seg[3 * segi + 2];
-  if (kHist) {
-    for (int i = tid; i < Dh * RB; i += kThreads) {
-      const int t = i / RB, rr = i % RB, bb = g * RB + rr;
-      Hs[i] = bb < A.B ? A.H[((size_t)bb * A.C + c) * Dh + t] : 0.f;
-    }
-    __syncthreads();
-  }
+  const float *Hc = A.H + (size_t)c * Dh * A.B;  // usage adjoint of this class, [bin][restart]
   const int r = tid % RB, b = g * RB + r, rows = kThreads / RB;
-  if (b >= A.B) return;
+  const bool bok = b < A.B;
+  __shared__ int s_wsum[32], s_wcnt[32];
+  int long_min = 0;
+  if (kHist) {
+    if (tid < 32) { s_wsum[tid] = 0; s_wcnt[tid] = 0; }
+    __syncthreads();
+    long_min = max(8, 2 * seg_mean_window(A.win, A.perm, s0, s1, b, bok, A.B, tid, RB, rows, s_wsum, s_wcnt) + 8);
+  }
   const size_t VB = (size_t)A.V * A.B;
-  const float c_dep = A.coef[b * 4 + 0], c_rec = A.coef[b * 4 + 1];
-  for (int vi = s0 + tid / RB; vi < s1; vi += rows) {
-    const int vc = A.perm[vi];
-    const size_t ci = (size_t)vc * A.B + b, gi = (size_t)vi * A.B + b;
-    const float mu = A.mu[ci], sg = A.sg[ci];
+  const int bs = bok ? b : 0;
+  const float c_dep = A.coef[bs * 4 + 0], c_rec = A.coef[bs * 4 + 1];
+  const float bc1 = kAdam ? A.coef[bs * 4 + 2] : 1.f, bc2 = kAdam ? A.coef[bs * 4 + 3] : 1.f;
+  const int n_items = (s1 - s0 + rows - 1) / rows;
+  for (int it = 0; it < n_items; ++it) {
+    const int vi = s0 + tid / RB + it * rows;
+    const bool valid = bok && vi < s1;
+    const int vcl = valid ? vi : s0;
+    const int vc = A.perm[vcl];
+    const size_t ci = (size_t)vc * A.B + bs, gi = (size_t)vcl * A.B + bs;
+    const float mu = valid ? A.mu[ci] : 0.f, sg = valid ? A.sg[ci] : 1.f;
+    const bool ok = valid && usable(mu, sg);
     float Ah = 0.f, Bh = 0.f;
-    const bool ok = usable(mu, sg);
-    if (kHist && ok) {
-      // dL/dC_v(t) = w_v (H(t) - H(t+1)) for the own points (P = C(t) - C(t-1))
-      const float inv_s = 1.0f / sg, wv = A.w[vi];
-      int a, bw;
-      window(mu, sg, A.k_win, A.D, a, bw);
-      for (int t = a; t <= bw; ++t) {
-        const float z = ((float)t + 0.5f - mu) * inv_s;
-        const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
-        const float gh = wv * (Hs[fold_bin(t, A.II) * RB + r] - Hs[fold_bin(t + 1, A.II) * RB + r]);
-        Ah += gh * f;
-        Bh += gh * z * f;
+    if (kHist) {
+      // dL/dC_v(t) = w_v (H(t) - H(t+1)) for the own points (P = C(t) - C(t-1));
+      // windows much longer than the warp's typical one are done by the whole warp
+      const float inv_s = ok ? 1.0f / sg : 1.0f, wv = A.w[vcl];
+      int a = 0, bw = -1;
+      if (ok) window(mu, sg, A.k_win, A.D, a, bw);
+      const int nfull = bw - a + 1;
+      const bool is_long = ok && nfull > long_min;
+      const int n = is_long ? 0 : nfull;
+      const int nmax = __reduce_max_sync(FULL, n);
+      for (int j = 0; j < nmax; ++j) {
+        if (j < n) {
+          const int t = a + j;
+          const float z = ((float)t + 0.5f - mu) * inv_s;
+          const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
+          const float gh = wv * (Hc[(size_t)fold_bin(t, A.II) * A.B + b] - Hc[(size_t)fold_bin(t + 1, A.II) * A.B + b]);
+          Ah += gh * f;
+          Bh += gh * z * f;
+        }
+      }
+      __syncwarp();
+      unsigned longmask = __ballot_sync(FULL, is_long);
+      while (longmask) {
+        const int src = __ffs(longmask) - 1;
+        longmask &= longmask - 1;
+        const int l_a = __shfl_sync(FULL, a, src), l_n = __shfl_sync(FULL, nfull, src);
+        const int l_b = __shfl_sync(FULL, b, src);
+        const float l_mu = __shfl_sync(FULL, mu, src), l_inv = __shfl_sync(FULL, inv_s, src);
+        const float l_w = __shfl_sync(FULL, wv, src);
+        float pa = 0.f, pb = 0.f;
+        for (int base = 0; base < l_n; base += 32) {
+          const int j = base + (threadIdx.x & 31);
+          if (j < l_n) {
+            const int t = l_a + j;
+            const float z = ((float)t + 0.5f - l_mu) * l_inv;
+            const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
+            const float gh = l_w * (Hc[(size_t)fold_bin(t, A.II) * A.B + l_b] -
+                                    Hc[(size_t)fold_bin(t + 1, A.II) * A.B + l_b]);
+            pa += gh * f;
+            pb += gh * z * f;
+          }
+        }
+        pa = warp_sum(pa);
+        pb = warp_sum(pb);
+        if ((threadIdx.x & 31) == src) { Ah = pa; Bh = pb; }
       }
     }
+    if (!valid) continue;
     float Asum = c_dep * A.gpart[0 * VB + gi] + A.gpart[2 * VB + gi] + c_rec * A.gpart[4 * VB + gi] + Ah;
     float Bsum = c_dep * A.gpart[1 * VB + gi] + A.gpart[3 * VB + gi] + c_rec * A.gpart[5 * VB + gi] + Bh;
     if (A.eslot && ok)
@@ -747,8 +861,6 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
       A.grad_mu[ci] = gm;
       A.grad_sg[ci] = gs;
     } else {
-      const int step = A.step_dev[b];
-      const float bc1 = 1.0f - powf(A.beta1, (float)step), bc2 = 1.0f - powf(A.beta2, (float)step);
       const float m1 = A.beta1 * A.m_mu[ci] + (1.0f - A.beta1) * gm;
       const float v1 = A.beta2 * A.v_mu[ci] + (1.0f - A.beta2) * gm * gm;
       const float m2 = A.beta1 * A.m_sg[ci] + (1.0f - A.beta1) * gs;

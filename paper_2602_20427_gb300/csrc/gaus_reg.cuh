@@ -183,16 +183,23 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
   }
 }
 
-// Reg per (restart, bin) from every block's partials (fixed order).
-__global__ void __launch_bounds__(256) k_reduce_reg(const long long *rpart, double *Ureg, int B, int Dh, int RB,
+// Reg per (restart, bin) from every block's partials: block = (group, bin),
+// threads = restarts x slices of the segment list, slices combined in order.
+__global__ void __launch_bounds__(256) k_reduce_reg(const long long *rpart, long long *Ureg, int B, int Dh, int RB,
                                                     int G, int nseg) {
-  const int per = 256 / RB, tiles = (Dh + per - 1) / per;
-  const int tile = blockIdx.x % tiles, g = blockIdx.x / tiles;
-  const int r = threadIdx.x % RB, d = tile * per + threadIdx.x / RB, b = g * RB + r;
-  if (d >= Dh || b >= B) return;
+  __shared__ long long part[256];
+  const int nsl = 256 / RB;
+  const int d = blockIdx.x % Dh, g = blockIdx.x / Dh;
+  const int r = threadIdx.x % RB, sl = threadIdx.x / RB, b = g * RB + r;
   long long acc = 0;
-  for (int s = 0; s < nseg; ++s) acc += rpart[((size_t)(s * G + g) * Dh + d) * RB + r];
-  Ureg[(size_t)b * Dh + d] = (double)acc * kInvFix;
+  for (int s = sl; s < nseg; s += nsl) acc += rpart[((size_t)(s * G + g) * Dh + d) * RB + r];
+  part[threadIdx.x] = acc;
+  __syncthreads();
+  if (sl == 0 && b < B) {
+    long long tot = 0;
+    for (int k = 0; k < nsl; ++k) tot += part[k * RB + r];
+    Ureg[(size_t)b * Dh + d] = tot;
+  }
 }
 
 __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
