@@ -61,7 +61,7 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   IterArgs A;
   A.mu = mu; A.sg = sg;
   A.V = P.V; A.B = P.B; A.D = P.D; A.II = P.II; A.Dh = P.Dh; A.C = P.C; A.RB = ctx->RB; A.G = ctx->G;
-  A.kc = ctx->kc;
+  A.W = ctx->W;
   A.k_win = ctx->hp.window_k; A.alpha = ctx->hp.alpha;
   A.perm = ctx->d_perm; A.w = ctx->d_w; A.lat = ctx->d_lat;
   A.in_ptr = ctx->d_in_ptr; A.in_src = ctx->d_in_src; A.in_lat = ctx->d_in_lat;
@@ -69,22 +69,23 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   A.bin_ptr = ctx->d_bin_ptr; A.bin_src = ctx->d_bin_src; A.bin_shift = ctx->d_bin_shift;
   A.bout_ptr = ctx->d_bout_ptr; A.bout_dst = ctx->d_bout_dst; A.bout_shift = ctx->d_bout_shift;
   A.seg = ctx->d_seg; A.hpart = ctx->d_hpart; A.hspan = ctx->d_hspan; A.fwd = ctx->d_fwd;
-  A.gpart = ctx->d_gpart; A.nonfinite = ctx->d_nonfinite; A.win = ctx->d_win;
+  A.nonfinite = ctx->d_nonfinite; A.win = ctx->d_win; A.tab = ctx->d_tab;
+  A.ed = ctx->d_ed; A.nEt = P.E + P.NB; A.ce = ctx->ce; A.eslot4 = ctx->d_eslot4;
   return A;
 }
 
-using FwdKernel = void (*)(const IterArgs);
+using EdgeKernel = void (*)(const IterArgs);
 
-FwdKernel pick_fwd(unsigned terms, int II) {
+EdgeKernel pick_edges(unsigned terms, int II) {
   const bool dep = terms & GAUS_DEP, com = terms & GAUS_COM, rec = (terms & GAUS_REC) && II > 0;
-  if (dep && com && rec) return k_fwd<true, true, true>;
-  if (dep && com) return k_fwd<true, true, false>;
-  if (dep && rec) return k_fwd<true, false, true>;
-  if (dep) return k_fwd<true, false, false>;
-  if (com && rec) return k_fwd<false, true, true>;
-  if (com) return k_fwd<false, true, false>;
-  if (rec) return k_fwd<false, false, true>;
-  return k_fwd<false, false, false>;
+  if (dep && com && rec) return k_edges<true, true, true>;
+  if (dep && com) return k_edges<true, true, false>;
+  if (dep && rec) return k_edges<true, false, true>;
+  if (dep) return k_edges<true, false, false>;
+  if (com && rec) return k_edges<false, true, true>;
+  if (com) return k_edges<false, true, false>;
+  if (rec) return k_edges<false, false, true>;
+  return k_edges<false, false, false>;
 }
 
 // Enqueue loss + gradient (adam == false: gradient written to grad_*), or the
@@ -97,16 +98,12 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   const Plan &P = ctx->plan;
   const unsigned on = ctx->hp.terms;
   IterArgs A = iter_args(ctx, mu, sg);
-  {
-    const size_t n = (size_t)P.V * P.B;
-    k_windows<<<(int)std::min<size_t>((n + 255) / 256, 8 * 152), 256, 0, st>>>(mu, sg, ctx->d_win, n,
-                                                                          ctx->hp.window_k, P.D);
-    CK(cudaGetLastError(), "k_windows launch");
-  }
+  k_nodes<<<ctx->nblk, kFwdThreads, ctx->smem_nodes, st>>>(A);
+  CK(cudaGetLastError(), "k_nodes launch");
   if (ev) CK(cudaEventRecord(ev[1], st), "event");
-  FwdKernel kf = pick_fwd(on, P.II);
-  kf<<<ctx->nblk, kFwdThreads, ctx->smem_fwd, st>>>(A);
-  CK(cudaGetLastError(), "k_fwd launch");
+  EdgeKernel ke = pick_edges(on, P.II);
+  ke<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
+  CK(cudaGetLastError(), "k_edges launch");
   if (ev) CK(cudaEventRecord(ev[2], st), "event");
   const bool reg = on & GAUS_REG_OBJ;
   RegArgs RA;
@@ -115,7 +112,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
     RA.V = P.V; RA.B = P.B; RA.D = P.D; RA.II = P.II; RA.Dh = P.Dh; RA.RB = ctx->RBr; RA.G = ctx->Gr;
     RA.k_win = ctx->hp.window_k; RA.perm = ctx->d_perm; RA.bits = ctx->d_bits;
     RA.out_ptr = ctx->d_out_ptr; RA.out_dst = ctx->d_out_dst; RA.seg = ctx->d_seg; RA.win = ctx->d_win;
-    RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gpart = ctx->d_gpart; RA.eslot = ctx->d_eslot;
+    RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gown = ctx->d_gown; RA.eslot = ctx->d_eslot;
     k_reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_fwd launch");
     k_reduce_reg<<<ctx->Gr * P.Dh, 256, 0, st>>>(ctx->d_rpart, ctx->d_Ureg, P.B, P.Dh, ctx->RBr, ctx->Gr,
@@ -134,7 +131,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   F.terms = on; F.tau = ctx->hp.tau; F.rho = ctx->hp.rho; F.alpha = ctx->hp.alpha;
   F.w_res = ctx->hp.w_res; F.w_mem = ctx->hp.w_mem;
   F.cls_seg_ptr = ctx->d_cls_seg_ptr; F.limit = ctx->d_limit;
-  F.hpart = ctx->d_hpart; F.hspan = ctx->d_hspan; F.fwd = ctx->d_fwd;
+  F.hpart = ctx->d_hpart; F.hspan = ctx->d_hspan; F.fwd = ctx->d_fwd; F.nfwd = ctx->nchunk;
   F.lambda = lambda; F.update_lambda = adam ? 1 : 0; F.step = adam ? S->step : nullptr;
   F.beta1 = ctx->hp.beta1; F.beta2 = ctx->hp.beta2;
   F.H = ctx->d_H; F.coef = ctx->d_coef; F.loss = loss; F.terms_out = terms;
@@ -148,11 +145,14 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   if (ev) CK(cudaEventRecord(ev[3], st), "event");
 
   UpdArgs U;
-  U.in_ptr = ctx->d_in_ptr; U.in_eslot = ctx->d_in_eslot; U.eslot = reg ? ctx->d_eslot : nullptr;
+  U.in_ptr = ctx->d_in_ptr; U.in_eslot = ctx->d_in_eslot; U.out_ptr = ctx->d_out_ptr;
+  U.bin_ptr = ctx->d_bin_ptr; U.bin_eslot = ctx->d_bin_eslot; U.bout_ptr = ctx->d_bout_ptr;
+  U.E = P.E; U.has_back = (on & GAUS_REC) && P.II > 0 && P.NB > 0; U.eslot4 = ctx->d_eslot4;
+  U.eslot = reg ? ctx->d_eslot : nullptr; U.gown = reg ? ctx->d_gown : nullptr;
   U.mu = const_cast<float *>(mu); U.sg = const_cast<float *>(sg);
   U.V = P.V; U.B = P.B; U.D = P.D; U.II = P.II; U.Dh = P.Dh; U.C = P.C; U.RB = ctx->RB; U.G = ctx->G;
   U.k_win = ctx->hp.window_k; U.perm = ctx->d_perm; U.win = ctx->d_win; U.w = ctx->d_w; U.seg = ctx->d_seg;
-  U.gpart = ctx->d_gpart; U.H = ctx->d_H; U.coef = ctx->d_coef;
+  U.H = ctx->d_H; U.coef = ctx->d_coef;
   U.grad_mu = grad_mu; U.grad_sg = grad_sg;
   U.m_mu = adam ? S->m_mu : nullptr; U.v_mu = adam ? S->v_mu : nullptr;
   U.m_sg = adam ? S->m_sigma : nullptr; U.v_sg = adam ? S->v_sigma : nullptr;
@@ -173,12 +173,8 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
 }
 
 gaus_status set_smem_attrs(gaus_ctx *ctx) {
-  const void *fwd[] = {(const void *)k_fwd<true, true, true>, (const void *)k_fwd<true, true, false>,
-                       (const void *)k_fwd<true, false, true>, (const void *)k_fwd<true, false, false>,
-                       (const void *)k_fwd<false, true, true>, (const void *)k_fwd<false, true, false>,
-                       (const void *)k_fwd<false, false, true>, (const void *)k_fwd<false, false, false>};
-  for (const void *f : fwd)
-    CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fwd), "smem attr fwd");
+  CK(cudaFuncSetAttribute((const void *)k_nodes, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_nodes),
+     "smem attr nodes");
   CK(cudaFuncSetAttribute((const void *)k_finalize, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fin),
      "smem attr fin");
   CK(cudaFuncSetAttribute((const void *)k_reg_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_rfwd),
@@ -211,20 +207,30 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   while (ctx->RB < P.B && ctx->RB < 32) ctx->RB <<= 1;
   ctx->G = (P.B + ctx->RB - 1) / ctx->RB;
   ctx->nblk = P.nseg * ctx->G;
+  // edge pass: about 8 blocks per SM over all restart groups, whole warp passes per block
+  {
+    const int nEt = P.E + P.NB, per_pass = (kFwdThreads / 32) * (32 / ctx->RB);
+    const long want = std::max(1L, (long)8 * nsm / ctx->G);
+    long ce = std::max<long>(per_pass, ((long)nEt + want - 1) / want);
+    ce = (ce + per_pass - 1) / per_pass * per_pass;
+    ctx->ce = (int)ce;
+    ctx->nchunk = std::max(1, (int)((nEt + ce - 1) / ce));
+  }
   ctx->red_blocks = ctx->G * P.C * P.Dh;
-  // k_fwd shared memory: the two histogram halves plus the own-window cache,
-  // sized for two resident blocks per SM when the histogram allows it.
-  const size_t hist = 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned);
-  const size_t per_pt = 3 * (size_t)kFwdThreads * sizeof(float);
-  const size_t budget2 = kMaxSmem / 2 - 1024, budget1 = kMaxSmem - 1024;
-  int kc = 0;
-  if (hist + 16 * per_pt <= budget2) kc = (int)std::min<size_t>(kCacheMax, (budget2 - hist) / per_pt);
-  else if (hist + 4 * per_pt <= budget1) kc = (int)std::min<size_t>(kCacheMax, (budget1 - hist) / per_pt);
-  if (kc < 4) {
+  // k_nodes shared memory: the two halves of the usage histogram
+  ctx->smem_nodes = 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned);
+  if (ctx->smem_nodes > kMaxSmem - 1024) {
     ctx->err = "usage histogram of this horizon/II does not fit in shared memory";
     return GAUS_EINVAL;
   }
-  ctx->kc = kc;
+  // CDF table rows: up to kTableMax points per (node, restart), a multiple of 4,
+  // with the table kept under kTableBytes (longer windows are evaluated directly)
+  {
+    const size_t per_pt = (size_t)P.V * P.B * sizeof(float);
+    size_t w = std::min<size_t>(kTableMax, kTableBytes / per_pt);
+    w = std::max<size_t>(4, w & ~(size_t)3);
+    ctx->W = (int)w;
+  }
   // storage-term kernels: their own restarts-per-row so that the storage histogram
   // (two u32 halves), its difference array and constants fit in shared memory
   ctx->RBr = ctx->RB;
@@ -240,7 +246,6 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   ctx->nblk_r = P.nseg * ctx->Gr;
   ctx->smem_rfwd = rfwd_bytes(ctx->RBr);
   ctx->smem_rbwd = (size_t)P.Dh * ctx->RBr * sizeof(float);
-  ctx->smem_fwd = hist + (size_t)kc * per_pt;
   ctx->smem_upd = (size_t)ctx->RB * P.Dh * sizeof(float);
   ctx->smem_fin = (size_t)(P.C + 1) * P.Dh * sizeof(double);
   ctx->smem_ver = ((size_t)P.C * P.Dh + (P.D + 1) + P.Dh) * sizeof(long long);
@@ -262,6 +267,12 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(upload(ctx, &ctx->d_out_ptr, P.out_ptr));
   TRY(upload(ctx, &ctx->d_out_dst, P.out_dst));
   TRY(upload(ctx, &ctx->d_in_eslot, P.in_eslot));
+  TRY(upload(ctx, &ctx->d_bin_eslot, P.bin_eslot));
+  {
+    int32_t *ed = nullptr;
+    TRY(upload(ctx, &ed, P.ed));
+    ctx->d_ed = reinterpret_cast<int4 *>(ed);
+  }
   TRY(upload(ctx, &ctx->d_bin_ptr, P.bin_ptr));
   TRY(upload(ctx, &ctx->d_bin_src, P.bin_src));
   TRY(upload(ctx, &ctx->d_bin_shift, P.bin_shift));
@@ -296,9 +307,10 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_U, (size_t)P.B * P.C * P.Dh));
   if (ctx->hp.terms & GAUS_REG_OBJ) TRY(alloc_storage_scratch(ctx));
   TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
-  TRY(scratch(ctx, &ctx->d_fwd, (size_t)ctx->nblk * ctx->RB * 3));
-  TRY(scratch(ctx, &ctx->d_gpart, 6 * VB));
+  TRY(scratch(ctx, &ctx->d_fwd, (size_t)ctx->nchunk * ctx->G * ctx->RB * 3));
+  TRY(scratch(ctx, &ctx->d_eslot4, 2 * ((size_t)P.E + P.NB) * P.B));
   TRY(scratch(ctx, &ctx->d_win, VB));
+  TRY(scratch(ctx, &ctx->d_tab, VB * ctx->W));
   TRY(scratch(ctx, &ctx->d_H, (size_t)P.B * P.C * P.Dh));
   TRY(scratch(ctx, &ctx->d_coef, (size_t)P.B * 4));
   TRY(scratch(ctx, &ctx->d_nonfinite, (size_t)P.B));
@@ -316,6 +328,7 @@ gaus_status alloc_storage_scratch(gaus_ctx *ctx) {
   TRY(scratch(ctx, &ctx->d_rpart, (size_t)ctx->nblk_r * P.Dh * ctx->RBr));
   TRY(scratch(ctx, &ctx->d_Ureg, (size_t)P.B * P.Dh));
   TRY(scratch(ctx, &ctx->d_Hreg, (size_t)P.B * P.Dh));
+  TRY(scratch(ctx, &ctx->d_gown, (size_t)P.V * P.B));
   TRY(scratch(ctx, &ctx->d_eslot, (size_t)std::max(1, P.E) * P.B));
   return GAUS_OK;
 }
@@ -488,7 +501,7 @@ gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_stat
     ctx->err = "gaus_profile_iterate: NULL pointer or n_iters < 0";
     return GAUS_EINVAL;
   }
-  constexpr int kEv = 5;  // before k_windows, before / after k_fwd, after finalize, after update
+  constexpr int kEv = 5;  // before k_nodes, before / after k_edges, after finalize, after update
   std::vector<cudaEvent_t> ev(kEv * (size_t)n_iters);
   for (auto &e : ev) CK(cudaEventCreate(&e), "event create");
   gaus_status st = GAUS_OK;

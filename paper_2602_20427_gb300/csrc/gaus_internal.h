@@ -15,7 +15,8 @@ namespace gaus {
 constexpr int kFwdThreads = 256;
 constexpr int kThreads = 128;
 // Most own-window points cached in shared memory per thread (longer windows recompute).
-constexpr int kCacheMax = 32;
+constexpr int kTableMax = 32;                    // points per CDF table row, at most
+constexpr size_t kTableBytes = (size_t)64 << 20;  // CDF table size bound
 // Fixed-point scale of the usage histograms: P * 2^32 accumulated in int64.
 constexpr float kFix = 4294967296.0f;
 constexpr double kInvFix = 1.0 / 4294967296.0;
@@ -42,6 +43,11 @@ struct Plan {
   std::vector<int32_t> bin_ptr, bin_src, bin_shift;
   // back edges grouped by internal producer j: consumer caller id i, same shift
   std::vector<int32_t> bout_ptr, bout_dst, bout_shift;
+  // bout position of each back edge in bin order
+  std::vector<int32_t> bin_eslot;
+  // edge list of the edge pass, 4 per edge: producer, consumer (caller ids),
+  // latency or shift, kind (0 forward, 1 back); E forward edges then NB back edges
+  std::vector<int32_t> ed;
   // segments of internal nodes, each inside one class: start, end, class
   std::vector<int32_t> seg;               // 3 * nseg
   std::vector<int32_t> cls_seg_ptr;       // C + 1, segments of class c
@@ -70,12 +76,13 @@ struct gaus_ctx {
   gaus_hparams hp;
   cudaStream_t stream = nullptr;
   std::string err;
-  int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per pass
-  int kc = 0;                    // own-window points cached per thread in k_fwd
+  int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per node pass
+  int ce = 0, nchunk = 0;        // edge pass: edges per block, edge chunks (blocks = nchunk * G)
+  int W = 0;                     // points per CDF table row
   int red_blocks = 0;
   int RBr = 32, Gr = 1, nblk_r = 0;  // storage-term kernels: restarts per row, groups, blocks
   size_t smem_rfwd = 0, smem_rbwd = 0;
-  size_t smem_fwd = 0, smem_upd = 0, smem_fin = 0, smem_ver = 0;
+  size_t smem_nodes = 0, smem_upd = 0, smem_fin = 0, smem_ver = 0;
   // device graph
   int32_t *d_perm = nullptr;
   float *d_w = nullptr, *d_bits = nullptr, *d_limit = nullptr;
@@ -96,15 +103,19 @@ struct gaus_ctx {
   // scratch
   long long *d_hpart = nullptr;  // nblk * Dh * RB fixed-point usage partials
   int2 *d_hspan = nullptr;       // nblk folded bin span written by each block
-  long long *d_fwd = nullptr;    // nblk * RB * 3 forward sums (dep, com, rec), 2^32 fixed point
+  long long *d_fwd = nullptr;    // nchunk * G * RB * 3 forward sums (dep, com, rec), 2^32 fixed point
   long long *d_U = nullptr;      // B * C * Dh usage (k_reduce), 2^32 fixed point
   long long *d_rpart = nullptr;  // nblk_r * Dh * RBr storage partials
   long long *d_Ureg = nullptr;   // B * Dh expected (folded) storage, 2^32 fixed point
   float *d_Hreg = nullptr;       // B * Dh storage adjoint
   float2 *d_eslot = nullptr;     // E * B successor shares of the storage gradient
   int32_t *d_in_eslot = nullptr; // E
-  float *d_gpart = nullptr;      // 6 * V * B partial gradient sums (internal index)
+  int32_t *d_bin_eslot = nullptr;  // NB
+  int4 *d_ed = nullptr;          // E + NB edge list of the edge pass
+  float4 *d_eslot4 = nullptr;    // 2 (E + NB) * B per-edge partials [edge][side][restart]
+  float2 *d_gown = nullptr;      // V * B own-window storage adjoint (internal index)
   unsigned *d_win = nullptr;     // V * B packed windows (caller order)
+  float *d_tab = nullptr;        // V * B * W CDF values at the window points (caller order)
   float *d_H = nullptr;          // B * C * Dh usage adjoint dL/dU
   float *d_coef = nullptr;       // B * 4 (c_dep, c_rec)
   int32_t *d_nonfinite = nullptr;  // B flags

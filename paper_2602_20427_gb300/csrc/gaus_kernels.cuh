@@ -7,14 +7,18 @@
 //   window_k * sigma_v of mu_v, with C_v(t) = 0 below and 1 above (Eq. round and
 // its open end bins), and evaluates each neighbour's CDF at the points it needs.
 //
-// k_fwd     : bin masses -> usage histogram (shared-memory int64 fixed point, one
-//             class per block, no global atomics) and every edge term from both
-//             endpoints (gathered through CSC as consumer and CSR as producer):
-//             forward sums and the unscaled partial gradients.
+// k_nodes   : windows, the CDF table (C at each window point, computed once per
+//             (node, restart) and read by every incident edge) and bin masses ->
+//             usage histogram (shared-memory fixed point, one class per block, no
+//             global atomics).
+// k_edges   : every edge term, once per (edge, restart), from both endpoints'
+//             table rows: forward sums and each endpoint's unscaled partial
+//             gradients, written to per-edge slots (no atomics).
 // k_finalize: one block per restart -- usage per class, LogSumExp (Eq. max),
 //             ReLU (Eq. relu), the augmented-Lagrangian coefficients (Sec. 3.3).
-// k_update  : usage adjoint of the node's own window, the combined gradient and
-//             (optionally) the Adam step.
+// k_update  : usage adjoint of the node's own window, the node's edge slots
+//             gathered in a fixed order, the combined gradient and (optionally)
+//             the Adam step.
 #pragma once
 
 #include <climits>
@@ -29,7 +33,7 @@ namespace gaus {
 
 struct IterArgs {
   const float *mu, *sg;  // (V, B) caller order
-  int V, B, D, II, Dh, C, RB, G, kc;
+  int V, B, D, II, Dh, C, RB, G, W;  // W: points per table row
   float k_win, alpha;
   const int32_t *perm;
   const float *w;
@@ -42,9 +46,12 @@ struct IterArgs {
   long long *hpart;
   int2 *hspan;
   long long *fwd;
-  float *gpart;
   int32_t *nonfinite;
-  const unsigned *win;  // (V, B) packed windows: a | (b + 1) << 16
+  unsigned *win;  // (V, B) packed windows a | (b + 1) << 16, written by k_nodes
+  float *tab;     // (V, B, W) CDF values at the window points, written by k_nodes
+  const int4 *ed; // edge list of the edge pass (nEt = E + NB edges, ce per block)
+  int nEt, ce;
+  float4 *eslot4; // (2 nEt, B) per-edge partials: [edge][producer, consumer][restart]
 };
 
 struct RedArgs {
@@ -66,7 +73,8 @@ struct FinArgs {
   const float *limit;
   const long long *hpart;
   const int2 *hspan;
-  const long long *fwd;
+  const long long *fwd;  // per (edge chunk, restart group) forward sums
+  int nfwd;              // edge chunks
   float *lambda;      // read; updated in place when update_lambda
   int update_lambda;
   int32_t *step;      // incremented when not NULL
@@ -76,8 +84,15 @@ struct FinArgs {
 };
 
 struct UpdArgs {
-  const int32_t *in_ptr, *in_eslot;  // storage term: successor shares gathered per in-edge
-  const float2 *eslot;               // NULL when the storage term is off
+  // per-edge partials of the edge pass, gathered per node: out-edges (CSR positions
+  // out_ptr), in-edges (in_eslot maps CSC to CSR position), back edges out
+  // (positions E + bout_ptr) and in (bin_eslot maps bin to bout position)
+  const int32_t *in_ptr, *in_eslot, *out_ptr;
+  const int32_t *bin_ptr, *bin_eslot, *bout_ptr;
+  int E, has_back;
+  const float4 *eslot4;
+  const float2 *eslot;               // storage term: successor shares (NULL when off)
+  const float2 *gown;                // storage term: own-window adjoint (NULL when off)
   float *mu, *sg;  // caller order; written when adam
   int V, B, D, II, Dh, C, RB, G;
   float k_win;
@@ -85,7 +100,6 @@ struct UpdArgs {
   const unsigned *win;  // (V, B) packed windows of the state being updated
   const float *w;
   const int32_t *seg;
-  const float *gpart;
   const float *H, *coef;
   float *grad_mu, *grad_sg;                  // gradient mode
   float *m_mu, *v_mu, *m_sg, *v_sg;          // Adam mode
@@ -128,424 +142,121 @@ __device__ __forceinline__ float warp_sum(float x) {
   return x;
 }
 
-// One (node, restart) item whose window is long, processed by the whole warp with
-// lanes over its points (32 at a time).  Same terms and formulas as the per-lane
-// path; the warp-reduced sums are returned in out[0..8] on every lane:
-// Ad, Bd, Ao, Bo, Ar, Br, fdep, fcom, frec.
-template <bool kDep, bool kCom, bool kRec>
-__device__ void coop_item(const IterArgs &A, int vcl, int b, int r, int RB, float mu, float inv_s, int a, int bw,
-                          float wv, unsigned *hlo, unsigned *hhi, float out[9]) {
-  constexpr unsigned FULL = 0xffffffffu;
-  const int lane = threadIdx.x & 31, n = bw - a + 1;
-  float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f, fdep = 0.f, fcom = 0.f, frec = 0.f;
-  float z_carry = 0.f, q_carry = 0.f;
-  for (int base = 0; base <= n; base += 32) {
-    const int pidx = base + lane;
-    const bool pt = pidx < n;
-    const int t = a + pidx;
-    const float z = ((float)t + 0.5f - mu) * inv_s;
-    const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
-    const float Cv = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
-    const float f = pt ? kInvSqrt2Pi * expf(-0.5f * z * z) : 0.f;
-    const float zf = z * f;
-    float zp = __shfl_up_sync(FULL, z, 1), qp = __shfl_up_sync(FULL, q, 1);
-    if (lane == 0) { zp = z_carry; qp = q_carry; }
-    if (pidx <= n) hist_add(hlo, hhi, fold_bin(t, A.II) * RB + r, wv * bin_mass(pt, pidx == 0, z, q, zp, qp));
-    z_carry = __shfl_sync(FULL, z, 31);
-    q_carry = __shfl_sync(FULL, q, 31);
-    if (kDep || kCom) {
-      for (int e = A.in_ptr[vcl]; e < A.in_ptr[vcl + 1]; ++e) {  // own = consumer
-        const int uc = A.in_src[e], L = A.in_lat[e];
-        const float mu_u = A.mu[(size_t)uc * A.B + b], sg_u = A.sg[(size_t)uc * A.B + b];
-        if (!usable(mu_u, sg_u)) continue;
-        const float inv_u = 1.0f / sg_u;
-        int au, bu;
-        window(mu_u, sg_u, A.k_win, A.D, au, bu);
-        if (pt) {
-          const float c_hi = cdf_at(t + 1 - L, mu_u, inv_u, au, bu);
-          const float p = c_hi - cdf_at(t - L, mu_u, inv_u, au, bu);
-          if (kDep) { fdep += Cv * p; Ad += p * f; Bd += p * zf; }
-          if (kCom) {
-            const float cu = (L == 1) ? c_hi : cdf_at(t, mu_u, inv_u, au, bu);
-            fcom += cu * (1.0f - Cv);
-            Ao -= A.alpha * cu * f;
-            Bo -= A.alpha * cu * zf;
-          }
-        }
-        if (kDep && base == 0 && lane == 0) fdep += 1.0f - cdf_at(bw + 1 - L, mu_u, inv_u, au, bu);
-      }
-      const int L = A.lat[vcl];
-      for (int e = A.out_ptr[vcl]; e < A.out_ptr[vcl + 1]; ++e) {  // own = producer
-        const int wc = A.out_dst[e];
-        const float mu_w = A.mu[(size_t)wc * A.B + b], sg_w = A.sg[(size_t)wc * A.B + b];
-        if (!usable(mu_w, sg_w)) continue;
-        const float inv_w = 1.0f / sg_w;
-        int aw, bw2;
-        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
-        if (pt) {
-          const float c_hi = cdf_at(t + L, mu_w, inv_w, aw, bw2);
-          const float c_lo = cdf_at(t + L - 1, mu_w, inv_w, aw, bw2);
-          if (kDep) { const float p = c_hi - c_lo; Ad -= p * f; Bd -= p * zf; }
-          if (kCom) {
-            const float cw = (L == 1) ? c_lo : cdf_at(t, mu_w, inv_w, aw, bw2);
-            Ao += A.alpha * (1.0f - cw) * f;
-            Bo += A.alpha * (1.0f - cw) * zf;
-            if (t < aw) fcom += Cv;
-          }
-        }
-        if (kCom && base == 0 && lane == 0) fcom += (float)max(0, aw - 1 - bw);
-      }
-    }
-    if (kRec) {
-      for (int e = A.bin_ptr[vcl]; e < A.bin_ptr[vcl + 1]; ++e) {  // own = consumer i
-        const int jc = A.bin_src[e], L = A.bin_shift[e];
-        const float mu_u = A.mu[(size_t)jc * A.B + b], sg_u = A.sg[(size_t)jc * A.B + b];
-        if (!usable(mu_u, sg_u)) continue;
-        const float inv_u = 1.0f / sg_u;
-        int au, bu;
-        window(mu_u, sg_u, A.k_win, A.D, au, bu);
-        if (pt) {
-          const float p = cdf_at(t + 1 - L, mu_u, inv_u, au, bu) - cdf_at(t - L, mu_u, inv_u, au, bu);
-          frec += Cv * p; Ar += p * f; Br += p * zf;
-        }
-        if (base == 0 && lane == 0) frec += 1.0f - cdf_at(bw + 1 - L, mu_u, inv_u, au, bu);
-      }
-      for (int e = A.bout_ptr[vcl]; e < A.bout_ptr[vcl + 1]; ++e) {  // own = producer j
-        const int ic = A.bout_dst[e], L = A.bout_shift[e];
-        const float mu_w = A.mu[(size_t)ic * A.B + b], sg_w = A.sg[(size_t)ic * A.B + b];
-        if (!usable(mu_w, sg_w)) continue;
-        const float inv_w = 1.0f / sg_w;
-        int aw, bw2;
-        window(mu_w, sg_w, A.k_win, A.D, aw, bw2);
-        if (pt) {
-          const float p = cdf_at(t + L, mu_w, inv_w, aw, bw2) - cdf_at(t + L - 1, mu_w, inv_w, aw, bw2);
-          Ar -= p * f; Br -= p * zf;
-        }
-      }
-    }
+// A neighbour's windowed CDF C_u(x): 0 below its window, 1 above it, inside it
+// the table value written by k_nodes, or -- for a window longer than the table
+// row -- evaluated from its mean and sigma (loaded only then).
+struct Nb {
+  const float *row;  // table row of (u, b)
+  int a, b;          // window points [a, b]
+  bool tab;          // the row holds every point of the window
+  float mu, inv;
+  __device__ __forceinline__ float at(int x) const {
+    if (x < a) return 0.0f;
+    if (x > b) return 1.0f;
+    return tab ? __ldg(row + (x - a)) : cdf_fast(((float)x + 0.5f - mu) * inv);
   }
-  __syncwarp();
-  out[0] = warp_sum(Ad); out[1] = warp_sum(Bd); out[2] = warp_sum(Ao); out[3] = warp_sum(Bo);
-  out[4] = warp_sum(Ar); out[5] = warp_sum(Br);
-  out[6] = warp_sum(fdep); out[7] = warp_sum(fcom); out[8] = warp_sum(frec);
-}
+};
 
-template <bool kDep, bool kCom, bool kRec>
-__global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
-  // Shared memory: usage histogram as two u32 halves [bin][restart] (conflict-free
-  // for any bins the lanes of a warp touch), then the own-window cache.
+// Window, CDF table and usage histogram (Eq. round, Eq. usage).  Block = one
+// segment (nodes of one class) x one restart group; lanes are restarts.  Every
+// (node, restart) gets its window [a, b] of points within window_k sigma, the CDF
+// values C(a..b) (from Q(|z|) = Phi(-|z|), so that both tails keep relative
+// accuracy) written to its table row for the edge pass, and its bin masses added
+// to the block's histogram as round(w P 2^32) in two exact 16-bit halves.  The
+// span of bins the block touched goes to the partials read by k_reduce.
+__global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
   extern __shared__ __align__(16) unsigned char smem[];
   constexpr int T = kFwdThreads;
-  const int tid = threadIdx.x, RB = A.RB, Dh = A.Dh, kc = A.kc;
-  unsigned *hlo = reinterpret_cast<unsigned *>(smem);
+  constexpr unsigned FULL = 0xffffffffu;
+  const int tid = threadIdx.x, lane = tid & 31, RB = A.RB, Dh = A.Dh, W = A.W;
+  unsigned *hlo = reinterpret_cast<unsigned *>(smem);  // [bin][restart]
   unsigned *hhi = hlo + (size_t)Dh * RB;
-  float *cC = reinterpret_cast<float *>(hhi + (size_t)Dh * RB);
-  float *cF = cC + (size_t)kc * T;
-  float *cZ = cF + (size_t)kc * T;
-  __shared__ int s_lo, s_hi, s_next, s_wsum[32], s_wcnt[32];
+  __shared__ int s_lo, s_hi, s_next;
 
   const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
   const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1];
   for (int i = tid; i < 2 * RB * Dh; i += T) hlo[i] = 0u;
   if (tid == 0) { s_lo = INT_MAX; s_hi = INT_MIN; s_next = 0; }
-  if (tid < 32) { s_wsum[tid] = 0; s_wcnt[tid] = 0; }
   __syncthreads();
 
-  const int r = tid % RB, b = g * RB + r, rows = T / RB;
+  const int r = tid % RB, b = g * RB + r;
   const bool bok = b < A.B;
-  // long-window threshold of this restart in this segment
-  const int long_min = min(kc, max(8, 3 * seg_mean_window(A.win, A.perm, s0, s1, b, bok, A.B, tid, RB, rows,
-                                                           s_wsum, s_wcnt) + 8));
-  const size_t VB = (size_t)A.V * A.B;
-  constexpr unsigned FULL = 0xffffffffu;
-  long long xdep = 0, xcom = 0, xrec = 0;  // forward sums, exact (order-free) fixed point
   int lo = INT_MAX, hi = INT_MIN;
-  // Control flow is kept warp-uniform: each warp claims the next group of
-  // 32 / RB nodes of the segment from a shared counter (so warps finish
-  // together), and every loop runs to the warp's maximum trip count with a
-  // per-lane predicate, so the warp never splits around the shared atomics.
   const int npw = 32 / RB;
   for (;;) {
     int base = 0;
-    if ((tid & 31) == 0) base = atomicAdd(&s_next, npw);
+    if (lane == 0) base = atomicAdd(&s_next, npw);
     base = __shfl_sync(FULL, base, 0);
     if (base >= s1 - s0) break;
-    const int vi = s0 + base + (tid & 31) / RB;
-    float fdep = 0.f, fcom = 0.f, frec = 0.f;  // this item's forward sums
-    bool valid = bok && vi < s1;
-    const int vcl = valid ? vi : s0;
+    const int vi = s0 + base + lane / RB;
+    const bool present = bok && vi < s1;
+    const int vcl = present ? vi : s0;
     const int vc = A.perm[vcl];
-    const size_t gi = (size_t)vcl * A.B + (bok ? b : 0);
-    const float mu = valid ? A.mu[(size_t)vc * A.B + b] : 0.f;
-    const float sg = valid ? A.sg[(size_t)vc * A.B + b] : 1.f;
-    if (valid && !usable(mu, sg)) {
-      A.nonfinite[b] = 1;
-      for (int k = 0; k < 6; ++k) A.gpart[k * VB + gi] = 0.f;
-      valid = false;
-    }
+    const size_t ci = (size_t)vc * A.B + (bok ? b : 0);
+    const float mu = present ? A.mu[ci] : 0.f, sg = present ? A.sg[ci] : 1.f;
+    const bool valid = present && usable(mu, sg);
+    if (present && !valid) A.nonfinite[b] = 1;
     const float inv_s = valid ? 1.0f / sg : 1.0f, wv = A.w[vcl];
-    int a = 0, bw = -2;
+    int a = 0, bw = -1;
     if (valid) window(mu, sg, A.k_win, A.D, a, bw);
-    const int nfull = bw - a + 1;                  // points; -1 for an idle lane
-    // Windows much longer than this restart's typical one in the segment (or
-    // than the cache) go to the cooperative path after this per-lane pass.
-    const bool is_long = valid && nfull > long_min;
-    const int n = is_long ? -1 : nfull;            // per-lane points
-    const bool vs = valid && !is_long;
-    const int nmax = __reduce_max_sync(FULL, n);
-
-    // ---- own points: cache C, phi, z*phi; bin masses into the usage histogram ----
-    // P(d) for d in [a, b+1] from Q(|z|) = Phi(-|z|) so that both tails keep
-    // relative accuracy: C = Q when z <= 0, 1 - Q otherwise.  Each mass enters
-    // the histogram as round(w P 2^32), split into 16-bit halves (exact sums).
+    if (present) A.win[ci] = (unsigned)a | ((unsigned)(bw + 1) << 16);
+    const int n = valid ? bw - a + 1 : -1;  // points; -1: nothing to add
+    // windows much longer than the warp's typical one go to the cooperative pass
+    // (the results do not depend on the split: the table values are per point
+    // and the histogram sums are exact)
+    const int nact = __popc(__ballot_sync(FULL, valid));
+    const int mean = nact ? __reduce_add_sync(FULL, max(n, 0)) / nact : 0;
+    const bool is_long = valid && n > max(8, 2 * mean + 8);
+    const int nl = is_long ? -1 : n;
+    const int nmax = __reduce_max_sync(FULL, nl);
+    float *row = A.tab + ci * W;
     float zp = 0.f, qp = 0.f;
     for (int j = 0; j <= nmax; ++j) {
-      const bool pt = j < n;                       // point a+j exists
+      const bool pt = j < nl;  // point a+j exists
       const float zc = ((float)(a + j) + 0.5f - mu) * inv_s;
       const float qc = pt ? 0.5f * erfcf(fabsf(zc) * kInvSqrt2) : 0.f;
-      if (pt && j < kc) {
-        const float f = kInvSqrt2Pi * expf(-0.5f * zc * zc);
-        cC[j * T + tid] = zc <= 0.f ? qc : 1.0f - qc;
-        cF[j * T + tid] = f;
-        cZ[j * T + tid] = zc * f;
-      }
-      if (j <= n) hist_add(hlo, hhi, fold_bin(a + j, A.II) * RB + r, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
+      if (pt && j < W) row[j] = zc <= 0.f ? qc : 1.0f - qc;
+      if (j <= nl) hist_add(hlo, hhi, fold_bin(a + j, A.II) * RB + r, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
       zp = zc;
       qp = qc;
     }
     __syncwarp();
-    if (valid) {
-      lo = min(lo, a);
-      hi = max(hi, bw + 1);
-    }
-
-    // own point j: C, phi, z*phi (recomputed beyond the cache)
-    auto own = [&](int j, float &C, float &f, float &zf) {
-      if (j < kc) {
-        C = cC[j * T + tid];
-        f = cF[j * T + tid];
-        zf = cZ[j * T + tid];
-      } else {
-        const float z = ((float)(a + j) + 0.5f - mu) * inv_s;
-        const float q = 0.5f * erfcf(fabsf(z) * kInvSqrt2);
-        C = z <= 0.f ? q : 1.0f - q;
-        f = kInvSqrt2Pi * expf(-0.5f * z * z);
-        zf = z * f;
-      }
-    };
-
-    float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f;
-    // ---- edges: every edge term is a dot product of the own window with the
-    // neighbour's CDF shifted by a latency; only the own points where the
-    // neighbour's values vary (or, for communication, are a constant 1) are
-    // visited, and the neighbour's mean and sigma are read only then. ----
-    // in-edges u -> v (own = consumer), latency L = Lat(u):
-    //   V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
-    //   dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
-    //   dL_com,e/dC_v(t) = -C_u(t)
-    if (kDep || kCom) {
-      const int e0 = A.in_ptr[vcl], deg = vs ? A.in_ptr[vcl + 1] - e0 : 0;
-      const int dmax = __reduce_max_sync(FULL, deg);
-      for (int q = 0; q < dmax; ++q) {
-        const bool eon = q < deg;
-        const int uc = eon ? A.in_src[e0 + q] : 0, L = eon ? A.in_lat[e0 + q] : 0;
-        const unsigned wm = eon ? A.win[(size_t)uc * A.B + b] : 0u;
-        const int au = (int)(wm & 0xFFFFu), bu = (int)(wm >> 16) - 1;
-        // P_u(t+1-L) != 0 for t in [au+L-1, bu+L]; C_u(t) != 0 for t >= au
-        const int jlo = max(0, au + min(kDep ? L - 1 : 0, 0) - a);
-        const int jhi = kCom ? n - 1 : min(n - 1, bu + L - a);
-        const int x0 = bw + 1 - L;
-        const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
-        const bool need = cnt > 0 || (kDep && eon && x0 >= au && x0 <= bu);
-        const float mu_u = need ? A.mu[(size_t)uc * A.B + b] : 0.f;
-        const float inv_u = need ? 1.0f / A.sg[(size_t)uc * A.B + b] : 1.f;
-        const int cmax = __reduce_max_sync(FULL, cnt);
-        float c_lo = cnt ? cdf_at(a + jlo - L, mu_u, inv_u, au, bu) : 0.f;
-        for (int k2 = 0; k2 < cmax; ++k2) {
-          if (k2 < cnt) {
-            const int j = jlo + k2, t = a + j;
-            const float c_hi = cdf_at(t + 1 - L, mu_u, inv_u, au, bu);
-            const float p = c_hi - c_lo;
-            float Cv, f, zf;
-            own(j, Cv, f, zf);
-            if (kDep) {
-              fdep += Cv * p;
-              Ad += p * f;
-              Bd += p * zf;
-            }
-            if (kCom) {
-              const float cu = (L == 1) ? c_hi : cdf_at(t, mu_u, inv_u, au, bu);
-              fcom += cu * (1.0f - Cv);
-              Ao -= A.alpha * cu * f;
-              Bo -= A.alpha * cu * zf;
-            }
-            c_lo = c_hi;
-          }
-        }
-        __syncwarp();
-        if (kDep && eon) fdep += 1.0f - cdf_at(x0, mu_u, inv_u, au, bu);
-      }
-    }
-    // out-edges v -> w (own = producer), latency L = Lat(v):
-    //   dV_e/dC_v(x) = -P_w(x + L), nonzero for x in [aw-L, bw+1-L]
-    //   dL_com,e/dC_v(x) = 1 - C_w(x), nonzero for x <= bw
-    //   L_com,e part = sum_{x in own, x < a_w} C_v(x) + max(0, a_w - 1 - b_v)
-    if (kDep || kCom) {
-      const int L = A.lat[vcl];
-      const int e0 = A.out_ptr[vcl], deg = vs ? A.out_ptr[vcl + 1] - e0 : 0;
-      const int dmax = __reduce_max_sync(FULL, deg);
-      for (int q = 0; q < dmax; ++q) {
-        const bool eon = q < deg;
-        const int wc = eon ? A.out_dst[e0 + q] : 0;
-        const unsigned wm = eon ? A.win[(size_t)wc * A.B + b] : 0u;
-        const int aw = (int)(wm & 0xFFFFu), bw2 = (int)(wm >> 16) - 1;
-        int jlo = max(0, aw - L - a), jhi = min(n - 1, bw2 + 1 - L - a);
-        if (kCom) {
-          jlo = 0;
-          jhi = max(jhi, min(n - 1, bw2 - a));
-        }
-        const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
-        const float mu_w = cnt ? A.mu[(size_t)wc * A.B + b] : 0.f;
-        const float inv_w = cnt ? 1.0f / A.sg[(size_t)wc * A.B + b] : 1.f;
-        const int cmax = __reduce_max_sync(FULL, cnt);
-        float c_lo = cnt ? cdf_at(a + jlo + L - 1, mu_w, inv_w, aw, bw2) : 0.f;
-        for (int k2 = 0; k2 < cmax; ++k2) {
-          if (k2 < cnt) {
-            const int j = jlo + k2, x = a + j;
-            const float c_hi = cdf_at(x + L, mu_w, inv_w, aw, bw2);
-            float Cv, f, zf;
-            own(j, Cv, f, zf);
-            if (kDep) {
-              const float p = c_hi - c_lo;
-              Ad -= p * f;
-              Bd -= p * zf;
-            }
-            if (kCom) {
-              const float cw = (L == 1) ? c_lo : cdf_at(x, mu_w, inv_w, aw, bw2);
-              Ao += A.alpha * (1.0f - cw) * f;
-              Bo += A.alpha * (1.0f - cw) * zf;
-              if (x < aw) fcom += Cv;
-            }
-            c_lo = c_hi;
-          }
-        }
-        __syncwarp();
-        if (kCom && eon) fcom += (float)max(0, aw - 1 - bw);
-      }
-    }
-    // back edges (App. B.3): a dependency with latency Lat(j) - k II
-    if (kRec) {
-      {  // own = consumer i
-        const int e0 = A.bin_ptr[vcl], deg = vs ? A.bin_ptr[vcl + 1] - e0 : 0;
-        const int dmax = __reduce_max_sync(FULL, deg);
-        for (int q = 0; q < dmax; ++q) {
-          const bool eon = q < deg;
-          const int jc = eon ? A.bin_src[e0 + q] : 0, L = eon ? A.bin_shift[e0 + q] : 0;
-          const unsigned wm = eon ? A.win[(size_t)jc * A.B + b] : 0u;
-          const int au = (int)(wm & 0xFFFFu), bu = (int)(wm >> 16) - 1;
-          const int jlo = max(0, au + L - 1 - a), jhi = min(n - 1, bu + L - a);
-          const int x0 = bw + 1 - L;
-          const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
-          const bool need = cnt > 0 || (eon && x0 >= au && x0 <= bu);
-          const float mu_u = need ? A.mu[(size_t)jc * A.B + b] : 0.f;
-          const float inv_u = need ? 1.0f / A.sg[(size_t)jc * A.B + b] : 1.f;
-          const int cmax = __reduce_max_sync(FULL, cnt);
-          float c_lo = cnt ? cdf_at(a + jlo - L, mu_u, inv_u, au, bu) : 0.f;
-          for (int k2 = 0; k2 < cmax; ++k2) {
-            if (k2 < cnt) {
-              const int j = jlo + k2;
-              const float c_hi = cdf_at(a + j + 1 - L, mu_u, inv_u, au, bu);
-              const float p = c_hi - c_lo;
-              float Cv, f, zf;
-              own(j, Cv, f, zf);
-              frec += Cv * p;
-              Ar += p * f;
-              Br += p * zf;
-              c_lo = c_hi;
-            }
-          }
-          __syncwarp();
-          if (eon) frec += 1.0f - cdf_at(x0, mu_u, inv_u, au, bu);
-        }
-      }
-      {  // own = producer j
-        const int e0 = A.bout_ptr[vcl], deg = vs ? A.bout_ptr[vcl + 1] - e0 : 0;
-        const int dmax = __reduce_max_sync(FULL, deg);
-        for (int q = 0; q < dmax; ++q) {
-          const bool eon = q < deg;
-          const int ic = eon ? A.bout_dst[e0 + q] : 0, L = eon ? A.bout_shift[e0 + q] : 0;
-          const unsigned wm = eon ? A.win[(size_t)ic * A.B + b] : 0u;
-          const int aw = (int)(wm & 0xFFFFu), bw2 = (int)(wm >> 16) - 1;
-          const int jlo = max(0, aw - L - a), jhi = min(n - 1, bw2 + 1 - L - a);
-          const int cnt = eon && jhi >= jlo ? jhi - jlo + 1 : 0;
-          const float mu_w = cnt ? A.mu[(size_t)ic * A.B + b] : 0.f;
-          const float inv_w = cnt ? 1.0f / A.sg[(size_t)ic * A.B + b] : 1.f;
-          const int cmax = __reduce_max_sync(FULL, cnt);
-          float c_lo = cnt ? cdf_at(a + jlo + L - 1, mu_w, inv_w, aw, bw2) : 0.f;
-          for (int k2 = 0; k2 < cmax; ++k2) {
-            if (k2 < cnt) {
-              const int j = jlo + k2;
-              const float c_hi = cdf_at(a + j + L, mu_w, inv_w, aw, bw2);
-              const float p = c_hi - c_lo;
-              float Cv, f, zf;
-              own(j, Cv, f, zf);
-              Ar -= p * f;
-              Br -= p * zf;
-              c_lo = c_hi;
-            }
-          }
-          __syncwarp();
-        }
-      }
-    }
-    // ---- cooperative pass over the long windows of this warp ----
     unsigned longmask = __ballot_sync(FULL, is_long);
     while (longmask) {
       const int src = __ffs(longmask) - 1;
       longmask &= longmask - 1;
-      const int l_v = __shfl_sync(FULL, vcl, src), l_b = __shfl_sync(FULL, b, src);
-      const int l_r = __shfl_sync(FULL, r, src), l_a = __shfl_sync(FULL, a, src);
-      const int l_bw = __shfl_sync(FULL, bw, src);
+      const int l_a = __shfl_sync(FULL, a, src), l_n = __shfl_sync(FULL, n, src);
+      const int l_r = __shfl_sync(FULL, r, src), l_vc = __shfl_sync(FULL, vc, src);
+      const int l_b = __shfl_sync(FULL, b, src);
       const float l_mu = __shfl_sync(FULL, mu, src), l_inv = __shfl_sync(FULL, inv_s, src);
       const float l_w = __shfl_sync(FULL, wv, src);
-      float sums[9];
-      coop_item<kDep, kCom, kRec>(A, l_v, l_b, l_r, RB, l_mu, l_inv, l_a, l_bw, l_w, hlo, hhi, sums);
-      if ((threadIdx.x & 31) == src) {
-        Ad = sums[0]; Bd = sums[1]; Ao = sums[2]; Bo = sums[3]; Ar = sums[4]; Br = sums[5];
-        fdep += sums[6]; fcom += sums[7]; frec += sums[8];
+      float *l_row = A.tab + ((size_t)l_vc * A.B + l_b) * W;
+      float z_carry = 0.f, q_carry = 0.f;
+      for (int p0 = 0; p0 <= l_n; p0 += 32) {
+        const int p = p0 + lane;
+        const bool pt = p < l_n;
+        const float z = ((float)(l_a + p) + 0.5f - l_mu) * l_inv;
+        const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
+        if (pt && p < W) l_row[p] = z <= 0.f ? q : 1.0f - q;
+        float zpv = __shfl_up_sync(FULL, z, 1), qpv = __shfl_up_sync(FULL, q, 1);
+        if (lane == 0) { zpv = z_carry; qpv = q_carry; }
+        if (p <= l_n) hist_add(hlo, hhi, fold_bin(l_a + p, A.II) * RB + l_r, l_w * bin_mass(pt, p == 0, z, q, zpv, qpv));
+        z_carry = __shfl_sync(FULL, z, 31);
+        q_carry = __shfl_sync(FULL, q, 31);
       }
     }
-    xdep += to_fix(fdep);
-    xcom += to_fix(fcom);
-    xrec += to_fix(frec);
     if (valid) {
-      A.gpart[0 * VB + gi] = Ad;
-      A.gpart[1 * VB + gi] = Bd;
-      A.gpart[2 * VB + gi] = Ao;
-      A.gpart[3 * VB + gi] = Bo;
-      A.gpart[4 * VB + gi] = Ar;
-      A.gpart[5 * VB + gi] = Br;
+      lo = min(lo, a);
+      hi = max(hi, bw + 1);
     }
   }
 
-  // ---- per-restart forward sums of this block (fixed order), reusing the cache ----
+  // ---- histogram rows restricted to the folded span the block touched ----
   if (lo <= hi) {
     atomicMin(&s_lo, lo);
     atomicMax(&s_hi, hi);
   }
   __syncthreads();
-  long long *red = reinterpret_cast<long long *>(cC);
-  red[0 * T + tid] = xdep;
-  red[1 * T + tid] = xcom;
-  red[2 * T + tid] = xrec;
-  __syncthreads();
-  if (tid < RB) {
-    long long acc[3] = {0, 0, 0};
-    for (int row = 0; row < rows; ++row)
-      for (int k = 0; k < 3; ++k) acc[k] += red[k * T + row * RB + tid];
-    for (int k = 0; k < 3; ++k) A.fwd[((size_t)blk * RB + tid) * 3 + k] = acc[k];
-  }
-  // ---- histogram rows restricted to the folded span the block touched ----
   int flo = s_lo, fhi = s_hi;
   if (flo > fhi) {
     flo = 1;
@@ -568,6 +279,278 @@ __global__ void __launch_bounds__(kFwdThreads) k_fwd(const IterArgs A) {
       const int cell = flo * RB + i;
       dst[cell] = (long long)(((unsigned long long)hhi[cell] << 16) + (unsigned long long)hlo[cell]);
     }
+  }
+}
+
+// One (edge, restart) whose endpoint windows are not both in the table, done by
+// the whole warp with lanes over the points of each endpoint (32 at a time).
+// Same terms and formulas as the per-lane path, with the own values evaluated
+// directly.  Returns the warp-reduced sums on every lane: the producer's and the
+// consumer's partials and the edge's forward sums.
+template <bool kDep, bool kCom>
+__device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, const Nb &Vn, float4 &su, float4 &sv,
+                          float &fd, float &fc, float &fr) {
+  const int lane = threadIdx.x & 31;
+  float s[11] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // su, sv, fd, fc, fr
+  // consumer side: own = v
+  const int nv = Vn.b - Vn.a + 1;
+  for (int base = 0; base == 0 || base < nv; base += 32) {
+    const int pidx = base + lane;
+    const bool pt = pidx < nv;
+    const int t = Vn.a + pidx;
+    const float z = ((float)t + 0.5f - Vn.mu) * Vn.inv;
+    const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
+    const float Cv = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
+    const float f = pt ? kInvSqrt2Pi * expf(-0.5f * z * z) : 0.f;
+    const float zf = z * f;
+    if (!back) {
+      if (pt) {
+        const float c_hi = U.at(t + 1 - L);
+        const float p = c_hi - U.at(t - L);
+        if (kDep) { s[8] += Cv * p; s[4] += p * f; s[5] += p * zf; }
+        if (kCom) {
+          const float cu = (L == 1) ? c_hi : U.at(t);
+          s[9] += cu * (1.0f - Cv);
+          s[6] -= A.alpha * cu * f;
+          s[7] -= A.alpha * cu * zf;
+        }
+      }
+      if (kDep && base == 0 && lane == 0) s[8] += 1.0f - U.at(Vn.b + 1 - L);
+    } else {
+      if (pt) {
+        const float p = U.at(t + 1 - L) - U.at(t - L);
+        s[10] += Cv * p; s[4] += p * f; s[5] += p * zf;
+      }
+      if (base == 0 && lane == 0) s[10] += 1.0f - U.at(Vn.b + 1 - L);
+    }
+  }
+  // producer side: own = u
+  const int nu = U.b - U.a + 1;
+  for (int base = 0; base == 0 || base < nu; base += 32) {
+    const int pidx = base + lane;
+    const bool pt = pidx < nu;
+    const int x = U.a + pidx;
+    const float z = ((float)x + 0.5f - U.mu) * U.inv;
+    const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
+    const float Cu = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
+    const float f = pt ? kInvSqrt2Pi * expf(-0.5f * z * z) : 0.f;
+    const float zf = z * f;
+    if (!back) {
+      if (pt) {
+        const float c_hi = Vn.at(x + L), c_lo = Vn.at(x + L - 1);
+        if (kDep) { const float p = c_hi - c_lo; s[0] -= p * f; s[1] -= p * zf; }
+        if (kCom) {
+          const float cw = (L == 1) ? c_lo : Vn.at(x);
+          s[2] += A.alpha * (1.0f - cw) * f;
+          s[3] += A.alpha * (1.0f - cw) * zf;
+          if (x < Vn.a) s[9] += Cu;
+        }
+      }
+      if (kCom && base == 0 && lane == 0) s[9] += (float)max(0, Vn.a - 1 - U.b);
+    } else if (pt) {
+      const float p = Vn.at(x + L) - Vn.at(x + L - 1);
+      s[0] -= p * f; s[1] -= p * zf;
+    }
+  }
+  __syncwarp();
+#pragma unroll
+  for (int k = 0; k < 11; ++k) s[k] = warp_sum(s[k]);
+  su = make_float4(s[0], s[1], s[2], s[3]);
+  sv = make_float4(s[4], s[5], s[6], s[7]);
+  fd = s[8]; fc = s[9]; fr = s[10];
+}
+
+// Edge pass (Eq. dep, Eq. com, App. B.3).  Block = a chunk of the edge list x one
+// restart group; lane = (edge, restart).  Each edge term is a dot product of one
+// endpoint's window with the other endpoint's CDF shifted by the latency; both
+// endpoints' CDF values come from the table written by k_nodes.  Per (edge,
+// restart) the pass writes the producer's and the consumer's partials
+// (dV/dmu-, dV/dsigma-type sums: Ad, Bd, Ao, Bo for a forward edge, Ar, Br for a
+// back edge) to the edge's two slots, which k_update gathers per node in a fixed
+// order, and adds the edge's forward sums (exact fixed point) to the block's.
+// An edge with an endpoint window longer than the table row is done by the
+// whole warp (coop_edge); the choice depends on that restart's windows only.
+template <bool kDep, bool kCom, bool kRec>
+__global__ void __launch_bounds__(kFwdThreads) k_edges(const IterArgs A) {
+  constexpr int T = kFwdThreads;
+  constexpr unsigned FULL = 0xffffffffu;
+  __shared__ long long s_red[3 * T];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, RB = A.RB, epw = 32 / RB;
+  const int blk = blockIdx.x, ch = blk / A.G, g = blk % A.G;
+  const int e_begin = ch * A.ce, e_end = min(A.nEt, e_begin + A.ce);
+  const int r = tid % RB, b = g * RB + r;
+  const bool bok = b < A.B;
+  long long xdep = 0, xcom = 0, xrec = 0;  // forward sums, exact (order-free) fixed point
+  const int per_pass = (T / 32) * epw;
+  for (int e0 = e_begin + warp * epw; e0 < e_end; e0 += per_pass) {
+    const int e = e0 + lane / RB;
+    const bool present = bok && e < e_end;
+    const int4 ed = present ? __ldg(A.ed + e) : make_int4(0, 0, 0, 0);
+    const int uc = ed.x, vc = ed.y, L = ed.z;
+    const bool back = ed.w != 0;
+    const size_t iu = (size_t)uc * A.B + (bok ? b : 0), iv = (size_t)vc * A.B + (bok ? b : 0);
+    const float mu_u = present ? A.mu[iu] : 0.f, sg_u = present ? A.sg[iu] : 1.f;
+    const float mu_v = present ? A.mu[iv] : 0.f, sg_v = present ? A.sg[iv] : 1.f;
+    const unsigned wu = present ? __ldg(A.win + iu) : 0u, wv = present ? __ldg(A.win + iv) : 0u;
+    const bool on = present && usable(mu_u, sg_u) && usable(mu_v, sg_v);
+    Nb U, Vn;
+    U.a = (int)(wu & 0xFFFFu); U.b = (int)(wu >> 16) - 1; U.row = A.tab + iu * A.W;
+    Vn.a = (int)(wv & 0xFFFFu); Vn.b = (int)(wv >> 16) - 1; Vn.row = A.tab + iv * A.W;
+    U.mu = on ? mu_u : 0.f; U.inv = on ? 1.0f / sg_u : 1.f;
+    Vn.mu = on ? mu_v : 0.f; Vn.inv = on ? 1.0f / sg_v : 1.f;
+    const int nu = U.b - U.a + 1, nv = Vn.b - Vn.a + 1;
+    U.tab = nu <= A.W;
+    Vn.tab = nv <= A.W;
+    const bool is_long = on && !(U.tab && Vn.tab);
+    const bool ps = on && !is_long;                 // per-lane path
+    const bool fw = ps && !back && (kDep || kCom);  // forward edge terms
+    const bool bk = kRec && ps && back;             // back edge term
+    float4 su = make_float4(0.f, 0.f, 0.f, 0.f), sv = make_float4(0.f, 0.f, 0.f, 0.f);
+    float fd = 0.f, fc = 0.f, fr = 0.f;
+
+    // own point j of the consumer (v) / producer (u): C from the table, phi, z phi
+    auto own = [&](const Nb &o, int j, float &C, float &f, float &zf) {
+      C = __ldg(o.row + j);
+      const float z = ((float)(o.a + j) + 0.5f - o.mu) * o.inv;
+      f = kInvSqrt2Pi * __expf(-0.5f * z * z);
+      zf = z * f;
+    };
+
+    // ---- consumer side (own = v):
+    //   V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
+    //   dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
+    //   dL_com,e/dC_v(t) = -C_u(t)
+    {
+      // P_u(t+1-L) != 0 for t in [au+L-1, bu+L]; C_u(t) != 0 for t >= au
+      int jlo = 0, jhi = -1;
+      if (fw) {
+        jlo = max(0, U.a + min(kDep ? L - 1 : 0, 0) - Vn.a);
+        jhi = kCom ? nv - 1 : min(nv - 1, U.b + L - Vn.a);
+      } else if (bk) {
+        jlo = max(0, U.a + L - 1 - Vn.a);
+        jhi = min(nv - 1, U.b + L - Vn.a);
+      }
+      const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
+      const int cmax = __reduce_max_sync(FULL, cnt);
+      float c_lo = cnt ? U.at(Vn.a + jlo - L) : 0.f;
+      for (int k2 = 0; k2 < cmax; ++k2) {
+        if (k2 < cnt) {
+          const int j = jlo + k2, t = Vn.a + j;
+          const float c_hi = U.at(t + 1 - L);
+          const float p = c_hi - c_lo;
+          float Cv, f, zf;
+          own(Vn, j, Cv, f, zf);
+          if (back) {
+            fr += Cv * p;
+            sv.x += p * f;
+            sv.y += p * zf;
+          } else {
+            if (kDep) {
+              fd += Cv * p;
+              sv.x += p * f;
+              sv.y += p * zf;
+            }
+            if (kCom) {
+              const float cu = (L == 1) ? c_hi : U.at(t);
+              fc += cu * (1.0f - Cv);
+              sv.z -= A.alpha * cu * f;
+              sv.w -= A.alpha * cu * zf;
+            }
+          }
+          c_lo = c_hi;
+        }
+      }
+      __syncwarp();
+      if ((kDep && fw) || bk) {
+        const float tail = 1.0f - U.at(Vn.b + 1 - L);
+        if (back) fr += tail; else fd += tail;
+      }
+    }
+    // ---- producer side (own = u):
+    //   dV_e/dC_u(x) = -P_v(x + L), nonzero for x in [av-L, bv+1-L]
+    //   dL_com,e/dC_u(x) = 1 - C_v(x), nonzero for x <= bv
+    //   L_com,e part = sum_{x in own, x < a_v} C_u(x) + max(0, a_v - 1 - b_u)
+    {
+      int jlo = 0, jhi = -1;
+      if (fw || bk) {
+        jlo = max(0, Vn.a - L - U.a);
+        jhi = min(nu - 1, Vn.b + 1 - L - U.a);
+        if (kCom && fw) {
+          jlo = 0;
+          jhi = max(jhi, min(nu - 1, Vn.b - U.a));
+        }
+      }
+      const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
+      const int cmax = __reduce_max_sync(FULL, cnt);
+      float c_lo = cnt ? Vn.at(U.a + jlo + L - 1) : 0.f;
+      for (int k2 = 0; k2 < cmax; ++k2) {
+        if (k2 < cnt) {
+          const int j = jlo + k2, x = U.a + j;
+          const float c_hi = Vn.at(x + L);
+          float Cu, f, zf;
+          own(U, j, Cu, f, zf);
+          if (back || kDep) {
+            const float p = c_hi - c_lo;
+            su.x -= p * f;
+            su.y -= p * zf;
+          }
+          if (kCom && !back) {
+            const float cw = (L == 1) ? c_lo : Vn.at(x);
+            su.z += A.alpha * (1.0f - cw) * f;
+            su.w += A.alpha * (1.0f - cw) * zf;
+            if (x < Vn.a) fc += Cu;
+          }
+          c_lo = c_hi;
+        }
+      }
+      __syncwarp();
+      if (kCom && fw) fc += (float)max(0, Vn.a - 1 - U.b);
+    }
+    // ---- cooperative pass over this warp's long (edge, restart) items ----
+    unsigned longmask = __ballot_sync(FULL, is_long);
+    while (longmask) {
+      const int src = __ffs(longmask) - 1;
+      longmask &= longmask - 1;
+      Nb lu, lv;
+      lu.a = __shfl_sync(FULL, U.a, src); lu.b = __shfl_sync(FULL, U.b, src);
+      lu.tab = __shfl_sync(FULL, (int)U.tab, src) != 0;
+      lu.mu = __shfl_sync(FULL, U.mu, src); lu.inv = __shfl_sync(FULL, U.inv, src);
+      lv.a = __shfl_sync(FULL, Vn.a, src); lv.b = __shfl_sync(FULL, Vn.b, src);
+      lv.tab = __shfl_sync(FULL, (int)Vn.tab, src) != 0;
+      lv.mu = __shfl_sync(FULL, Vn.mu, src); lv.inv = __shfl_sync(FULL, Vn.inv, src);
+      const int l_uc = __shfl_sync(FULL, uc, src), l_vc = __shfl_sync(FULL, vc, src);
+      const int l_b = __shfl_sync(FULL, b, src), l_L = __shfl_sync(FULL, L, src);
+      const bool l_back = __shfl_sync(FULL, (int)back, src) != 0;
+      lu.row = A.tab + ((size_t)l_uc * A.B + l_b) * A.W;
+      lv.row = A.tab + ((size_t)l_vc * A.B + l_b) * A.W;
+      float4 csu, csv;
+      float cfd, cfc, cfr;
+      if (!l_back) coop_edge<kDep, kCom>(A, false, l_L, lu, lv, csu, csv, cfd, cfc, cfr);
+      else coop_edge<true, false>(A, true, l_L, lu, lv, csu, csv, cfd, cfc, cfr);
+      if (lane == src) {
+        su = csu; sv = csv;
+        fd = cfd; fc = cfc; fr = cfr;
+      }
+    }
+    if (present) {
+      A.eslot4[(size_t)(2 * e) * A.B + b] = su;
+      A.eslot4[(size_t)(2 * e + 1) * A.B + b] = sv;
+    }
+    xdep += to_fix(fd);
+    xcom += to_fix(fc);
+    xrec += to_fix(fr);
+  }
+
+  // ---- per-restart forward sums of this block (fixed order) ----
+  s_red[0 * T + tid] = xdep;
+  s_red[1 * T + tid] = xcom;
+  s_red[2 * T + tid] = xrec;
+  __syncthreads();
+  if (tid < RB) {
+    long long acc[3] = {0, 0, 0};
+    for (int row = 0; row < T / RB; ++row)
+      for (int k = 0; k < 3; ++k) acc[k] += s_red[k * T + row * RB + tid];
+    for (int k = 0; k < 3; ++k) A.fwd[((size_t)blk * RB + tid) * 3 + k] = acc[k];
   }
 }
 
@@ -604,17 +587,6 @@ __global__ void __launch_bounds__(256) k_reduce(const RedArgs A) {
     long long tot = 0;
     for (int k = 0; k < nsl; ++k) tot += part[k * RB + r];
     A.U[((size_t)b * A.C + c) * Dh + d] = tot;
-  }
-}
-
-// Window of every (node, restart): a | (b + 1) << 16 with the points [a, b] of
-// window(); an unusable mean/sigma gets the empty window at the horizon start.
-__global__ void k_windows(const float *mu, const float *sg, unsigned *win, size_t n, float k, int D) {
-  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
-    int a = 0, b = -1;
-    const float m = mu[i], s = sg[i];
-    if (usable(m, s)) window(m, s, k, D, a, b);
-    win[i] = (unsigned)a | ((unsigned)(b + 1) << 16);
   }
 }
 
@@ -683,8 +655,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
 
   // forward sums of the edge terms over every block of this restart group
   long long f3[3] = {0, 0, 0};
-  const int nseg = A.cls_seg_ptr[A.C];
-  for (int s = tid; s < nseg; s += 256)
+  for (int s = tid; s < A.nfwd; s += 256)
     for (int k = 0; k < 3; ++k) f3[k] += A.fwd[((size_t)(s * A.G + g) * A.RB + r) * 3 + k];
   const float vdep = (float)((double)block_sum_i64(f3[0], shl) * kInvFix);
   const float lcom = (float)((double)block_sum_i64(f3[1], shl) * kInvFix);
@@ -785,7 +756,6 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
     __syncthreads();
     long_min = max(8, 2 * seg_mean_window(A.win, A.perm, s0, s1, b, bok, A.B, tid, RB, rows, s_wsum, s_wcnt) + 8);
   }
-  const size_t VB = (size_t)A.V * A.B;
   const int bs = bok ? b : 0;
   const float c_dep = A.coef[bs * 4 + 0], c_rec = A.coef[bs * 4 + 1];
   const float bc1 = kAdam ? A.coef[bs * 4 + 2] : 1.f, bc2 = kAdam ? A.coef[bs * 4 + 3] : 1.f;
@@ -847,8 +817,34 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
       }
     }
     if (!valid) continue;
-    float Asum = c_dep * A.gpart[0 * VB + gi] + A.gpart[2 * VB + gi] + c_rec * A.gpart[4 * VB + gi] + Ah;
-    float Bsum = c_dep * A.gpart[1 * VB + gi] + A.gpart[3 * VB + gi] + c_rec * A.gpart[5 * VB + gi] + Bh;
+    // the node's edge partials in a fixed order: out-edges, in-edges, back edges
+    float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f;
+    if (ok) {
+      for (int e = A.out_ptr[vi]; e < A.out_ptr[vi + 1]; ++e) {
+        const float4 s = A.eslot4[(size_t)(2 * e) * A.B + b];
+        Ad += s.x; Bd += s.y; Ao += s.z; Bo += s.w;
+      }
+      for (int e = A.in_ptr[vi]; e < A.in_ptr[vi + 1]; ++e) {
+        const float4 s = A.eslot4[(size_t)(2 * A.in_eslot[e] + 1) * A.B + b];
+        Ad += s.x; Bd += s.y; Ao += s.z; Bo += s.w;
+      }
+      if (A.has_back) {
+        for (int e = A.bout_ptr[vi]; e < A.bout_ptr[vi + 1]; ++e) {
+          const float4 s = A.eslot4[(size_t)(2 * (A.E + e)) * A.B + b];
+          Ar += s.x; Br += s.y;
+        }
+        for (int e = A.bin_ptr[vi]; e < A.bin_ptr[vi + 1]; ++e) {
+          const float4 s = A.eslot4[(size_t)(2 * (A.E + A.bin_eslot[e]) + 1) * A.B + b];
+          Ar += s.x; Br += s.y;
+        }
+      }
+      if (A.gown) {
+        const float2 s = A.gown[gi];
+        Ao += s.x; Bo += s.y;
+      }
+    }
+    float Asum = c_dep * Ad + Ao + c_rec * Ar + Ah;
+    float Bsum = c_dep * Bd + Bo + c_rec * Br + Bh;
     if (A.eslot && ok)
       for (int e = A.in_ptr[vi]; e < A.in_ptr[vi + 1]; ++e) {
         const float2 sh = A.eslot[(size_t)A.in_eslot[e] * A.B + b];

@@ -211,6 +211,7 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
   }
   for (int i = 0; i < V; ++i) { P.bin_ptr[i + 1] += P.bin_ptr[i]; P.bout_ptr[i + 1] += P.bout_ptr[i]; }
   P.bin_src.resize(NB); P.bin_shift.resize(NB); P.bout_dst.resize(NB); P.bout_shift.resize(NB);
+  P.bin_eslot.resize(NB);
   {
     std::vector<int32_t> fi(P.bin_ptr.begin(), P.bin_ptr.end() - 1), fo(P.bout_ptr.begin(), P.bout_ptr.end() - 1);
     for (int q = 0; q < NB; ++q) {
@@ -220,8 +221,27 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
       P.bin_src[a] = j; P.bin_shift[a] = shift;
       int b = fo[P.inv[j]]++;
       P.bout_dst[b] = i; P.bout_shift[b] = shift;
+      P.bin_eslot[a] = b;
     }
   }
+  // edge list of the edge pass: forward edges in internal CSR order (producer,
+  // consumer, Lat(producer), 0), then back edges in producer order (j, i, shift, 1)
+  P.ed.resize(4 * ((size_t)E + NB));
+  for (int i = 0; i < V; ++i)
+    for (int o = P.out_ptr[i]; o < P.out_ptr[i + 1]; ++o) {
+      P.ed[4 * (size_t)o + 0] = P.perm[i];
+      P.ed[4 * (size_t)o + 1] = P.out_dst[o];
+      P.ed[4 * (size_t)o + 2] = P.lat[i];
+      P.ed[4 * (size_t)o + 3] = 0;
+    }
+  for (int i = 0; i < V; ++i)
+    for (int q = P.bout_ptr[i]; q < P.bout_ptr[i + 1]; ++q) {
+      const size_t k = 4 * ((size_t)E + q);
+      P.ed[k + 0] = P.perm[i];
+      P.ed[k + 1] = P.bout_dst[q];
+      P.ed[k + 2] = P.bout_shift[q];
+      P.ed[k + 3] = 1;
+    }
   // caller-order CSC / CSR / back edges for the integer kernels
   P.cpred_ptr.assign(p->pred_ptr, p->pred_ptr + V + 1);
   P.cpred_src.assign(p->pred_idx, p->pred_idx + E);

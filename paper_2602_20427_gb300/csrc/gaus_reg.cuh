@@ -41,7 +41,7 @@ struct RegArgs {
   long long *rpart;                  // blocks * Dh * RB
   // backward
   const float *Hreg;                 // (B, Dh): w_mem * softmax of (M)Reg
-  float *gpart;                      // 6 * V * B; slots 2, 3 receive the own adjoint
+  float2 *gown;                      // (V, B) internal order: the own-window adjoint
   float2 *eslot;                     // (E, B) per out-edge slot (CSR position)
 };
 
@@ -219,7 +219,6 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
   __syncthreads();
 
   const int lane = tid & 31, r = tid % RB, b = g * RB + r, npw = 32 / RB;
-  const size_t VB = (size_t)A.V * A.B;
   for (;;) {
     int base = 0;
     if (lane == 0) base = atomicAdd(&s_next, npw);
@@ -255,11 +254,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
       }
     }
     __syncwarp();
-    if (valid) {
-      const size_t gi = (size_t)vcl * A.B + b;
-      A.gpart[2 * VB + gi] += Ao;
-      A.gpart[3 * VB + gi] += Bo;
-    }
+    if (valid) A.gown[(size_t)vcl * A.B + b] = make_float2(Ao, Bo);
     // successors' shares: dL/dC_j(d) = -G(d) b_i C_i(d) prod_{j' != j} C_j'(d) on j's window
     for (int q = 0; q < dmax; ++q) {
       const bool eon = q < deg;
