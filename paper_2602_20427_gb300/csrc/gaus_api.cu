@@ -70,7 +70,7 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   A.bout_ptr = ctx->d_bout_ptr; A.bout_dst = ctx->d_bout_dst; A.bout_shift = ctx->d_bout_shift;
   A.seg = ctx->d_seg; A.hpart = ctx->d_hpart; A.hspan = ctx->d_hspan; A.fwd = ctx->d_fwd;
   A.nonfinite = ctx->d_nonfinite; A.win = ctx->d_win; A.tab = ctx->d_tab;
-  A.ed = ctx->d_ed; A.nEt = P.E + P.NB; A.ce = ctx->ce; A.eslot4 = ctx->d_eslot4;
+  A.ed = ctx->d_ed; A.nEt = P.E + P.NB; A.ce = ctx->ce; A.E = P.E; A.eslot4 = ctx->d_eslot4;
   return A;
 }
 
@@ -146,12 +146,12 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
 
   UpdArgs U;
   U.in_ptr = ctx->d_in_ptr; U.in_eslot = ctx->d_in_eslot; U.out_ptr = ctx->d_out_ptr;
-  U.bin_ptr = ctx->d_bin_ptr; U.bin_eslot = ctx->d_bin_eslot; U.bout_ptr = ctx->d_bout_ptr;
-  U.E = P.E; U.has_back = (on & GAUS_REC) && P.II > 0 && P.NB > 0; U.eslot4 = ctx->d_eslot4;
+  U.bin_ptr = ctx->d_bin_ptr; U.bout_ptr = ctx->d_bout_ptr;
+  U.E = P.E; U.nEt = P.E + P.NB; U.has_back = (on & GAUS_REC) && P.II > 0 && P.NB > 0; U.eslot4 = ctx->d_eslot4;
   U.eslot = reg ? ctx->d_eslot : nullptr; U.gown = reg ? ctx->d_gown : nullptr;
   U.mu = const_cast<float *>(mu); U.sg = const_cast<float *>(sg);
   U.V = P.V; U.B = P.B; U.D = P.D; U.II = P.II; U.Dh = P.Dh; U.C = P.C; U.RB = ctx->RB; U.G = ctx->G;
-  U.k_win = ctx->hp.window_k; U.perm = ctx->d_perm; U.win = ctx->d_win; U.w = ctx->d_w; U.seg = ctx->d_seg;
+  U.k_win = ctx->hp.window_k; U.W = ctx->W; U.perm = ctx->d_perm; U.cls = ctx->d_cls; U.w = ctx->d_w;
   U.H = ctx->d_H; U.coef = ctx->d_coef;
   U.grad_mu = grad_mu; U.grad_sg = grad_sg;
   U.m_mu = adam ? S->m_mu : nullptr; U.v_mu = adam ? S->v_mu : nullptr;
@@ -161,11 +161,11 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   U.sigma_min = ctx->hp.sigma_min;
   const bool hist = on & (GAUS_RES_OBJ | GAUS_RES_VIOL);
   if (adam) {
-    if (hist) k_update<true, true><<<ctx->nblk, kThreads, 0, st>>>(U);
-    else k_update<true, false><<<ctx->nblk, kThreads, 0, st>>>(U);
+    if (hist) k_update<true, true><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
+    else k_update<true, false><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
   } else {
-    if (hist) k_update<false, true><<<ctx->nblk, kThreads, 0, st>>>(U);
-    else k_update<false, false><<<ctx->nblk, kThreads, 0, st>>>(U);
+    if (hist) k_update<false, true><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
+    else k_update<false, false><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
   }
   CK(cudaGetLastError(), "k_update launch");
   if (ev) CK(cudaEventRecord(ev[4], st), "event");
@@ -215,6 +215,11 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     ce = (ce + per_pass - 1) / per_pass * per_pass;
     ctx->ce = (int)ce;
     ctx->nchunk = std::max(1, (int)((nEt + ce - 1) / ce));
+  }
+  // k_update: one warp-item (32 / RB nodes x one restart group) per warp
+  {
+    const long nwi = ((long)P.V + (32 / ctx->RB) - 1) / (32 / ctx->RB) * ctx->G;
+    ctx->nblk_u = (int)std::max(1L, (nwi + kUpdThreads / 32 - 1) / (kUpdThreads / 32));
   }
   ctx->red_blocks = ctx->G * P.C * P.Dh;
   // k_nodes shared memory: the two halves of the usage histogram
@@ -267,7 +272,6 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(upload(ctx, &ctx->d_out_ptr, P.out_ptr));
   TRY(upload(ctx, &ctx->d_out_dst, P.out_dst));
   TRY(upload(ctx, &ctx->d_in_eslot, P.in_eslot));
-  TRY(upload(ctx, &ctx->d_bin_eslot, P.bin_eslot));
   {
     int32_t *ed = nullptr;
     TRY(upload(ctx, &ed, P.ed));

@@ -15,6 +15,7 @@ namespace gaus {
 constexpr int kFwdThreads = 256;
 constexpr int kThreads = 128;
 // Most own-window points cached in shared memory per thread (longer windows recompute).
+constexpr int kUpdThreads = 256;               // threads per k_update block
 constexpr int kTableMax = 32;                    // points per CDF table row, at most
 constexpr size_t kTableBytes = (size_t)64 << 20;  // CDF table size bound
 // Fixed-point scale of the usage histograms: P * 2^32 accumulated in int64.
@@ -78,6 +79,7 @@ struct gaus_ctx {
   std::string err;
   int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per node pass
   int ce = 0, nchunk = 0;        // edge pass: edges per block, edge chunks (blocks = nchunk * G)
+  int nblk_u = 0;                // k_update blocks
   int W = 0;                     // points per CDF table row
   int red_blocks = 0;
   int RBr = 32, Gr = 1, nblk_r = 0;  // storage-term kernels: restarts per row, groups, blocks
@@ -110,7 +112,6 @@ struct gaus_ctx {
   float *d_Hreg = nullptr;       // B * Dh storage adjoint
   float2 *d_eslot = nullptr;     // E * B successor shares of the storage gradient
   int32_t *d_in_eslot = nullptr; // E
-  int32_t *d_bin_eslot = nullptr;  // NB
   int4 *d_ed = nullptr;          // E + NB edge list of the edge pass
   float4 *d_eslot4 = nullptr;    // 2 (E + NB) * B per-edge partials [edge][side][restart]
   float2 *d_gown = nullptr;      // V * B own-window storage adjoint (internal index)

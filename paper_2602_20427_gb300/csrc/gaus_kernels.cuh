@@ -50,8 +50,10 @@ struct IterArgs {
   unsigned *win;  // (V, B) packed windows a | (b + 1) << 16, written by k_nodes
   float *tab;     // (V, B, W) CDF values at the window points, written by k_nodes
   const int4 *ed; // edge list of the edge pass (nEt = E + NB edges, ce per block)
-  int nEt, ce;
-  float4 *eslot4; // (2 nEt, B) per-edge partials: [edge][producer, consumer][restart]
+  int nEt, ce, E;
+  float4 *eslot4; // per-edge partials [side][position][restart]: producer side at
+                  // the edge's index (CSR / bout order), consumer side at its
+                  // CSC / bin position (+E for back edges), offset nEt * B
 };
 
 struct RedArgs {
@@ -88,18 +90,17 @@ struct UpdArgs {
   // out_ptr), in-edges (in_eslot maps CSC to CSR position), back edges out
   // (positions E + bout_ptr) and in (bin_eslot maps bin to bout position)
   const int32_t *in_ptr, *in_eslot, *out_ptr;
-  const int32_t *bin_ptr, *bin_eslot, *bout_ptr;
-  int E, has_back;
+  const int32_t *bin_ptr, *bout_ptr;
+  int E, nEt, has_back;
   const float4 *eslot4;
   const float2 *eslot;               // storage term: successor shares (NULL when off)
   const float2 *gown;                // storage term: own-window adjoint (NULL when off)
   float *mu, *sg;  // caller order; written when adam
   int V, B, D, II, Dh, C, RB, G;
   float k_win;
-  const int32_t *perm;
-  const unsigned *win;  // (V, B) packed windows of the state being updated
+  int W;  // table row length: longer own windows are done by the whole warp
+  const int32_t *perm, *cls;
   const float *w;
-  const int32_t *seg;
   const float *H, *coef;
   float *grad_mu, *grad_sg;                  // gradient mode
   float *m_mu, *v_mu, *m_sg, *v_sg;          // Adam mode
@@ -371,7 +372,7 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
 // An edge with an endpoint window longer than the table row is done by the
 // whole warp (coop_edge); the choice depends on that restart's windows only.
 template <bool kDep, bool kCom, bool kRec>
-__global__ void __launch_bounds__(kFwdThreads) k_edges(const IterArgs A) {
+__global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   constexpr int T = kFwdThreads;
   constexpr unsigned FULL = 0xffffffffu;
   __shared__ long long s_red[3 * T];
@@ -387,7 +388,8 @@ __global__ void __launch_bounds__(kFwdThreads) k_edges(const IterArgs A) {
     const bool present = bok && e < e_end;
     const int4 ed = present ? __ldg(A.ed + e) : make_int4(0, 0, 0, 0);
     const int uc = ed.x, vc = ed.y, L = ed.z;
-    const bool back = ed.w != 0;
+    const bool back = (ed.w & 1) != 0;
+    const int cpos = (ed.w >> 1) + (back ? A.E : 0);  // consumer-side slot
     const size_t iu = (size_t)uc * A.B + (bok ? b : 0), iv = (size_t)vc * A.B + (bok ? b : 0);
     const float mu_u = present ? A.mu[iu] : 0.f, sg_u = present ? A.sg[iu] : 1.f;
     const float mu_v = present ? A.mu[iv] : 0.f, sg_v = present ? A.sg[iv] : 1.f;
@@ -533,8 +535,8 @@ __global__ void __launch_bounds__(kFwdThreads) k_edges(const IterArgs A) {
       }
     }
     if (present) {
-      A.eslot4[(size_t)(2 * e) * A.B + b] = su;
-      A.eslot4[(size_t)(2 * e + 1) * A.B + b] = sv;
+      A.eslot4[(size_t)e * A.B + b] = su;
+      A.eslot4[((size_t)A.nEt + cpos) * A.B + b] = sv;
     }
     xdep += to_fix(fd);
     xcom += to_fix(fc);
@@ -740,43 +742,38 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   (void)kInvFixF;
 }
 
+// Gradient and Adam step (Sec. 3.3).  Warp-item = 32 / RB internal nodes x one
+// restart group (lanes are restarts), taken grid-stride.  Per (node, restart):
+// the usage adjoint over the own window, dL/dC_v(t) = w_v (H(t) - H(t+1)); the
+// node's edge partials from the edge pass in a fixed order (out-edges, in-edges,
+// back edges out and in, all contiguous per node); the combined gradient
+//   dL/dmu = -(c_dep Ad + Ao + c_rec Ar + Ah) / sigma, same with B.. for sigma,
+// and, in Adam mode, the Adam step with the per-restart bias corrections.
+// Windows longer than the table row are done by the whole warp.
 template <bool kAdam, bool kHist>
-__global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
+__global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
   constexpr unsigned FULL = 0xffffffffu;
-  const int tid = threadIdx.x, RB = A.RB, Dh = A.Dh;
-  const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
-  const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1], c = A.seg[3 * segi + 2];
-  const float *Hc = A.H + (size_t)c * Dh * A.B;  // usage adjoint of this class, [bin][restart]
-  const int r = tid % RB, b = g * RB + r, rows = kThreads / RB;
-  const bool bok = b < A.B;
-  __shared__ int s_wsum[32], s_wcnt[32];
-  int long_min = 0;
-  if (kHist) {
-    if (tid < 32) { s_wsum[tid] = 0; s_wcnt[tid] = 0; }
-    __syncthreads();
-    long_min = max(8, 2 * seg_mean_window(A.win, A.perm, s0, s1, b, bok, A.B, tid, RB, rows, s_wsum, s_wcnt) + 8);
-  }
-  const int bs = bok ? b : 0;
-  const float c_dep = A.coef[bs * 4 + 0], c_rec = A.coef[bs * 4 + 1];
-  const float bc1 = kAdam ? A.coef[bs * 4 + 2] : 1.f, bc2 = kAdam ? A.coef[bs * 4 + 3] : 1.f;
-  const int n_items = (s1 - s0 + rows - 1) / rows;
-  for (int it = 0; it < n_items; ++it) {
-    const int vi = s0 + tid / RB + it * rows;
-    const bool valid = bok && vi < s1;
-    const int vcl = valid ? vi : s0;
+  const int lane = threadIdx.x & 31, RB = A.RB, npw = 32 / RB, Dh = A.Dh;
+  const int r = lane % RB;
+  const int nwi = (A.V + npw - 1) / npw * A.G;
+  const int wstride = gridDim.x * (kUpdThreads / 32);
+  const size_t nP = (size_t)A.nEt * A.B;  // consumer-side slots follow the producer side
+  for (int wi = blockIdx.x * (kUpdThreads / 32) + (threadIdx.x >> 5); wi < nwi; wi += wstride) {
+    const int g = wi % A.G, vi = (wi / A.G) * npw + lane / RB, b = g * RB + r;
+    const bool valid = b < A.B && vi < A.V;
+    const int vcl = valid ? vi : 0, bs = valid ? b : 0;
     const int vc = A.perm[vcl];
     const size_t ci = (size_t)vc * A.B + bs, gi = (size_t)vcl * A.B + bs;
     const float mu = valid ? A.mu[ci] : 0.f, sg = valid ? A.sg[ci] : 1.f;
     const bool ok = valid && usable(mu, sg);
     float Ah = 0.f, Bh = 0.f;
     if (kHist) {
-      // dL/dC_v(t) = w_v (H(t) - H(t+1)) for the own points (P = C(t) - C(t-1));
-      // windows much longer than the warp's typical one are done by the whole warp
+      const float *Hc = A.H + (size_t)A.cls[vcl] * Dh * A.B;  // [bin][restart]
       const float inv_s = ok ? 1.0f / sg : 1.0f, wv = A.w[vcl];
       int a = 0, bw = -1;
       if (ok) window(mu, sg, A.k_win, A.D, a, bw);
       const int nfull = bw - a + 1;
-      const bool is_long = ok && nfull > long_min;
+      const bool is_long = ok && nfull > A.W;
       const int n = is_long ? 0 : nfull;
       const int nmax = __reduce_max_sync(FULL, n);
       for (int j = 0; j < nmax; ++j) {
@@ -798,22 +795,23 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
         const int l_b = __shfl_sync(FULL, b, src);
         const float l_mu = __shfl_sync(FULL, mu, src), l_inv = __shfl_sync(FULL, inv_s, src);
         const float l_w = __shfl_sync(FULL, wv, src);
+        const float *l_H = A.H + (size_t)A.cls[__shfl_sync(FULL, vcl, src)] * Dh * A.B;
         float pa = 0.f, pb = 0.f;
         for (int base = 0; base < l_n; base += 32) {
-          const int j = base + (threadIdx.x & 31);
+          const int j = base + lane;
           if (j < l_n) {
             const int t = l_a + j;
             const float z = ((float)t + 0.5f - l_mu) * l_inv;
             const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
-            const float gh = l_w * (Hc[(size_t)fold_bin(t, A.II) * A.B + l_b] -
-                                    Hc[(size_t)fold_bin(t + 1, A.II) * A.B + l_b]);
+            const float gh = l_w * (l_H[(size_t)fold_bin(t, A.II) * A.B + l_b] -
+                                    l_H[(size_t)fold_bin(t + 1, A.II) * A.B + l_b]);
             pa += gh * f;
             pb += gh * z * f;
           }
         }
         pa = warp_sum(pa);
         pb = warp_sum(pb);
-        if ((threadIdx.x & 31) == src) { Ah = pa; Bh = pb; }
+        if (lane == src) { Ah = pa; Bh = pb; }
       }
     }
     if (!valid) continue;
@@ -821,20 +819,20 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
     float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f;
     if (ok) {
       for (int e = A.out_ptr[vi]; e < A.out_ptr[vi + 1]; ++e) {
-        const float4 s = A.eslot4[(size_t)(2 * e) * A.B + b];
+        const float4 s = A.eslot4[(size_t)e * A.B + b];
         Ad += s.x; Bd += s.y; Ao += s.z; Bo += s.w;
       }
       for (int e = A.in_ptr[vi]; e < A.in_ptr[vi + 1]; ++e) {
-        const float4 s = A.eslot4[(size_t)(2 * A.in_eslot[e] + 1) * A.B + b];
+        const float4 s = A.eslot4[nP + (size_t)e * A.B + b];
         Ad += s.x; Bd += s.y; Ao += s.z; Bo += s.w;
       }
       if (A.has_back) {
         for (int e = A.bout_ptr[vi]; e < A.bout_ptr[vi + 1]; ++e) {
-          const float4 s = A.eslot4[(size_t)(2 * (A.E + e)) * A.B + b];
+          const float4 s = A.eslot4[(size_t)(A.E + e) * A.B + b];
           Ar += s.x; Br += s.y;
         }
         for (int e = A.bin_ptr[vi]; e < A.bin_ptr[vi + 1]; ++e) {
-          const float4 s = A.eslot4[(size_t)(2 * (A.E + A.bin_eslot[e]) + 1) * A.B + b];
+          const float4 s = A.eslot4[nP + (size_t)(A.E + e) * A.B + b];
           Ar += s.x; Br += s.y;
         }
       }
@@ -843,6 +841,7 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
         Ao += s.x; Bo += s.y;
       }
     }
+    const float c_dep = A.coef[b * 4 + 0], c_rec = A.coef[b * 4 + 1];
     float Asum = c_dep * Ad + Ao + c_rec * Ar + Ah;
     float Bsum = c_dep * Bd + Bo + c_rec * Br + Bh;
     if (A.eslot && ok)
@@ -857,6 +856,7 @@ __global__ void __launch_bounds__(kThreads) k_update(const UpdArgs A) {
       A.grad_mu[ci] = gm;
       A.grad_sg[ci] = gs;
     } else {
+      const float bc1 = A.coef[b * 4 + 2], bc2 = A.coef[b * 4 + 3];
       const float m1 = A.beta1 * A.m_mu[ci] + (1.0f - A.beta1) * gm;
       const float v1 = A.beta2 * A.v_mu[ci] + (1.0f - A.beta2) * gm * gm;
       const float m2 = A.beta1 * A.m_sg[ci] + (1.0f - A.beta1) * gs;

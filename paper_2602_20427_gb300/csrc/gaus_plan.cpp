@@ -225,23 +225,31 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
     }
   }
   // edge list of the edge pass: forward edges in internal CSR order (producer,
-  // consumer, Lat(producer), 0), then back edges in producer order (j, i, shift, 1)
-  P.ed.resize(4 * ((size_t)E + NB));
-  for (int i = 0; i < V; ++i)
-    for (int o = P.out_ptr[i]; o < P.out_ptr[i + 1]; ++o) {
-      P.ed[4 * (size_t)o + 0] = P.perm[i];
-      P.ed[4 * (size_t)o + 1] = P.out_dst[o];
-      P.ed[4 * (size_t)o + 2] = P.lat[i];
-      P.ed[4 * (size_t)o + 3] = 0;
-    }
-  for (int i = 0; i < V; ++i)
-    for (int q = P.bout_ptr[i]; q < P.bout_ptr[i + 1]; ++q) {
-      const size_t k = 4 * ((size_t)E + q);
-      P.ed[k + 0] = P.perm[i];
-      P.ed[k + 1] = P.bout_dst[q];
-      P.ed[k + 2] = P.bout_shift[q];
-      P.ed[k + 3] = 1;
-    }
+  // consumer, Lat(producer), kind | consumer position << 1), then back edges in
+  // producer order (j, i, shift, ...).  kind: 0 forward, 1 back; the consumer
+  // position is the edge's place in its consumer's CSC (forward) or bin (back)
+  // list, where the consumer's partial is written.
+  {
+    std::vector<int32_t> csc_of(E), bin_of(NB);
+    for (int c = 0; c < E; ++c) csc_of[P.in_eslot[c]] = c;
+    for (int a = 0; a < NB; ++a) bin_of[P.bin_eslot[a]] = a;
+    P.ed.resize(4 * ((size_t)E + NB));
+    for (int i = 0; i < V; ++i)
+      for (int o = P.out_ptr[i]; o < P.out_ptr[i + 1]; ++o) {
+        P.ed[4 * (size_t)o + 0] = P.perm[i];
+        P.ed[4 * (size_t)o + 1] = P.out_dst[o];
+        P.ed[4 * (size_t)o + 2] = P.lat[i];
+        P.ed[4 * (size_t)o + 3] = csc_of[o] << 1;
+      }
+    for (int i = 0; i < V; ++i)
+      for (int q = P.bout_ptr[i]; q < P.bout_ptr[i + 1]; ++q) {
+        const size_t k = 4 * ((size_t)E + q);
+        P.ed[k + 0] = P.perm[i];
+        P.ed[k + 1] = P.bout_dst[q];
+        P.ed[k + 2] = P.bout_shift[q];
+        P.ed[k + 3] = 1 | (bin_of[q] << 1);
+      }
+  }
   // caller-order CSC / CSR / back edges for the integer kernels
   P.cpred_ptr.assign(p->pred_ptr, p->pred_ptr + V + 1);
   P.cpred_src.assign(p->pred_idx, p->pred_idx + E);
