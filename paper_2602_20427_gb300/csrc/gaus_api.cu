@@ -183,6 +183,10 @@ gaus_status set_smem_attrs(gaus_ctx *ctx) {
      "smem attr reg bwd");
   CK(cudaFuncSetAttribute((const void *)k_verify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_ver),
      "smem attr ver");
+  if (ctx->smem_leg)
+    CK(cudaFuncSetAttribute((const void *)k_legalize_regular_smem, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                            (int)ctx->smem_leg),
+       "smem attr legalize");
   return GAUS_OK;
 }
 
@@ -254,6 +258,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   ctx->smem_upd = (size_t)ctx->RB * P.Dh * sizeof(float);
   ctx->smem_fin = (size_t)(P.C + 1) * P.Dh * sizeof(double);
   ctx->smem_ver = ((size_t)P.C * P.Dh + (P.D + 1) + P.Dh) * sizeof(long long);
+  ctx->smem_leg = (size_t)P.V * sizeof(int) <= kMaxSmem - 1024 ? (size_t)P.V * sizeof(int) : 0;
   if (ctx->smem_upd > kMaxSmem || ctx->smem_fin > kMaxSmem || ctx->smem_ver > kMaxSmem) {
     ctx->err = "histogram of this horizon/II does not fit in shared memory";
     return GAUS_EINVAL;
@@ -287,6 +292,9 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(upload(ctx, &ctx->d_cls_seg_ptr, P.cls_seg_ptr));
   TRY(upload(ctx, &ctx->d_lvl_ptr, P.lvl_ptr));
   TRY(upload(ctx, &ctx->d_lvl_nodes, P.lvl_nodes));
+  TRY(upload(ctx, &ctx->d_lq_ptr, P.lq_ptr));
+  TRY(upload(ctx, &ctx->d_lq_src, P.lq_src));
+  TRY(upload(ctx, &ctx->d_lq_lat, P.lq_lat));
   TRY(upload(ctx, &ctx->d_cpred_ptr, P.cpred_ptr));
   TRY(upload(ctx, &ctx->d_cpred_src, P.cpred_src));
   TRY(upload(ctx, &ctx->d_csucc_ptr, P.csucc_ptr));
@@ -547,8 +555,10 @@ gaus_status gaus_legalize(gaus_ctx *ctx, const float *mu, int32_t *sched, int32_
   A.pred_ptr = ctx->d_cpred_ptr; A.pred_src = ctx->d_cpred_src; A.lat = ctx->d_c_lat;
   A.back_ptr = ctx->d_cback_ptr; A.back_src = ctx->d_cback_src; A.back_shift = ctx->d_cback_shift;
   A.asap = ctx->d_asap; A.alap = ctx->d_alap;
+  A.lq_ptr = ctx->d_lq_ptr; A.lq_src = ctx->d_lq_src; A.lq_lat = ctx->d_lq_lat;
   const int grid = (P.B + 31) / 32;
   if (P.II > 0) k_legalize_modulo<<<grid, 256, 0, ctx->stream>>>(A);
+  else if (ctx->smem_leg) k_legalize_regular_smem<<<P.B, 512, ctx->smem_leg, ctx->stream>>>(A);
   else k_legalize_regular<<<grid, 256, 0, ctx->stream>>>(A);
   CK(cudaGetLastError(), "legalize launch");
   return GAUS_OK;

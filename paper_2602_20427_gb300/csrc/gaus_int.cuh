@@ -19,6 +19,8 @@ struct LegArgs {
   const int32_t *pred_ptr, *pred_src, *lat;
   const int32_t *back_ptr, *back_src, *back_shift;
   const int32_t *asap, *alap;
+  // predecessors of the node at each level-order position q: producer, Lat(producer)
+  const int32_t *lq_ptr, *lq_src, *lq_lat;
 };
 
 // s = floor(mu + 1/2), evaluated exactly in double for every fp32 mu.
@@ -71,6 +73,39 @@ __global__ void __launch_bounds__(256) k_legalize_regular(const LegArgs A) {
     __syncthreads();
   }
   if (row == 0 && bok) A.status[b] = bad_lane[lane] ? GAUS_ENONFINITE : GAUS_OK;
+}
+
+// Alg. 1 with one restart per block and its whole schedule in shared memory
+// (4 |V| bytes): the same clamp and level-by-level forward pass, each level's
+// nodes in parallel, predecessors read from the level-ordered lists.  Same
+// fixed point, so the same result bit for bit.
+__global__ void __launch_bounds__(512) k_legalize_regular_smem(const LegArgs A) {
+  extern __shared__ int s_sched[];  // V, caller order
+  __shared__ int bad;
+  const int b = blockIdx.x, tid = threadIdx.x, nt = blockDim.x;
+  if (tid == 0) bad = 0;
+  __syncthreads();
+  for (int v = tid; v < A.V; v += nt) {
+    bool bd = false;
+    int x = round_half_up(A.mu[(size_t)v * A.B + b], bd);
+    if (bd) bad = 1;
+    x = max(x, A.asap[v]);
+    x = min(x, A.alap[v]);
+    s_sched[v] = x;
+  }
+  __syncthreads();
+  for (int l = 1; l < A.nlvl; ++l) {
+    const int q1 = A.lvl_ptr[l + 1];
+    for (int q = A.lvl_ptr[l] + tid; q < q1; q += nt) {
+      const int v = A.lvl_nodes[q], e1 = A.lq_ptr[q + 1];
+      int x = s_sched[v];
+      for (int e = A.lq_ptr[q]; e < e1; ++e) x = max(x, s_sched[A.lq_src[e]] + A.lq_lat[e]);
+      s_sched[v] = x;
+    }
+    __syncthreads();
+  }
+  for (int v = tid; v < A.V; v += nt) A.s[(size_t)v * A.B + b] = s_sched[v];
+  if (tid == 0) A.status[b] = bad ? GAUS_ENONFINITE : GAUS_OK;
 }
 
 // Alg. 2: sweeps in topological (level) order of

@@ -55,6 +55,7 @@ struct Plan {
   int nseg = 0;
   // caller-order data for the integer kernels
   std::vector<int32_t> lvl_ptr, lvl_nodes;           // nodes (caller ids) by level
+  std::vector<int32_t> lq_ptr, lq_src, lq_lat;       // predecessors by level-order position
   std::vector<int32_t> cpred_ptr, cpred_src;         // CSC by caller consumer id
   std::vector<int32_t> csucc_ptr, csucc_dst;         // CSR by caller producer id
   std::vector<int32_t> cback_ptr, cback_src, cback_shift;  // back edges by caller consumer
@@ -95,6 +96,8 @@ struct gaus_ctx {
   int32_t *d_bout_ptr = nullptr, *d_bout_dst = nullptr, *d_bout_shift = nullptr;
   int32_t *d_seg = nullptr, *d_cls_seg_ptr = nullptr;
   int32_t *d_lvl_ptr = nullptr, *d_lvl_nodes = nullptr;
+  int32_t *d_lq_ptr = nullptr, *d_lq_src = nullptr, *d_lq_lat = nullptr;
+  size_t smem_leg = 0;           // k_legalize_regular_smem (0: schedule does not fit)
   int32_t *d_cpred_ptr = nullptr, *d_cpred_src = nullptr;
   int32_t *d_csucc_ptr = nullptr, *d_csucc_dst = nullptr;
   int32_t *d_cback_ptr = nullptr, *d_cback_src = nullptr, *d_cback_shift = nullptr;

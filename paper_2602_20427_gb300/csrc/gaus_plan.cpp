@@ -278,6 +278,17 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
     std::vector<int32_t> f(P.lvl_ptr.begin(), P.lvl_ptr.end() - 1);
     for (int v = 0; v < V; ++v) P.lvl_nodes[f[P.level[v]]++] = v;
   }
+  P.lq_ptr.assign(V + 1, 0);
+  P.lq_src.clear();
+  P.lq_lat.clear();
+  for (int q = 0; q < V; ++q) {
+    const int v = P.lvl_nodes[q];
+    for (int e = p->pred_ptr[v]; e < p->pred_ptr[v + 1]; ++e) {
+      P.lq_src.push_back(p->pred_idx[e]);
+      P.lq_lat.push_back(p->latency[p->pred_idx[e]]);
+    }
+    P.lq_ptr[q + 1] = (int32_t)P.lq_src.size();
+  }
 
   // segments: contiguous internal nodes of one class, sized so that the per-node
   // kernels launch about target_blocks blocks over all restart groups
