@@ -16,6 +16,7 @@ constexpr int kFwdThreads = 256;
 constexpr int kThreads = 128;
 // Most own-window points cached in shared memory per thread (longer windows recompute).
 constexpr int kUpdThreads = 256;               // threads per k_update block
+constexpr int kReduceSpans = 1024;             // segment spans staged per k_reduce pass
 constexpr int kTableMax = 32;                    // points per CDF table row, at most
 constexpr size_t kTableBytes = (size_t)64 << 20;  // CDF table size bound
 // Fixed-point scale of the usage histograms: P * 2^32 accumulated in int64.

@@ -557,31 +557,30 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
 }
 
 // Usage per (restart, class, bin) from the partials of every block of the class:
-// block = (group g, class c, bin d); threads = restarts x slices of the segment
-// list (four independent loads in flight per thread); slices are combined in a
+// block = (group g, class c, bin d).  The class's segment spans are staged in
+// shared memory first, so that every thread then issues its partial loads
+// independently (restarts x slices of the segment list); slices are combined in a
 // fixed order (exact int64 sums, kept in 2^32 fixed point).
 __global__ void __launch_bounds__(256) k_reduce(const RedArgs A) {
   __shared__ long long part[256];
+  __shared__ int2 s_sp[kReduceSpans];
   const int RB = A.RB, Dh = A.Dh, nsl = 256 / RB;
   int x = blockIdx.x;
   const int d = x % Dh; x /= Dh;
   const int c = x % A.C, g = x / A.C;
   const int r = threadIdx.x % RB, sl = threadIdx.x / RB, b = g * RB + r;
-  const int s_end = A.cls_seg_ptr[c + 1];
+  const int s_beg = A.cls_seg_ptr[c], s_end = A.cls_seg_ptr[c + 1];
   long long acc = 0;
-  for (int s = A.cls_seg_ptr[c] + sl; s < s_end; s += 4 * nsl) {
-    long long v[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int ss = s + u * nsl;
-      v[u] = 0;
-      if (ss < s_end) {
-        const int blk = ss * A.G + g;
-        const int2 sp = A.hspan[blk];
-        if (d >= sp.x && d <= sp.y) v[u] = A.hpart[((size_t)blk * Dh + d) * RB + r];
-      }
+  for (int t0 = s_beg; t0 < s_end; t0 += kReduceSpans) {
+    const int t1 = min(s_end, t0 + kReduceSpans);
+    __syncthreads();
+    for (int s = t0 + threadIdx.x; s < t1; s += 256) s_sp[s - t0] = A.hspan[s * A.G + g];
+    __syncthreads();
+#pragma unroll 8
+    for (int s = t0 + sl; s < t1; s += nsl) {
+      const int2 sp = s_sp[s - t0];
+      if (d >= sp.x && d <= sp.y) acc += __ldcg(A.hpart + ((size_t)(s * A.G + g) * Dh + d) * RB + r);
     }
-    acc += v[0] + v[1] + v[2] + v[3];
   }
   part[threadIdx.x] = acc;
   __syncthreads();
@@ -818,10 +817,12 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
     // the node's edge partials in a fixed order: out-edges, in-edges, back edges
     float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f;
     if (ok) {
+#pragma unroll 8
       for (int e = A.out_ptr[vi]; e < A.out_ptr[vi + 1]; ++e) {
         const float4 s = A.eslot4[(size_t)e * A.B + b];
         Ad += s.x; Bd += s.y; Ao += s.z; Bo += s.w;
       }
+#pragma unroll 4
       for (int e = A.in_ptr[vi]; e < A.in_ptr[vi + 1]; ++e) {
         const float4 s = A.eslot4[nP + (size_t)e * A.B + b];
         Ad += s.x; Bd += s.y; Ao += s.z; Bo += s.w;
