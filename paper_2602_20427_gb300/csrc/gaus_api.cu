@@ -70,6 +70,7 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   A.bout_ptr = ctx->d_bout_ptr; A.bout_dst = ctx->d_bout_dst; A.bout_shift = ctx->d_bout_shift;
   A.seg = ctx->d_seg; A.hpart = ctx->d_hpart; A.hspan = ctx->d_hspan; A.fwd = ctx->d_fwd;
   A.nonfinite = ctx->d_nonfinite; A.win = ctx->d_win; A.tab = ctx->d_tab;
+  A.wstat = ctx->d_wstat;
   A.ed = ctx->d_ed; A.nEt = P.E + P.NB; A.ce = ctx->ce; A.E = P.E; A.eslot4 = ctx->d_eslot4;
   return A;
 }
@@ -135,6 +136,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   F.lambda = lambda; F.update_lambda = adam ? 1 : 0; F.step = adam ? S->step : nullptr;
   F.beta1 = ctx->hp.beta1; F.beta2 = ctx->hp.beta2;
   F.H = ctx->d_H; F.coef = ctx->d_coef; F.loss = loss; F.terms_out = terms;
+  F.wstat = ctx->d_wstat; F.thr = ctx->d_thr; F.W = ctx->W;
   F.status = status; F.nonfinite = ctx->d_nonfinite;
   k_finalize<<<P.B, 256, ctx->smem_fin, st>>>(F);
   CK(cudaGetLastError(), "k_finalize launch");
@@ -152,7 +154,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   U.mu = const_cast<float *>(mu); U.sg = const_cast<float *>(sg);
   U.V = P.V; U.B = P.B; U.D = P.D; U.II = P.II; U.Dh = P.Dh; U.C = P.C; U.RB = ctx->RB; U.G = ctx->G;
   U.k_win = ctx->hp.window_k; U.W = ctx->W; U.perm = ctx->d_perm; U.cls = ctx->d_cls; U.w = ctx->d_w;
-  U.H = ctx->d_H; U.coef = ctx->d_coef;
+  U.H = ctx->d_H; U.coef = ctx->d_coef; U.thr = ctx->d_thr;
   U.grad_mu = grad_mu; U.grad_sg = grad_sg;
   U.m_mu = adam ? S->m_mu : nullptr; U.v_mu = adam ? S->v_mu : nullptr;
   U.m_sg = adam ? S->m_sigma : nullptr; U.v_sg = adam ? S->v_sigma : nullptr;
@@ -325,6 +327,8 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_tab, VB * ctx->W));
   TRY(scratch(ctx, &ctx->d_H, (size_t)P.B * P.C * P.Dh));
   TRY(scratch(ctx, &ctx->d_coef, (size_t)P.B * 4));
+  TRY(scratch(ctx, &ctx->d_wstat, (size_t)P.B * 2));
+  TRY(scratch(ctx, &ctx->d_thr, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_nonfinite, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_status_tmp, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_loss_tmp, (size_t)P.B));

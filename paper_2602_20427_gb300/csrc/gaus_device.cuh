@@ -31,6 +31,26 @@ __device__ __forceinline__ float cdf_fast(float z) {
   return z <= 0.f ? q : 1.0f - q;
 }
 
+// Upper tail Q(|z|) = Phi(-|z|) from the same Mills-ratio fit: relative error
+// ~1e-6 on |z| <= 12 (the fit) plus the fast exponential's, so both tails of the
+// bin masses keep their relative accuracy.
+__device__ __forceinline__ float tail_fast(float z) {
+  const float x = fabsf(z);
+  const float e = __expf(-0.5f * z * z);
+  const float num = (((kMillsP[4] * x + kMillsP[3]) * x + kMillsP[2]) * x + kMillsP[1]) * x + kMillsP[0];
+  const float den = ((((kMillsQ[5] * x + kMillsQ[4]) * x + kMillsQ[3]) * x + kMillsQ[2]) * x + kMillsQ[1]) * x + 1.0f;
+  return e * __fdividef(num, den);
+}
+
+// One Adam step of a parameter (torch.optim.Adam semantics): m, v updated in
+// place; inv_bc1 = 1 / (1 - beta1^t), rs_bc2 = 1 / sqrt(1 - beta2^t).
+__device__ __forceinline__ float adam_update(float th, float g, float &m, float &v, float lr, float beta1,
+                                             float beta2, float eps, float inv_bc1, float rs_bc2) {
+  m = beta1 * m + (1.0f - beta1) * g;
+  v = beta2 * v + (1.0f - beta2) * g * g;
+  return th - __fdividef(lr * m * inv_bc1, sqrtf(v) * rs_bc2 + eps);
+}
+
 // Windowed CDF of a neighbour at integer point x.
 __device__ __forceinline__ float cdf_at(int x, float mu, float inv_s, int a, int b) {
   if (x < a) return 0.0f;

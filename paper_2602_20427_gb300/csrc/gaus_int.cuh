@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "gaus_device.cuh"
 #include "gaus_internal.h"
 
 namespace gaus {
@@ -277,16 +278,15 @@ __global__ void __launch_bounds__(256) k_verify(const VerArgs A) {
 __global__ void k_adam(float *mu, float *sg, const float *gmu, const float *gsg, float *m1, float *v1,
                        float *m2, float *v2, size_t n, int step, float lr, float beta1, float beta2,
                        float eps, float sigma_min) {
-  const float bc1 = 1.0f - powf(beta1, (float)step), bc2 = 1.0f - powf(beta2, (float)step);
+  const float inv_bc1 = 1.0f / (1.0f - powf(beta1, (float)step));
+  const float rs_bc2 = 1.0f / sqrtf(1.0f - powf(beta2, (float)step));
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
-    const float g1 = gmu[i], g2 = gsg[i];
-    const float a1 = beta1 * m1[i] + (1.0f - beta1) * g1;
-    const float b1 = beta2 * v1[i] + (1.0f - beta2) * g1 * g1;
-    const float a2 = beta1 * m2[i] + (1.0f - beta1) * g2;
-    const float b2 = beta2 * v2[i] + (1.0f - beta2) * g2 * g2;
+    float a1 = m1[i], b1 = v1[i], a2 = m2[i], b2 = v2[i];
+    const float nmu = adam_update(mu[i], gmu[i], a1, b1, lr, beta1, beta2, eps, inv_bc1, rs_bc2);
+    const float nsg = adam_update(sg[i], gsg[i], a2, b2, lr, beta1, beta2, eps, inv_bc1, rs_bc2);
     m1[i] = a1; v1[i] = b1; m2[i] = a2; v2[i] = b2;
-    mu[i] = mu[i] - lr * (a1 / bc1) / (sqrtf(b1 / bc2) + eps);
-    sg[i] = fmaxf(sg[i] - lr * (a2 / bc1) / (sqrtf(b2 / bc2) + eps), sigma_min);
+    mu[i] = nmu;
+    sg[i] = fmaxf(nsg, sigma_min);
   }
 }
 

@@ -122,7 +122,9 @@ struct gaus_ctx {
   unsigned *d_win = nullptr;     // V * B packed windows (caller order)
   float *d_tab = nullptr;        // V * B * W CDF values at the window points (caller order)
   float *d_H = nullptr;          // B * C * Dh usage adjoint dL/dU
-  float *d_coef = nullptr;       // B * 4 (c_dep, c_rec)
+  float *d_coef = nullptr;       // B * 4 (c_dep, c_rec, Adam bias corrections)
+  unsigned long long *d_wstat = nullptr;  // B * 2 window statistics of the iteration
+  int32_t *d_thr = nullptr;      // B long-window thresholds
   int32_t *d_nonfinite = nullptr;  // B flags
   int32_t *d_status_tmp = nullptr; // B
   float *d_loss_tmp = nullptr, *d_terms_tmp = nullptr;

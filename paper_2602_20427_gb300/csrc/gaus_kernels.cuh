@@ -51,6 +51,7 @@ struct IterArgs {
   float *tab;     // (V, B, W) CDF values at the window points, written by k_nodes
   const int4 *ed; // edge list of the edge pass (nEt = E + NB edges, ce per block)
   int nEt, ce, E;
+  unsigned long long *wstat;  // (B, 2) window points / valid items of this iteration
   float4 *eslot4; // per-edge partials [side][position][restart]: producer side at
                   // the edge's index (CSR / bout order), consumer side at its
                   // CSC / bin position (+E for back edges), offset nEt * B
@@ -80,9 +81,12 @@ struct FinArgs {
   float *lambda;      // read; updated in place when update_lambda
   int update_lambda;
   int32_t *step;      // incremented when not NULL
-  float beta1, beta2; // Adam, for the bias corrections written to coef[2], coef[3]
+  float beta1, beta2; // Adam: 1 / (1 - beta1^t), 1 / sqrt(1 - beta2^t) written to coef[2], coef[3]
   float *H, *coef, *loss, *terms_out;
   int32_t *status, *nonfinite;
+  unsigned long long *wstat;  // read into thr and cleared for the next iteration
+  int32_t *thr;
+  int W;
 };
 
 struct UpdArgs {
@@ -95,6 +99,7 @@ struct UpdArgs {
   const float4 *eslot4;
   const float2 *eslot;               // storage term: successor shares (NULL when off)
   const float2 *gown;                // storage term: own-window adjoint (NULL when off)
+  const int32_t *thr;                // per-restart long-window threshold (k_finalize)
   float *mu, *sg;  // caller order; written when adam
   int V, B, D, II, Dh, C, RB, G;
   float k_win;
@@ -113,6 +118,17 @@ __device__ __forceinline__ long long to_fix(float x) {
   const float xs = fmaxf(x, 0.0f) * 65536.0f;
   const float fh = floorf(xs);
   return ((long long)(unsigned)fh << 16) + (long long)__float2uint_rn((xs - fh) * 65536.0f);
+}
+
+// Window length above which an item of restart b is done by the whole warp:
+// twice the restart's mean window (over all its nodes, this iteration) plus 4,
+// at least 8 and at most the table row.  It depends on restart b alone, so the
+// split -- and with it every rounding -- does not depend on the other restarts.
+__device__ __forceinline__ int long_threshold(const unsigned long long *ws, int b, int W) {
+  const unsigned long long c = ws[2 * b + 1];
+  if (c == 0) return W;
+  const int mean = (int)(ws[2 * b] / c);
+  return min(W, max(8, 2 * mean + 4));
 }
 
 // Mean window length (points) of restart b over the nodes s0..s1 of a segment,
@@ -172,12 +188,13 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
   const int tid = threadIdx.x, lane = tid & 31, RB = A.RB, Dh = A.Dh, W = A.W;
   unsigned *hlo = reinterpret_cast<unsigned *>(smem);  // [bin][restart]
   unsigned *hhi = hlo + (size_t)Dh * RB;
-  __shared__ int s_lo, s_hi, s_next;
+  __shared__ int s_lo, s_hi, s_next, s_ws[32], s_wc[32];
 
   const int blk = blockIdx.x, segi = blk / A.G, g = blk % A.G;
   const int s0 = A.seg[3 * segi], s1 = A.seg[3 * segi + 1];
   for (int i = tid; i < 2 * RB * Dh; i += T) hlo[i] = 0u;
   if (tid == 0) { s_lo = INT_MAX; s_hi = INT_MIN; s_next = 0; }
+  if (tid < 32) { s_ws[tid] = 0; s_wc[tid] = 0; }
   __syncthreads();
 
   const int r = tid % RB, b = g * RB + r;
@@ -202,6 +219,10 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
     if (valid) window(mu, sg, A.k_win, A.D, a, bw);
     if (present) A.win[ci] = (unsigned)a | ((unsigned)(bw + 1) << 16);
     const int n = valid ? bw - a + 1 : -1;  // points; -1: nothing to add
+    if (valid) {
+      atomicAdd(&s_ws[r], min(n, 4096));
+      atomicAdd(&s_wc[r], 1);
+    }
     // windows much longer than the warp's typical one go to the cooperative pass
     // (the results do not depend on the split: the table values are per point
     // and the histogram sums are exact)
@@ -215,7 +236,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
     for (int j = 0; j <= nmax; ++j) {
       const bool pt = j < nl;  // point a+j exists
       const float zc = ((float)(a + j) + 0.5f - mu) * inv_s;
-      const float qc = pt ? 0.5f * erfcf(fabsf(zc) * kInvSqrt2) : 0.f;
+      const float qc = pt ? tail_fast(zc) : 0.f;
       if (pt && j < W) row[j] = zc <= 0.f ? qc : 1.0f - qc;
       if (j <= nl) hist_add(hlo, hhi, fold_bin(a + j, A.II) * RB + r, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
       zp = zc;
@@ -237,7 +258,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
         const int p = p0 + lane;
         const bool pt = p < l_n;
         const float z = ((float)(l_a + p) + 0.5f - l_mu) * l_inv;
-        const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
+        const float q = pt ? tail_fast(z) : 0.f;
         if (pt && p < W) l_row[p] = z <= 0.f ? q : 1.0f - q;
         float zpv = __shfl_up_sync(FULL, z, 1), qpv = __shfl_up_sync(FULL, q, 1);
         if (lane == 0) { zpv = z_carry; qpv = q_carry; }
@@ -258,6 +279,11 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
     atomicMax(&s_hi, hi);
   }
   __syncthreads();
+  // per-restart window statistics (exact integer sums, any order)
+  if (tid < RB && bok && s_wc[tid]) {
+    atomicAdd(&A.wstat[2 * b], (unsigned long long)s_ws[tid]);
+    atomicAdd(&A.wstat[2 * b + 1], (unsigned long long)s_wc[tid]);
+  }
   int flo = s_lo, fhi = s_hi;
   if (flo > fhi) {
     flo = 1;
@@ -300,9 +326,9 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
     const bool pt = pidx < nv;
     const int t = Vn.a + pidx;
     const float z = ((float)t + 0.5f - Vn.mu) * Vn.inv;
-    const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
+    const float q = pt ? tail_fast(z) : 0.f;
     const float Cv = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
-    const float f = pt ? kInvSqrt2Pi * expf(-0.5f * z * z) : 0.f;
+    const float f = pt ? kInvSqrt2Pi * __expf(-0.5f * z * z) : 0.f;
     const float zf = z * f;
     if (!back) {
       if (pt) {
@@ -332,9 +358,9 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
     const bool pt = pidx < nu;
     const int x = U.a + pidx;
     const float z = ((float)x + 0.5f - U.mu) * U.inv;
-    const float q = pt ? 0.5f * erfcf(fabsf(z) * kInvSqrt2) : 0.f;
+    const float q = pt ? tail_fast(z) : 0.f;
     const float Cu = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
-    const float f = pt ? kInvSqrt2Pi * expf(-0.5f * z * z) : 0.f;
+    const float f = pt ? kInvSqrt2Pi * __expf(-0.5f * z * z) : 0.f;
     const float zf = z * f;
     if (!back) {
       if (pt) {
@@ -369,8 +395,8 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
 // (dV/dmu-, dV/dsigma-type sums: Ad, Bd, Ao, Bo for a forward edge, Ar, Br for a
 // back edge) to the edge's two slots, which k_update gathers per node in a fixed
 // order, and adds the edge's forward sums (exact fixed point) to the block's.
-// An edge with an endpoint window longer than the table row is done by the
-// whole warp (coop_edge); the choice depends on that restart's windows only.
+// An edge with an endpoint window longer than the restart's threshold (at most
+// the table row) is done by the whole warp (coop_edge).
 template <bool kDep, bool kCom, bool kRec>
 __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   constexpr int T = kFwdThreads;
@@ -381,6 +407,7 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   const int e_begin = ch * A.ce, e_end = min(A.nEt, e_begin + A.ce);
   const int r = tid % RB, b = g * RB + r;
   const bool bok = b < A.B;
+  const int thr = bok ? long_threshold(A.wstat, b, A.W) : A.W;
   long long xdep = 0, xcom = 0, xrec = 0;  // forward sums, exact (order-free) fixed point
   const int per_pass = (T / 32) * epw;
   for (int e0 = e_begin + warp * epw; e0 < e_end; e0 += per_pass) {
@@ -403,7 +430,7 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
     const int nu = U.b - U.a + 1, nv = Vn.b - Vn.a + 1;
     U.tab = nu <= A.W;
     Vn.tab = nv <= A.W;
-    const bool is_long = on && !(U.tab && Vn.tab);
+    const bool is_long = on && (nu > thr || nv > thr);
     const bool ps = on && !is_long;                 // per-lane path
     const bool fw = ps && !back && (kDep || kCom);  // forward edge terms
     const bool bk = kRec && ps && back;             // back edge term
@@ -711,6 +738,9 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
     A.loss[b] = (float)L;
     A.coef[b * 4 + 0] = on_dep ? (float)((double)lam[GAUS_K_DEP] + (double)A.rho * Vk[0]) : 0.f;
     A.coef[b * 4 + 1] = on_rec ? (float)((double)lam[GAUS_K_REC] + (double)A.rho * Vk[2]) : 0.f;
+    A.thr[b] = long_threshold(A.wstat, b, A.W);
+    A.wstat[2 * b] = 0ull;
+    A.wstat[2 * b + 1] = 0ull;
     const int bad = A.nonfinite[b];
     if (A.status) A.status[b] = bad ? GAUS_ENONFINITE : GAUS_OK;
     A.nonfinite[b] = 0;
@@ -722,9 +752,10 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
     if (A.step) {
       const int st = A.step[b] + 1;
       A.step[b] = st;
-      // Adam bias corrections of this step (torch.optim.Adam)
-      A.coef[b * 4 + 2] = 1.0f - powf(A.beta1, (float)st);
-      A.coef[b * 4 + 3] = 1.0f - powf(A.beta2, (float)st);
+      // Adam bias corrections of this step (torch.optim.Adam): 1 / (1 - beta1^t)
+      // and 1 / sqrt(1 - beta2^t)
+      A.coef[b * 4 + 2] = 1.0f / (1.0f - powf(A.beta1, (float)st));
+      A.coef[b * 4 + 3] = 1.0f / sqrtf(1.0f - powf(A.beta2, (float)st));
     }
   }
   // usage adjoint dL/dU_c(t) = w_res softmax_c(t) + c_res [U_c(t) > R_c], [class][bin][restart]
@@ -748,7 +779,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
 // back edges out and in, all contiguous per node); the combined gradient
 //   dL/dmu = -(c_dep Ad + Ao + c_rec Ar + Ah) / sigma, same with B.. for sigma,
 // and, in Adam mode, the Adam step with the per-restart bias corrections.
-// Windows longer than the table row are done by the whole warp.
+// Windows longer than the restart's threshold are done by the whole warp.
 template <bool kAdam, bool kHist>
 __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
   constexpr unsigned FULL = 0xffffffffu;
@@ -772,14 +803,14 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
       int a = 0, bw = -1;
       if (ok) window(mu, sg, A.k_win, A.D, a, bw);
       const int nfull = bw - a + 1;
-      const bool is_long = ok && nfull > A.W;
+      const bool is_long = ok && nfull > A.thr[bs];
       const int n = is_long ? 0 : nfull;
       const int nmax = __reduce_max_sync(FULL, n);
       for (int j = 0; j < nmax; ++j) {
         if (j < n) {
           const int t = a + j;
           const float z = ((float)t + 0.5f - mu) * inv_s;
-          const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
+          const float f = kInvSqrt2Pi * __expf(-0.5f * z * z);
           const float gh = wv * (Hc[(size_t)fold_bin(t, A.II) * A.B + b] - Hc[(size_t)fold_bin(t + 1, A.II) * A.B + b]);
           Ah += gh * f;
           Bh += gh * z * f;
@@ -801,7 +832,7 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
           if (j < l_n) {
             const int t = l_a + j;
             const float z = ((float)t + 0.5f - l_mu) * l_inv;
-            const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
+            const float f = kInvSqrt2Pi * __expf(-0.5f * z * z);
             const float gh = l_w * (l_H[(size_t)fold_bin(t, A.II) * A.B + l_b] -
                                     l_H[(size_t)fold_bin(t + 1, A.II) * A.B + l_b]);
             pa += gh * f;
@@ -852,19 +883,17 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
         Bsum += sh.y;
       }
     // dC/dmu = -phi/sigma, dC/dsigma = -z phi/sigma
-    const float gm = ok ? -Asum / sg : 0.f, gs = ok ? -Bsum / sg : 0.f;
+    const float rs = ok ? __frcp_rn(sg) : 0.f;
+    const float gm = -Asum * rs, gs = -Bsum * rs;
     if (!kAdam) {
       A.grad_mu[ci] = gm;
       A.grad_sg[ci] = gs;
     } else {
-      const float bc1 = A.coef[b * 4 + 2], bc2 = A.coef[b * 4 + 3];
-      const float m1 = A.beta1 * A.m_mu[ci] + (1.0f - A.beta1) * gm;
-      const float v1 = A.beta2 * A.v_mu[ci] + (1.0f - A.beta2) * gm * gm;
-      const float m2 = A.beta1 * A.m_sg[ci] + (1.0f - A.beta1) * gs;
-      const float v2 = A.beta2 * A.v_sg[ci] + (1.0f - A.beta2) * gs * gs;
+      const float inv_bc1 = A.coef[b * 4 + 2], rs_bc2 = A.coef[b * 4 + 3];
+      float m1 = A.m_mu[ci], v1 = A.v_mu[ci], m2 = A.m_sg[ci], v2 = A.v_sg[ci];
+      const float nmu = adam_update(mu, gm, m1, v1, A.lr, A.beta1, A.beta2, A.eps, inv_bc1, rs_bc2);
+      const float nsg = adam_update(sg, gs, m2, v2, A.lr, A.beta1, A.beta2, A.eps, inv_bc1, rs_bc2);
       A.m_mu[ci] = m1; A.v_mu[ci] = v1; A.m_sg[ci] = m2; A.v_sg[ci] = v2;
-      const float nmu = mu - A.lr * (m1 / bc1) / (sqrtf(v1 / bc2) + A.eps);
-      const float nsg = sg - A.lr * (m2 / bc1) / (sqrtf(v2 / bc2) + A.eps);
       A.mu[ci] = nmu;
       A.sg[ci] = fmaxf(nsg, A.sigma_min);
     }
