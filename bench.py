@@ -46,6 +46,9 @@ def parse():
     ap.add_argument("--iters", type=int, default=2000, help="fused iterations per solve (one step)")
     ap.add_argument("--period", type=int, default=100, help="iterations between legalize + verify")
     ap.add_argument("--impl", default="gaus", choices=["gaus", "reference"])
+    ap.add_argument("--phase-probe", type=int, default=None, metavar="N",
+                    help="run N iterations kernel by kernel, then one more, print the phase times and exit "
+                         "(a fixed launch sequence for ncu captures at iteration N)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -131,10 +134,10 @@ def algorithmic_flops(torch, mu, sg, src, dst, k, D):
 
 
 def profiled_traffic():
-    """DRAM bytes per k_fwd launch from the committed ncu summary, or None when the
+    """DRAM bytes per k_edges launch from the committed ncu summary, or None when the
     kernel sources changed since that capture."""
     import hashlib
-    prof = os.path.join(ROOT, "profiles", "k_fwd_logic_network_v10000_b64.md")
+    prof = os.path.join(ROOT, "profiles", "k_edges_logic_network_v10000_b64.md")
     if not os.path.exists(prof):
         return None
     txt = open(prof).read()
@@ -252,21 +255,22 @@ def gpu_arm(args):
     src = torch.from_numpy(np.asarray(p.src, np.int64)).cuda()
     dst = torch.from_numpy(np.asarray(p.dst, np.int64)).cuda()
     ph_ms = np.zeros(4)
-    flops_total, t_fwd_total, npt_total, neb_total = 0.0, 0.0, 0.0, 0.0
+    t_edges_total, t_nodes_total, npt_total, neb_total = 0.0, 0.0, 0.0, 0.0
     fwd_first = fwd_last = None
     nchunk = iters // period
     for k in range(nchunk):
-        f0, n0, e0 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
+        _, n0, e0 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
         kms = np.array(ctx.profile_iterate(period, st))
-        f1, n1, e1 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
+        _, n1, e1 = algorithmic_flops(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D)
         ph_ms += kms / nchunk
-        flops_total += period * 0.5 * (f0 + f1)
         npt_total += period * 0.5 * (n0 + n1)
         neb_total += period * 0.5 * (e0 + e1)
-        t_fwd_total += period * kms[1] * 1e-3
+        t_nodes_total += period * kms[0] * 1e-3
+        t_edges_total += period * kms[1] * 1e-3
         fwd_first = kms[1] if fwd_first is None else fwd_first
         fwd_last = kms[1]
-    achieved = flops_total / t_fwd_total / 1e12
+    achieved = 8.0 * neb_total / t_edges_total / 1e12           # edge pass: 8 flop per edge-bin
+    nodes_achieved = 20.0 * npt_total / t_nodes_total / 1e12    # node pass: 20 flop per CDF point
     peak = SM_COUNT * FP32_LANES_PER_SM * 2 * SM_MAX_MHZ * 1e6 / 1e12
     traffic = profiled_traffic()
 
@@ -287,7 +291,7 @@ def gpu_arm(args):
     fixed_ph = ctx0.profile_iterate(20, st0)
     ctx0.close()
     steady = {"value": B / (fixed_ms / 1e3), "unit": UNIT, "sigma": 1.5, "ms_per_iteration": fixed_ms,
-              "k_fwd_ms": fixed_ph[1],
+              "k_edges_ms": fixed_ph[1],
               "note": "initial state of the same workload with lr = 1e-20, so every iteration has the "
                       "initial +-6 sigma windows (the most expensive point of the run)"}
 
@@ -338,15 +342,18 @@ def gpu_arm(args):
                                parallelism=f"restarts sharded, {world} replica(s)"),
                 "e2e": e2e, "gpu_launches": args.steps * launches_per_step,
                 "clocks": clocks,
-                "roofline": {"bound": "alu", "kernel": "k_fwd (node + edge pass)", "achieved": achieved,
+                "roofline": {"bound": "alu", "kernel": "k_edges (edge pass)", "achieved": achieved,
                              "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
                              "peak_note": "FP32: 152 SM x 128 lanes x 2 flop x 2070 MHz (max SM clock)",
-                             "cost_model": "20 flop per CDF point + 8 flop per edge-bin",
-                             "points_per_iter": npt_total / iters,
-                             "edge_bins_per_iter": neb_total / iters},
-                "phase_ms_per_iteration": {"k_windows": ph_ms[0], "k_fwd": ph_ms[1],
+                             "cost_model": "8 flop per edge-bin (edge pass)",
+                             "edge_bins_per_iter": neb_total / iters,
+                             "node_pass": {"kernel": "k_nodes", "achieved": nodes_achieved,
+                                           "frac": nodes_achieved / peak,
+                                           "cost_model": "20 flop per CDF point",
+                                           "points_per_iter": npt_total / iters}},
+                "phase_ms_per_iteration": {"k_nodes": ph_ms[0], "k_edges": ph_ms[1],
                                            "reduce_finalize": ph_ms[2], "k_update": ph_ms[3],
-                                           "k_fwd_first_period": fwd_first, "k_fwd_last_period": fwd_last},
+                                           "k_edges_first_period": fwd_first, "k_edges_last_period": fwd_last},
                 "legalize_verify_ms": legalize_verify_ms,
                 "steady_fixed_sigma": steady,
                 "step_ms": step_ms,
@@ -355,6 +362,26 @@ def gpu_arm(args):
         print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
+
+
+def phase_probe(args):
+    """Iterations 0..N-1 and then iteration N of the benchmark workload, launched
+    kernel by kernel (k_nodes, k_edges, k_reduce, k_finalize, k_update each once per
+    iteration), so that `ncu -k regex:k_edges -s N -c 1` captures iteration N."""
+    import torch
+
+    import paper_2602_20427_gb300 as g
+    g.build()
+    p, B, mu0, sg0 = workload(0)
+    ctx = g.Gaus(p, B, g.default_hparams(terms=p.terms))
+    st = ctx.new_state(torch.from_numpy(mu0).cuda(), torch.from_numpy(sg0).cuda())
+    if args.phase_probe > 0:
+        ctx.profile_iterate(args.phase_probe, st)
+    ms = ctx.profile_iterate(1, st)
+    torch.cuda.synchronize()
+    print(json.dumps({"iteration": args.phase_probe, "phase_ms": {"k_nodes": ms[0], "k_edges": ms[1],
+                                                                  "reduce_finalize": ms[2], "k_update": ms[3]}}))
+    ctx.close()
 
 
 def _oracle_iteration(op, ohp, mu, sg, lam, mom, step, lr):
@@ -433,7 +460,9 @@ def reference_arm(args):
 
 if __name__ == "__main__":
     a = parse()
-    if a.impl == "reference":
+    if a.phase_probe is not None:
+        phase_probe(a)
+    elif a.impl == "reference":
         reference_arm(a)
     else:
         gpu_arm(a)
