@@ -77,16 +77,22 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
 
 using EdgeKernel = void (*)(const IterArgs);
 
-EdgeKernel pick_edges(unsigned terms, int II) {
+EdgeKernel pick_edges(unsigned terms, int II, bool unit) {
   const bool dep = terms & GAUS_DEP, com = terms & GAUS_COM, rec = (terms & GAUS_REC) && II > 0;
-  if (dep && com && rec) return k_edges<true, true, true>;
-  if (dep && com) return k_edges<true, true, false>;
-  if (dep && rec) return k_edges<true, false, true>;
-  if (dep) return k_edges<true, false, false>;
-  if (com && rec) return k_edges<false, true, true>;
-  if (com) return k_edges<false, true, false>;
-  if (rec) return k_edges<false, false, true>;
-  return k_edges<false, false, false>;
+  if (dep && com && rec) return k_edges<true, true, true, false>;
+  if (dep && rec) return k_edges<true, false, true, false>;
+  if (com && rec) return k_edges<false, true, true, false>;
+  if (rec) return k_edges<false, false, true, false>;
+  if (unit) {
+    if (dep && com) return k_edges<true, true, false, true>;
+    if (dep) return k_edges<true, false, false, true>;
+    if (com) return k_edges<false, true, false, true>;
+    return k_edges<false, false, false, true>;
+  }
+  if (dep && com) return k_edges<true, true, false, false>;
+  if (dep) return k_edges<true, false, false, false>;
+  if (com) return k_edges<false, true, false, false>;
+  return k_edges<false, false, false, false>;
 }
 
 // Enqueue loss + gradient (adam == false: gradient written to grad_*), or the
@@ -102,7 +108,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   k_nodes<<<ctx->nblk, kFwdThreads, ctx->smem_nodes, st>>>(A);
   CK(cudaGetLastError(), "k_nodes launch");
   if (ev) CK(cudaEventRecord(ev[1], st), "event");
-  EdgeKernel ke = pick_edges(on, P.II);
+  EdgeKernel ke = pick_edges(on, P.II, P.unit_lat != 0);
   ke<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
   CK(cudaGetLastError(), "k_edges launch");
   if (ev) CK(cudaEventRecord(ev[2], st), "event");

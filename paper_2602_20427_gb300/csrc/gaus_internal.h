@@ -66,6 +66,7 @@ struct Plan {
   std::vector<float> limit;
   int nlvl = 0;
   int has_reg_succ_any = 0;
+  int unit_lat = 0;  // every producer of an edge has latency 1
 };
 
 // Returns GAUS_OK or an error with a message.

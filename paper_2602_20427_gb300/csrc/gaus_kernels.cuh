@@ -122,13 +122,13 @@ __device__ __forceinline__ long long to_fix(float x) {
 
 // Window length above which an item of restart b is done by the whole warp:
 // twice the restart's mean window (over all its nodes, this iteration) plus 4,
-// at least 8 and at most the table row.  It depends on restart b alone, so the
+// at least 8.  It depends on restart b alone, so the
 // split -- and with it every rounding -- does not depend on the other restarts.
-__device__ __forceinline__ int long_threshold(const unsigned long long *ws, int b, int W) {
+__device__ __forceinline__ int long_threshold(const unsigned long long *ws, int b) {
   const unsigned long long c = ws[2 * b + 1];
-  if (c == 0) return W;
+  if (c == 0) return 8;
   const int mean = (int)(ws[2 * b] / c);
-  return min(W, max(8, 2 * mean + 4));
+  return min(1 << 20, max(8, 2 * mean + 4));
 }
 
 // Mean window length (points) of restart b over the nodes s0..s1 of a segment,
@@ -160,17 +160,30 @@ __device__ __forceinline__ float warp_sum(float x) {
 }
 
 // A neighbour's windowed CDF C_u(x): 0 below its window, 1 above it, inside it
-// the table value written by k_nodes, or -- for a window longer than the table
-// row -- evaluated from its mean and sigma (loaded only then).
+// the table value written by k_nodes, or -- for a window the table row cannot
+// hold -- evaluated from its mean and sigma.
 struct Nb {
-  const float *row;  // table row of (u, b)
+  const float *row;  // table row of (u, b): [0, C(a), ..., C(b), 1, ...]
   int a, b;          // window points [a, b]
-  bool tab;          // the row holds every point of the window
+  bool tab;          // the row holds the window with both sentinels (b - a + 3 <= W)
   float mu, inv;
+  // any window: 0 below, 1 above, the table or a direct evaluation inside
   __device__ __forceinline__ float at(int x) const {
     if (x < a) return 0.0f;
     if (x > b) return 1.0f;
-    return tab ? __ldg(row + (x - a)) : cdf_fast(((float)x + 0.5f - mu) * inv);
+    return tab ? __ldg(row + (x - a + 1)) : cdf_fast(((float)x + 0.5f - mu) * inv);
+  }
+  // a tabled window: the sentinels make the clamped index exact everywhere
+  __device__ __forceinline__ float at_tab(int x) const {
+    return __ldg(row + min(max(x - a + 1, 0), b - a + 2));
+  }
+  // a window the table row cannot hold: direct evaluation
+  __device__ __forceinline__ float at_direct(int x) const {
+    return x < a ? 0.0f : (x > b ? 1.0f : cdf_fast(((float)x + 0.5f - mu) * inv));
+  }
+  template <bool kTab>
+  __device__ __forceinline__ float val(int x) const {
+    return kTab ? at_tab(x) : at_direct(x);
   }
 };
 
@@ -231,13 +244,16 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
     const bool is_long = valid && n > max(8, 2 * mean + 8);
     const int nl = is_long ? -1 : n;
     const int nmax = __reduce_max_sync(FULL, nl);
+    // table row [0, C(a), ..., C(b), 1] when the window fits it
     float *row = A.tab + ci * W;
+    const bool tabled = n >= 0 && n + 3 <= W;
+    if (tabled && !is_long) row[0] = 0.0f;
     float zp = 0.f, qp = 0.f;
     for (int j = 0; j <= nmax; ++j) {
       const bool pt = j < nl;  // point a+j exists
       const float zc = ((float)(a + j) + 0.5f - mu) * inv_s;
       const float qc = pt ? tail_fast(zc) : 0.f;
-      if (pt && j < W) row[j] = zc <= 0.f ? qc : 1.0f - qc;
+      if (tabled && j <= nl) row[j + 1] = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;
       if (j <= nl) hist_add(hlo, hhi, fold_bin(a + j, A.II) * RB + r, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
       zp = zc;
       qp = qc;
@@ -253,13 +269,15 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
       const float l_mu = __shfl_sync(FULL, mu, src), l_inv = __shfl_sync(FULL, inv_s, src);
       const float l_w = __shfl_sync(FULL, wv, src);
       float *l_row = A.tab + ((size_t)l_vc * A.B + l_b) * W;
+      const bool l_tabled = l_n + 3 <= W;
+      if (l_tabled && lane == 0) l_row[0] = 0.0f;
       float z_carry = 0.f, q_carry = 0.f;
       for (int p0 = 0; p0 <= l_n; p0 += 32) {
         const int p = p0 + lane;
         const bool pt = p < l_n;
         const float z = ((float)(l_a + p) + 0.5f - l_mu) * l_inv;
         const float q = pt ? tail_fast(z) : 0.f;
-        if (pt && p < W) l_row[p] = z <= 0.f ? q : 1.0f - q;
+        if (l_tabled && p <= l_n) l_row[p + 1] = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
         float zpv = __shfl_up_sync(FULL, z, 1), qpv = __shfl_up_sync(FULL, q, 1);
         if (lane == 0) { zpv = z_carry; qpv = q_carry; }
         if (p <= l_n) hist_add(hlo, hhi, fold_bin(l_a + p, A.II) * RB + l_r, l_w * bin_mass(pt, p == 0, z, q, zpv, qpv));
@@ -387,6 +405,117 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
   fd = s[8]; fc = s[9]; fr = s[10];
 }
 
+// Per-lane terms of one (edge, restart) from both endpoints: the consumer's own
+// window (own = v) and then the producer's (own = u), each visiting only the own
+// points where a term can be nonzero.  kTab: both rows are in the table (clamped
+// reads against the sentinels); otherwise the values are evaluated directly.
+// All lanes of the warp call it (warp-wide trip counts).
+template <bool kDep, bool kCom, bool kUnit, bool kTab>
+__device__ __forceinline__ void edge_sides(const IterArgs &A, bool fw, bool bk, int L, const Nb &U, const Nb &Vn,
+                                           float4 &su, float4 &sv, float &fd, float &fc, float &fr) {
+  constexpr unsigned FULL = 0xffffffffu;
+  const int nu = U.b - U.a + 1, nv = Vn.b - Vn.a + 1;
+  const bool back = bk;
+  // own point j of the consumer (v) / producer (u): C from the table, phi, z phi
+  auto own = [&](const Nb &o, int j, float &C, float &f, float &zf) {
+    const float z = ((float)(o.a + j) + 0.5f - o.mu) * o.inv;
+    C = kTab ? __ldg(o.row + j + 1) : cdf_fast(z);
+    f = kInvSqrt2Pi * __expf(-0.5f * z * z);
+    zf = z * f;
+  };
+
+  // ---- consumer side (own = v):
+  //   V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
+  //   dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
+  //   dL_com,e/dC_v(t) = -C_u(t)
+  {
+    // P_u(t+1-L) != 0 for t in [au+L-1, bu+L]; C_u(t) != 0 for t >= au
+    int jlo = 0, jhi = -1;
+    if (fw) {
+      jlo = max(0, U.a + min(kDep ? L - 1 : 0, 0) - Vn.a);
+      jhi = kCom ? nv - 1 : min(nv - 1, U.b + L - Vn.a);
+    } else if (bk) {
+      jlo = max(0, U.a + L - 1 - Vn.a);
+      jhi = min(nv - 1, U.b + L - Vn.a);
+    }
+    const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
+    const int cmax = __reduce_max_sync(FULL, cnt);
+    float c_lo = cnt ? U.template val<kTab>(Vn.a + jlo - L) : 0.f;
+    for (int k2 = 0; k2 < cmax; ++k2) {
+      if (k2 < cnt) {
+        const int j = jlo + k2, t = Vn.a + j;
+        const float c_hi = U.template val<kTab>(t + 1 - L);
+        const float p = c_hi - c_lo;
+        float Cv, f, zf;
+        own(Vn, j, Cv, f, zf);
+        if (back) {
+          fr += Cv * p;
+          sv.x += p * f;
+          sv.y += p * zf;
+        } else {
+          if (kDep) {
+            fd += Cv * p;
+            sv.x += p * f;
+            sv.y += p * zf;
+          }
+          if (kCom) {
+            const float cu = (kUnit || L == 1) ? c_hi : U.template val<kTab>(t);
+            fc += cu * (1.0f - Cv);
+            sv.z -= A.alpha * cu * f;
+            sv.w -= A.alpha * cu * zf;
+          }
+        }
+        c_lo = c_hi;
+      }
+    }
+    __syncwarp();
+    if ((kDep && fw) || bk) {
+      const float tail = 1.0f - U.template val<kTab>(Vn.b + 1 - L);
+      if (back) fr += tail; else fd += tail;
+    }
+  }
+  // ---- producer side (own = u):
+  //   dV_e/dC_u(x) = -P_v(x + L), nonzero for x in [av-L, bv+1-L]
+  //   dL_com,e/dC_u(x) = 1 - C_v(x), nonzero for x <= bv
+  //   L_com,e part = sum_{x in own, x < a_v} C_u(x) + max(0, a_v - 1 - b_u)
+  {
+    int jlo = 0, jhi = -1;
+    if (fw || bk) {
+      jlo = max(0, Vn.a - L - U.a);
+      jhi = min(nu - 1, Vn.b + 1 - L - U.a);
+      if (kCom && fw) {
+        jlo = 0;
+        jhi = max(jhi, min(nu - 1, Vn.b - U.a));
+      }
+    }
+    const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
+    const int cmax = __reduce_max_sync(FULL, cnt);
+    float c_lo = cnt ? Vn.template val<kTab>(U.a + jlo + L - 1) : 0.f;
+    for (int k2 = 0; k2 < cmax; ++k2) {
+      if (k2 < cnt) {
+        const int j = jlo + k2, x = U.a + j;
+        const float c_hi = Vn.template val<kTab>(x + L);
+        float Cu, f, zf;
+        own(U, j, Cu, f, zf);
+        if (back || kDep) {
+          const float p = c_hi - c_lo;
+          su.x -= p * f;
+          su.y -= p * zf;
+        }
+        if (kCom && !back) {
+          const float cw = (kUnit || L == 1) ? c_lo : Vn.template val<kTab>(x);
+          su.z += A.alpha * (1.0f - cw) * f;
+          su.w += A.alpha * (1.0f - cw) * zf;
+          if (x < Vn.a) fc += Cu;
+        }
+        c_lo = c_hi;
+      }
+    }
+    __syncwarp();
+    if (kCom && fw) fc += (float)max(0, Vn.a - 1 - U.b);
+  }
+}
+
 // Edge pass (Eq. dep, Eq. com, App. B.3).  Block = a chunk of the edge list x one
 // restart group; lane = (edge, restart).  Each edge term is a dot product of one
 // endpoint's window with the other endpoint's CDF shifted by the latency; both
@@ -395,9 +524,11 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
 // (dV/dmu-, dV/dsigma-type sums: Ad, Bd, Ao, Bo for a forward edge, Ar, Br for a
 // back edge) to the edge's two slots, which k_update gathers per node in a fixed
 // order, and adds the edge's forward sums (exact fixed point) to the block's.
-// An edge with an endpoint window longer than the restart's threshold (at most
-// the table row) is done by the whole warp (coop_edge).
-template <bool kDep, bool kCom, bool kRec>
+// Per lane, an endpoint whose window the table row cannot hold is evaluated
+// directly; an edge with an endpoint window longer than the restart's threshold
+// is done by the whole warp (coop_edge).  kUnit: every edge has latency 1 (no
+// back edges), so C_u(t) is the bin mass's upper value.
+template <bool kDep, bool kCom, bool kRec, bool kUnit>
 __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   constexpr int T = kFwdThreads;
   constexpr unsigned FULL = 0xffffffffu;
@@ -407,14 +538,14 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   const int e_begin = ch * A.ce, e_end = min(A.nEt, e_begin + A.ce);
   const int r = tid % RB, b = g * RB + r;
   const bool bok = b < A.B;
-  const int thr = bok ? long_threshold(A.wstat, b, A.W) : A.W;
+  const int thr = bok ? long_threshold(A.wstat, b) : A.W;
   long long xdep = 0, xcom = 0, xrec = 0;  // forward sums, exact (order-free) fixed point
   const int per_pass = (T / 32) * epw;
   for (int e0 = e_begin + warp * epw; e0 < e_end; e0 += per_pass) {
     const int e = e0 + lane / RB;
     const bool present = bok && e < e_end;
     const int4 ed = present ? __ldg(A.ed + e) : make_int4(0, 0, 0, 0);
-    const int uc = ed.x, vc = ed.y, L = ed.z;
+    const int uc = ed.x, vc = ed.y, L = kUnit ? 1 : ed.z;
     const bool back = (ed.w & 1) != 0;
     const int cpos = (ed.w >> 1) + (back ? A.E : 0);  // consumer-side slot
     const size_t iu = (size_t)uc * A.B + (bok ? b : 0), iv = (size_t)vc * A.B + (bok ? b : 0);
@@ -425,11 +556,11 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
     Nb U, Vn;
     U.a = (int)(wu & 0xFFFFu); U.b = (int)(wu >> 16) - 1; U.row = A.tab + iu * A.W;
     Vn.a = (int)(wv & 0xFFFFu); Vn.b = (int)(wv >> 16) - 1; Vn.row = A.tab + iv * A.W;
-    U.mu = on ? mu_u : 0.f; U.inv = on ? 1.0f / sg_u : 1.f;
-    Vn.mu = on ? mu_v : 0.f; Vn.inv = on ? 1.0f / sg_v : 1.f;
+    U.mu = on ? mu_u : 0.f; U.inv = on ? __frcp_rn(sg_u) : 1.f;
+    Vn.mu = on ? mu_v : 0.f; Vn.inv = on ? __frcp_rn(sg_v) : 1.f;
     const int nu = U.b - U.a + 1, nv = Vn.b - Vn.a + 1;
-    U.tab = nu <= A.W;
-    Vn.tab = nv <= A.W;
+    U.tab = nu + 3 <= A.W;
+    Vn.tab = nv + 3 <= A.W;
     const bool is_long = on && (nu > thr || nv > thr);
     const bool ps = on && !is_long;                 // per-lane path
     const bool fw = ps && !back && (kDep || kCom);  // forward edge terms
@@ -437,104 +568,13 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
     float4 su = make_float4(0.f, 0.f, 0.f, 0.f), sv = make_float4(0.f, 0.f, 0.f, 0.f);
     float fd = 0.f, fc = 0.f, fr = 0.f;
 
-    // own point j of the consumer (v) / producer (u): C from the table, phi, z phi
-    auto own = [&](const Nb &o, int j, float &C, float &f, float &zf) {
-      C = __ldg(o.row + j);
-      const float z = ((float)(o.a + j) + 0.5f - o.mu) * o.inv;
-      f = kInvSqrt2Pi * __expf(-0.5f * z * z);
-      zf = z * f;
-    };
+    // ---- per-lane terms: both rows in the table (branch-free reads), then, if any
+    // lane needs it, the lanes with a window the table cannot hold ----
+    const bool tabbed = U.tab && Vn.tab;
+    edge_sides<kDep, kCom, kUnit, true>(A, fw && tabbed, bk && tabbed, L, U, Vn, su, sv, fd, fc, fr);
+    if (__any_sync(FULL, (fw || bk) && !tabbed))
+      edge_sides<kDep, kCom, kUnit, false>(A, fw && !tabbed, bk && !tabbed, L, U, Vn, su, sv, fd, fc, fr);
 
-    // ---- consumer side (own = v):
-    //   V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
-    //   dV_e/dC_v(t) = P_u(t + 1 - L);  L_com,e part = sum_{t in own} C_u(t) (1 - C_v(t))
-    //   dL_com,e/dC_v(t) = -C_u(t)
-    {
-      // P_u(t+1-L) != 0 for t in [au+L-1, bu+L]; C_u(t) != 0 for t >= au
-      int jlo = 0, jhi = -1;
-      if (fw) {
-        jlo = max(0, U.a + min(kDep ? L - 1 : 0, 0) - Vn.a);
-        jhi = kCom ? nv - 1 : min(nv - 1, U.b + L - Vn.a);
-      } else if (bk) {
-        jlo = max(0, U.a + L - 1 - Vn.a);
-        jhi = min(nv - 1, U.b + L - Vn.a);
-      }
-      const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
-      const int cmax = __reduce_max_sync(FULL, cnt);
-      float c_lo = cnt ? U.at(Vn.a + jlo - L) : 0.f;
-      for (int k2 = 0; k2 < cmax; ++k2) {
-        if (k2 < cnt) {
-          const int j = jlo + k2, t = Vn.a + j;
-          const float c_hi = U.at(t + 1 - L);
-          const float p = c_hi - c_lo;
-          float Cv, f, zf;
-          own(Vn, j, Cv, f, zf);
-          if (back) {
-            fr += Cv * p;
-            sv.x += p * f;
-            sv.y += p * zf;
-          } else {
-            if (kDep) {
-              fd += Cv * p;
-              sv.x += p * f;
-              sv.y += p * zf;
-            }
-            if (kCom) {
-              const float cu = (L == 1) ? c_hi : U.at(t);
-              fc += cu * (1.0f - Cv);
-              sv.z -= A.alpha * cu * f;
-              sv.w -= A.alpha * cu * zf;
-            }
-          }
-          c_lo = c_hi;
-        }
-      }
-      __syncwarp();
-      if ((kDep && fw) || bk) {
-        const float tail = 1.0f - U.at(Vn.b + 1 - L);
-        if (back) fr += tail; else fd += tail;
-      }
-    }
-    // ---- producer side (own = u):
-    //   dV_e/dC_u(x) = -P_v(x + L), nonzero for x in [av-L, bv+1-L]
-    //   dL_com,e/dC_u(x) = 1 - C_v(x), nonzero for x <= bv
-    //   L_com,e part = sum_{x in own, x < a_v} C_u(x) + max(0, a_v - 1 - b_u)
-    {
-      int jlo = 0, jhi = -1;
-      if (fw || bk) {
-        jlo = max(0, Vn.a - L - U.a);
-        jhi = min(nu - 1, Vn.b + 1 - L - U.a);
-        if (kCom && fw) {
-          jlo = 0;
-          jhi = max(jhi, min(nu - 1, Vn.b - U.a));
-        }
-      }
-      const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
-      const int cmax = __reduce_max_sync(FULL, cnt);
-      float c_lo = cnt ? Vn.at(U.a + jlo + L - 1) : 0.f;
-      for (int k2 = 0; k2 < cmax; ++k2) {
-        if (k2 < cnt) {
-          const int j = jlo + k2, x = U.a + j;
-          const float c_hi = Vn.at(x + L);
-          float Cu, f, zf;
-          own(U, j, Cu, f, zf);
-          if (back || kDep) {
-            const float p = c_hi - c_lo;
-            su.x -= p * f;
-            su.y -= p * zf;
-          }
-          if (kCom && !back) {
-            const float cw = (L == 1) ? c_lo : Vn.at(x);
-            su.z += A.alpha * (1.0f - cw) * f;
-            su.w += A.alpha * (1.0f - cw) * zf;
-            if (x < Vn.a) fc += Cu;
-          }
-          c_lo = c_hi;
-        }
-      }
-      __syncwarp();
-      if (kCom && fw) fc += (float)max(0, Vn.a - 1 - U.b);
-    }
     // ---- cooperative pass over this warp's long (edge, restart) items ----
     unsigned longmask = __ballot_sync(FULL, is_long);
     while (longmask) {
@@ -738,7 +778,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
     A.loss[b] = (float)L;
     A.coef[b * 4 + 0] = on_dep ? (float)((double)lam[GAUS_K_DEP] + (double)A.rho * Vk[0]) : 0.f;
     A.coef[b * 4 + 1] = on_rec ? (float)((double)lam[GAUS_K_REC] + (double)A.rho * Vk[2]) : 0.f;
-    A.thr[b] = long_threshold(A.wstat, b, A.W);
+    A.thr[b] = long_threshold(A.wstat, b);
     A.wstat[2 * b] = 0ull;
     A.wstat[2 * b + 1] = 0ull;
     const int bad = A.nonfinite[b];

@@ -224,6 +224,9 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
       P.bin_eslot[a] = b;
     }
   }
+  P.unit_lat = 1;
+  for (int i = 0; i < V; ++i)
+    if (P.out_ptr[i + 1] > P.out_ptr[i] && P.lat[i] != 1) P.unit_lat = 0;
   // edge list of the edge pass: forward edges in internal CSR order (producer,
   // consumer, Lat(producer), kind | consumer position << 1), then back edges in
   // producer order (j, i, shift, ...).  kind: 0 forward, 1 back; the consumer
