@@ -367,9 +367,41 @@ uint64_t state_hash(const gaus_state *s) {
 }
 
 void drop_graph(gaus_ctx *ctx) {
-  if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
-  ctx->gexec = nullptr;
+  for (cudaGraphExec_t *g : {&ctx->gexec, &ctx->gexec_n}) {
+    if (*g) cudaGraphExecDestroy(*g);
+    *g = nullptr;
+  }
   ctx->ghash = 0;
+}
+
+// Capture `iters` fused iterations into one executable graph.
+gaus_status capture_iterations(gaus_ctx *ctx, const gaus_state *S, int iters, cudaGraphExec_t *out) {
+  cudaStream_t cap;
+  CK(cudaStreamCreateWithFlags(&cap, cudaStreamNonBlocking), "capture stream");
+  cudaError_t e = cudaStreamBeginCapture(cap, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) {
+    cudaStreamDestroy(cap);
+    return cuda_fail(ctx, e, "begin capture");
+  }
+  gaus_status st = GAUS_OK;
+  for (int i = 0; i < iters && st == GAUS_OK; ++i)
+    st = enqueue_iteration(ctx, cap, S->mu, S->sigma, S->lambda, true, nullptr, nullptr, S->loss, S->terms,
+                           S->status, S);
+  cudaGraph_t graph = nullptr;
+  e = cudaStreamEndCapture(cap, &graph);
+  cudaStreamDestroy(cap);
+  if (st != GAUS_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return st;
+  }
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "end capture");
+  e = cudaGraphInstantiate(out, graph, 0);
+  cudaGraphDestroy(graph);
+  if (e != cudaSuccess) {
+    *out = nullptr;
+    return cuda_fail(ctx, e, "graph instantiate");
+  }
+  return GAUS_OK;
 }
 
 }  // namespace
@@ -484,35 +516,17 @@ gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *S) {
     return GAUS_EINVAL;
   }
   if (n_iters == 0) return GAUS_OK;
+  // two captured graphs of the same iteration: kGraphUnroll iterations, and one
   const uint64_t h = state_hash(S);
   if (!ctx->gexec || ctx->ghash != h) {
     drop_graph(ctx);
-    cudaStream_t cap;
-    CK(cudaStreamCreateWithFlags(&cap, cudaStreamNonBlocking), "capture stream");
-    cudaError_t e = cudaStreamBeginCapture(cap, cudaStreamCaptureModeThreadLocal);
-    if (e != cudaSuccess) {
-      cudaStreamDestroy(cap);
-      return cuda_fail(ctx, e, "begin capture");
-    }
-    gaus_status st = enqueue_iteration(ctx, cap, S->mu, S->sigma, S->lambda, true, nullptr, nullptr, S->loss,
-                                       S->terms, S->status, S);
-    cudaGraph_t graph = nullptr;
-    e = cudaStreamEndCapture(cap, &graph);
-    cudaStreamDestroy(cap);
-    if (st != GAUS_OK) {
-      if (graph) cudaGraphDestroy(graph);
-      return st;
-    }
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "end capture");
-    e = cudaGraphInstantiate(&ctx->gexec, graph, 0);
-    cudaGraphDestroy(graph);
-    if (e != cudaSuccess) {
-      ctx->gexec = nullptr;
-      return cuda_fail(ctx, e, "graph instantiate");
-    }
+    TRY(capture_iterations(ctx, S, 1, &ctx->gexec));
+    TRY(capture_iterations(ctx, S, kGraphUnroll, &ctx->gexec_n));
     ctx->ghash = h;
   }
-  for (int i = 0; i < n_iters; ++i) CK(cudaGraphLaunch(ctx->gexec, ctx->stream), "graph launch");
+  int left = n_iters;
+  for (; left >= kGraphUnroll; left -= kGraphUnroll) CK(cudaGraphLaunch(ctx->gexec_n, ctx->stream), "graph launch");
+  for (; left > 0; --left) CK(cudaGraphLaunch(ctx->gexec, ctx->stream), "graph launch");
   return GAUS_OK;
 }
 
@@ -594,7 +608,7 @@ const char *gaus_last_error(const gaus_ctx *ctx) { return ctx ? ctx->err.c_str()
 
 void gaus_destroy(gaus_ctx *ctx) {
   if (!ctx) return;
-  if (!ctx->allocs.empty() || ctx->gexec) {
+  if (!ctx->allocs.empty() || ctx->gexec || ctx->gexec_n) {
     if (ctx->stream) cudaStreamSynchronize(ctx->stream);
     else cudaDeviceSynchronize();
   }

@@ -16,6 +16,7 @@ constexpr int kFwdThreads = 256;
 constexpr int kThreads = 128;
 // Most own-window points cached in shared memory per thread (longer windows recompute).
 constexpr int kUpdThreads = 256;               // threads per k_update block
+constexpr int kGraphUnroll = 10;               // iterations per captured graph
 constexpr int kReduceSpans = 1024;             // segment spans staged per k_reduce pass
 constexpr int kTableMax = 32;                    // points per CDF table row, at most
 constexpr size_t kTableBytes = (size_t)64 << 20;  // CDF table size bound
@@ -130,7 +131,7 @@ struct gaus_ctx {
   int32_t *d_status_tmp = nullptr; // B
   float *d_loss_tmp = nullptr, *d_terms_tmp = nullptr;
   // captured iteration
-  cudaGraphExec_t gexec = nullptr;
+  cudaGraphExec_t gexec = nullptr, gexec_n = nullptr;  // one iteration, kGraphUnroll iterations
   gaus_state gstate{};
   uint64_t ghash = 0;
   std::vector<void *> allocs;
