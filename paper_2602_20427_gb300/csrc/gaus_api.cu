@@ -108,6 +108,17 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   k_nodes<<<ctx->nblk, kFwdThreads, ctx->smem_nodes, st>>>(A);
   CK(cudaGetLastError(), "k_nodes launch");
   if (ev) CK(cudaEventRecord(ev[1], st), "event");
+  // usage reduction (needs only the node pass) on the side stream, beside the edge pass
+  CK(cudaEventRecord(ctx->ev_fork, st), "fork");
+  CK(cudaStreamWaitEvent(ctx->side, ctx->ev_fork, 0), "fork wait");
+  {
+    RedArgs R;
+    R.B = P.B; R.C = P.C; R.Dh = P.Dh; R.RB = ctx->RB; R.G = ctx->G;
+    R.cls_seg_ptr = ctx->d_cls_seg_ptr; R.hpart = ctx->d_hpart; R.hspan = ctx->d_hspan; R.U = ctx->d_U;
+    k_reduce<<<ctx->red_blocks, 256, 0, ctx->side>>>(R);
+    CK(cudaGetLastError(), "k_reduce launch");
+  }
+  CK(cudaEventRecord(ctx->ev_join, ctx->side), "join record");
   EdgeKernel ke = pick_edges(on, P.II, P.unit_lat != 0);
   ke<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
   CK(cudaGetLastError(), "k_edges launch");
@@ -126,11 +137,8 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
                                                  P.nseg);
     CK(cudaGetLastError(), "k_reduce_reg launch");
   }
-  RedArgs R;
-  R.B = P.B; R.C = P.C; R.Dh = P.Dh; R.RB = ctx->RB; R.G = ctx->G;
-  R.cls_seg_ptr = ctx->d_cls_seg_ptr; R.hpart = ctx->d_hpart; R.hspan = ctx->d_hspan; R.U = ctx->d_U;
-  k_reduce<<<ctx->red_blocks, 256, 0, st>>>(R);
-  CK(cudaGetLastError(), "k_reduce launch");
+  // (k_reduce runs on the side stream, forked after k_nodes; joined here)
+  CK(cudaStreamWaitEvent(st, ctx->ev_join, 0), "join");
 
   FinArgs F;
   F.B = P.B; F.C = P.C; F.Dh = P.Dh; F.RB = ctx->RB; F.G = ctx->G; F.Ug = ctx->d_U;
@@ -272,6 +280,9 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     return GAUS_EINVAL;
   }
   TRY(set_smem_attrs(ctx));
+  CK(cudaStreamCreateWithFlags(&ctx->side, cudaStreamNonBlocking), "side stream");
+  CK(cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming), "event");
+  CK(cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming), "event");
 
   TRY(upload(ctx, &ctx->d_perm, P.perm));
   TRY(upload(ctx, &ctx->d_w, P.w));
@@ -613,7 +624,11 @@ void gaus_destroy(gaus_ctx *ctx) {
     else cudaDeviceSynchronize();
   }
   drop_graph(ctx);
+  if (ctx->side) cudaStreamSynchronize(ctx->side);
   for (void *p : ctx->allocs) cudaFree(p);
+  if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
+  if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
+  if (ctx->side) cudaStreamDestroy(ctx->side);
   delete ctx;
 }
 

@@ -80,6 +80,8 @@ struct gaus_ctx {
   gaus::Plan plan;
   gaus_hparams hp;
   cudaStream_t stream = nullptr;
+  cudaStream_t side = nullptr;                     // usage reduction beside the edge pass
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   std::string err;
   int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per node pass
   int ce = 0, nchunk = 0;        // edge pass: edges per block, edge chunks (blocks = nchunk * G)
