@@ -68,7 +68,7 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   A.out_ptr = ctx->d_out_ptr; A.out_dst = ctx->d_out_dst;
   A.bin_ptr = ctx->d_bin_ptr; A.bin_src = ctx->d_bin_src; A.bin_shift = ctx->d_bin_shift;
   A.bout_ptr = ctx->d_bout_ptr; A.bout_dst = ctx->d_bout_dst; A.bout_shift = ctx->d_bout_shift;
-  A.seg = ctx->d_seg; A.hpart = ctx->d_hpart; A.hspan = ctx->d_hspan; A.fwd = ctx->d_fwd;
+  A.seg = ctx->d_seg; A.hpart = ctx->d_hpart; A.hspan = ctx->d_hspan; A.fwdtot = ctx->d_fwdtot;
   A.nonfinite = ctx->d_nonfinite; A.win = ctx->d_win; A.tab = ctx->d_tab;
   A.wstat = ctx->d_wstat;
   A.ed = ctx->d_ed; A.nEt = P.E + P.NB; A.ce = ctx->ce; A.E = P.E; A.eslot4 = ctx->d_eslot4;
@@ -146,7 +146,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   F.terms = on; F.tau = ctx->hp.tau; F.rho = ctx->hp.rho; F.alpha = ctx->hp.alpha;
   F.w_res = ctx->hp.w_res; F.w_mem = ctx->hp.w_mem;
   F.cls_seg_ptr = ctx->d_cls_seg_ptr; F.limit = ctx->d_limit;
-  F.hpart = ctx->d_hpart; F.hspan = ctx->d_hspan; F.fwd = ctx->d_fwd; F.nfwd = ctx->nchunk;
+  F.hpart = ctx->d_hpart; F.hspan = ctx->d_hspan; F.fwdtot = ctx->d_fwdtot;
   F.lambda = lambda; F.update_lambda = adam ? 1 : 0; F.step = adam ? S->step : nullptr;
   F.beta1 = ctx->hp.beta1; F.beta2 = ctx->hp.beta2;
   F.H = ctx->d_H; F.coef = ctx->d_coef; F.loss = loss; F.terms_out = terms;
@@ -338,7 +338,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_U, (size_t)P.B * P.C * P.Dh));
   if (ctx->hp.terms & GAUS_REG_OBJ) TRY(alloc_storage_scratch(ctx));
   TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
-  TRY(scratch(ctx, &ctx->d_fwd, (size_t)ctx->nchunk * ctx->G * ctx->RB * 3));
+  TRY(scratch(ctx, &ctx->d_fwdtot, (size_t)P.B * 3));
   TRY(scratch(ctx, &ctx->d_eslot4, 2 * ((size_t)P.E + P.NB) * P.B));
   TRY(scratch(ctx, &ctx->d_win, VB));
   TRY(scratch(ctx, &ctx->d_tab, VB * ctx->W));

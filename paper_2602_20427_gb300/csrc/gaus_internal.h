@@ -113,7 +113,7 @@ struct gaus_ctx {
   // scratch
   long long *d_hpart = nullptr;  // nblk * Dh * RB fixed-point usage partials
   int2 *d_hspan = nullptr;       // nblk folded bin span written by each block
-  long long *d_fwd = nullptr;    // nchunk * G * RB * 3 forward sums (dep, com, rec), 2^32 fixed point
+  unsigned long long *d_fwdtot = nullptr;  // B * 3 forward sums (dep, com, rec), 2^32 fixed point
   long long *d_U = nullptr;      // B * C * Dh usage (k_reduce), 2^32 fixed point
   long long *d_rpart = nullptr;  // nblk_r * Dh * RBr storage partials
   long long *d_Ureg = nullptr;   // B * Dh expected (folded) storage, 2^32 fixed point

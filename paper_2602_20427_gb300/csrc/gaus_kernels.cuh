@@ -45,7 +45,7 @@ struct IterArgs {
   const int32_t *seg;
   long long *hpart;
   int2 *hspan;
-  long long *fwd;
+  unsigned long long *fwdtot;  // (B, 3) forward sums (dep, com, rec), 2^32 fixed point
   int32_t *nonfinite;
   unsigned *win;  // (V, B) packed windows a | (b + 1) << 16, written by k_nodes
   float *tab;     // (V, B, W) CDF values at the window points, written by k_nodes
@@ -76,8 +76,7 @@ struct FinArgs {
   const float *limit;
   const long long *hpart;
   const int2 *hspan;
-  const long long *fwd;  // per (edge chunk, restart group) forward sums
-  int nfwd;              // edge chunks
+  unsigned long long *fwdtot;  // (B, 3) forward sums; read and cleared
   float *lambda;      // read; updated in place when update_lambda
   int update_lambda;
   int32_t *step;      // incremented when not NULL
@@ -610,16 +609,18 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
     xrec += to_fix(fr);
   }
 
-  // ---- per-restart forward sums of this block (fixed order) ----
+  // ---- per-restart forward sums of this block ----
   s_red[0 * T + tid] = xdep;
   s_red[1 * T + tid] = xcom;
   s_red[2 * T + tid] = xrec;
   __syncthreads();
-  if (tid < RB) {
+  if (tid < RB && bok) {
     long long acc[3] = {0, 0, 0};
     for (int row = 0; row < T / RB; ++row)
       for (int k = 0; k < 3; ++k) acc[k] += s_red[k * T + row * RB + tid];
-    for (int k = 0; k < 3; ++k) A.fwd[((size_t)blk * RB + tid) * 3 + k] = acc[k];
+    // per-restart totals: exact integer sums, any order
+    for (int k = 0; k < 3; ++k)
+      if (acc[k]) atomicAdd(&A.fwdtot[3 * b + k], (unsigned long long)acc[k]);
   }
 }
 
@@ -702,11 +703,9 @@ __device__ __forceinline__ long long block_max_ll(long long x, long long *sh) {
 __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   extern __shared__ __align__(16) unsigned char smem_f[];
   long long *U = reinterpret_cast<long long *>(smem_f);  // (C + 1) * Dh
-  __shared__ long long shl[8];
-  __shared__ float shf[8];
   __shared__ long long s_m[kMaxClasses + 1], s_R[kMaxClasses];
   __shared__ float s_s[kMaxClasses + 1];
-  const int b = blockIdx.x, g = b / A.RB, r = b % A.RB, tid = threadIdx.x, Dh = A.Dh;
+  const int b = blockIdx.x, tid = threadIdx.x, Dh = A.Dh;
   const float kInvFixF = 2.3283064365386963e-10f;
 
   for (int i = tid; i < A.C * Dh; i += 256) U[i] = A.Ug[(size_t)b * A.C * Dh + i];
@@ -721,34 +720,64 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   }
   __syncthreads();
 
-  // forward sums of the edge terms over every block of this restart group
-  long long f3[3] = {0, 0, 0};
-  for (int s = tid; s < A.nfwd; s += 256)
-    for (int k = 0; k < 3; ++k) f3[k] += A.fwd[((size_t)(s * A.G + g) * A.RB + r) * 3 + k];
-  const float vdep = (float)((double)block_sum_i64(f3[0], shl) * kInvFix);
-  const float lcom = (float)((double)block_sum_i64(f3[1], shl) * kInvFix);
-  const float vrec = (float)((double)block_sum_i64(f3[2], shl) * kInvFix);
-
-  // ReLU excess over finite limits (Eq. relu), exact
-  long long ex = 0;
-  for (int i = tid; i < A.C * Dh; i += 256) {
-    const long long R = s_R[i / Dh];
-    if (R != LLONG_MAX && U[i] > R) ex += U[i] - R;
+  // forward sums of the edge terms (per-restart totals of the edge pass)
+  __shared__ float s_f3[3];
+  if (tid == 0) {
+    for (int k = 0; k < 3; ++k) {
+      s_f3[k] = (float)((double)(long long)A.fwdtot[3 * b + k] * kInvFix);
+      A.fwdtot[3 * b + k] = 0ull;
+    }
   }
-  ex = block_sum_i64(ex, shl);
 
-  // LogSumExp per class (Eq. max) and of the storage, max shifted out
+  // per class: the max (Eq. max, max shifted out) and the exact ReLU excess over
+  // finite limits (Eq. relu) in one pass, then the sums of exp; every class is
+  // warp-reduced first and the warps are combined in order after one barrier
   const int nh = A.C + (A.Ureg ? 1 : 0);
+  const int lane = tid & 31, wid = tid >> 5;
+  __shared__ long long s_wm[kMaxClasses + 1][8], s_wx[8], s_ex;
+  __shared__ float s_wsum[kMaxClasses + 1][8];
+  long long ex = 0;
   for (int c = 0; c < nh; ++c) {
+    const long long R = c < A.C ? s_R[c] : LLONG_MAX;
     long long m = LLONG_MIN;
-    for (int t = tid; t < Dh; t += 256) m = max(m, U[c * Dh + t]);
-    m = block_max_ll(m, shl);
-    float sacc = 0.f;
-    for (int t = tid; t < Dh; t += 256) sacc += expf(fix_to_float(U[c * Dh + t] - m) / A.tau);
-    sacc = block_sum_f(sacc, shf);
-    if (tid == 0) { s_m[c] = m; s_s[c] = sacc; }
+    for (int t = tid; t < Dh; t += 256) {
+      const long long u = U[c * Dh + t];
+      m = max(m, u);
+      if (R != LLONG_MAX && u > R) ex += u - R;
+    }
+    for (int o = 16; o > 0; o >>= 1) m = max(m, (long long)__shfl_xor_sync(0xffffffffu, m, o));
+    if (lane == 0) s_wm[c][wid] = m;
+  }
+  for (int o = 16; o > 0; o >>= 1) ex += __shfl_xor_sync(0xffffffffu, ex, o);
+  if (lane == 0) s_wx[wid] = ex;
+  __syncthreads();
+  if (tid < nh) {
+    long long m = LLONG_MIN;
+    for (int w = 0; w < 8; ++w) m = max(m, s_wm[tid][w]);
+    s_m[tid] = m;
+  }
+  if (tid == 32) {
+    long long e = 0;
+    for (int w = 0; w < 8; ++w) e += s_wx[w];
+    s_ex = e;
   }
   __syncthreads();
+  for (int c = 0; c < nh; ++c) {
+    const long long m = s_m[c];
+    float sacc = 0.f;
+    for (int t = tid; t < Dh; t += 256) sacc += expf(fix_to_float(U[c * Dh + t] - m) / A.tau);
+    sacc = warp_sum(sacc);
+    if (lane == 0) s_wsum[c][wid] = sacc;
+  }
+  __syncthreads();
+  if (tid < nh) {
+    float t = 0.f;
+    for (int w = 0; w < 8; ++w) t += s_wsum[tid][w];
+    s_s[tid] = t;
+  }
+  __syncthreads();
+  const float vdep = s_f3[0], lcom = s_f3[1], vrec = s_f3[2];
+  ex = s_ex;
 
   const bool on_dep = A.terms & GAUS_DEP, on_com = A.terms & GAUS_COM;
   const bool on_robj = A.terms & GAUS_RES_OBJ, on_rv = A.terms & GAUS_RES_VIOL;
