@@ -55,10 +55,28 @@ def parse():
 
 
 def workload(rank=0):
+    """The benchmark workload of one rank: the same logic-network DAG on every rank,
+    and B = 64 restarts of its own (initial state seeded by the rank), so the ranks'
+    restarts are independent and need no data-path collective (weak scaling)."""
     p = W.logic_network(1)
     B = 64
     mu, sg = W.init_state(p, B, seed=1 + rank)
     return p, B, mu, sg
+
+
+def max_over_ranks(ms, world, dist=None, device="cpu"):
+    """The job's time: the slowest rank's (max all-reduce; the only collective)."""
+    if world <= 1:
+        return float(ms)
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(steps, iters, B, world, ms):
+    """Whole-job restart-iterations/s: every rank's units over the slowest rank's time."""
+    return steps * iters * B * world / (ms / 1e3)
 
 
 def describe(p, B, iters, period=None):
@@ -232,13 +250,11 @@ def gpu_arm(args):
     ms = sum(step_ms)
     if world > 1:
         dist.barrier()
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, dist, "cuda")
     status_ok = bool(int(st["status"].abs().sum()) == 0)
     feasible = int((lstat == 0).sum())
     units = args.steps * iters * B * world
-    value = units / (ms / 1e3)
+    value = job_throughput(args.steps, iters, B, world, ms)
 
     # ---- legalize + verify alone (part of every step above; reported separately)
     lv = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -319,11 +335,7 @@ def gpu_arm(args):
             h_loss.copy_(st["loss"], non_blocking=True)
             eev[k][1].record()
         torch.cuda.synchronize()
-        ems = sum(a.elapsed_time(b) for a, b in eev)
-        if world > 1:
-            t = torch.tensor([ems], dtype=torch.float64, device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
+        ems = max_over_ranks(sum(a.elapsed_time(b) for a, b in eev), world, dist, "cuda")
         h2d = 2 * p.V * B * 4
         d2h = 2 * p.V * B * 4 + p.V * B * 4 + B * 200 + B * 4
         e2e = {"value": units / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
