@@ -74,6 +74,7 @@ def lib():
         _lib.orc_phi.argtypes = [C.c_double]
         _lib.orc_asap_alap.restype = C.c_int
         _lib.orc_legalize_modulo.restype = C.c_int
+        _lib.orc_outer_step.restype = C.c_int32
     return _lib
 
 
@@ -208,3 +209,58 @@ def verify(op: OracleProblem, s) -> dict:
     out = {f: int(getattr(r, f)) for f in REPORT_FIELDS}
     out["peak"] = [int(r.peak[c]) for c in range(min(op.C, 16))]
     return out
+
+
+def init_state(op: OracleProblem, B: int, kappa: float, sigma_min: float, mu0=None):
+    """Sec. 3.3 Initialization for B restarts; kappa and sigma_min as the float32
+    values the library receives.  Returns mu, sigma (V, B) float32."""
+    rc, order, asap, alap, cp = asap_alap(op)
+    assert rc == 0
+    mu = np.zeros((B, op.V), np.float32)
+    sg = np.zeros((B, op.V), np.float32)
+    m0 = None if mu0 is None else np.ascontiguousarray(np.asarray(mu0, np.float32).T)
+    for b in range(B):
+        lib().orc_init_state(C.c_int32(op.V), _p(asap), _p(alap), C.c_double(float(np.float32(kappa))),
+                             C.c_float(float(np.float32(sigma_min))), None if m0 is None else _p(m0[b]),
+                             _p(mu[b]), _p(sg[b]))
+    return np.ascontiguousarray(mu.T), np.ascontiguousarray(sg.T)
+
+
+def outer_step(op: OracleProblem, terms: int, w_res: float, alpha: float, w_mem: float, it: int,
+               s_legal, leg_ok, sigma_init, best: dict, state: dict):
+    """One outer step of Alg. GauS on B restarts, in place on `best` (sched (V, B)
+    int32, score (B,) float64, iter (B,) int32) and `state` (mu, sigma, m_mu, v_mu,
+    m_sigma, v_sigma (V, B) float32, step (B,) int32).  s_legal (V, B): the
+    legalization of round(mu); leg_ok (B,): its success.  The report of each
+    legalized schedule is the oracle's own verify.  Returns moved (B,)."""
+    rc, order, asap, alap, cp = asap_alap(op)
+    V, B = np.asarray(s_legal).shape
+    T = lambda a, dt: np.ascontiguousarray(np.asarray(a, dt).T)
+    sl = T(s_legal, np.int32)
+    si = T(sigma_init, np.float32)
+    bs = T(best["sched"], np.int32)
+    arr = {k: T(state[k], np.float32) for k in ("mu", "sigma", "m_mu", "v_mu", "m_sigma", "v_sigma")}
+    score = np.ascontiguousarray(best["score"], np.float64).copy()
+    biter = np.ascontiguousarray(best["iter"], np.int32).copy()
+    step = np.ascontiguousarray(state["step"], np.int32).copy()
+    moved = np.zeros(B, np.int32)
+    for b in range(B):
+        r = _Report()
+        lib().orc_verify(C.byref(op.c), _p(sl[b]), C.byref(r))
+        sc = np.zeros(1, np.float64); sc[0] = score[b]
+        it_ = np.zeros(1, np.int32); it_[0] = biter[b]
+        st_ = np.zeros(1, np.int32); st_[0] = step[b]
+        moved[b] = lib().orc_outer_step(
+            C.c_int32(V), C.c_int32(int(bool(leg_ok[b]))), _p(sl[b]), C.byref(r), C.c_uint32(terms),
+            C.c_int32(op.II), C.c_double(float(np.float32(w_res))), C.c_double(float(np.float32(alpha))),
+            C.c_double(float(np.float32(w_mem))), C.c_int32(it), _p(asap), _p(alap), _p(si[b]), _p(bs[b]),
+            _p(sc), _p(it_), _p(arr["mu"][b]), _p(arr["sigma"][b]), _p(arr["m_mu"][b]), _p(arr["v_mu"][b]),
+            _p(arr["m_sigma"][b]), _p(arr["v_sigma"][b]), _p(st_))
+        score[b], biter[b], step[b] = sc[0], it_[0], st_[0]
+    best["sched"][...] = bs.T
+    best["score"][...] = score
+    best["iter"][...] = biter
+    for k, a in arr.items():
+        state[k][...] = a.T
+    state["step"][...] = step
+    return moved

@@ -480,3 +480,60 @@ void orc_verify(const orc_problem *p, const int32_t *s, orc_report *r) {
   r->feasible = (r->n_dep_viol == 0 && r->n_lat_viol == 0 && r->n_rec_viol == 0);
   r->res_ok = (r->n_res_viol == 0);
 }
+
+/* ---- Outer loop of Alg. GauS ---- */
+
+/* Sec. 3.3 Initialization: "sigma = kappa (s_ALAP - s_ASAP)" and mu the midpoint
+ * of [ASAP, ALAP] (or a given mu0).  sigma is floored at sigma_min because a node
+ * without slack would otherwise start with sigma = 0. */
+void orc_init_state(int32_t V, const int32_t *asap, const int32_t *alap, double kappa, float sigma_min,
+                    const float *mu0, float *mu, float *sigma) {
+  for (int32_t v = 0; v < V; ++v) {
+    float sv = (float)(kappa * (double)(alap[v] - asap[v]));
+    if (!(sv >= sigma_min)) sv = sigma_min;
+    sigma[v] = sv;
+    mu[v] = mu0 ? mu0[v] : (float)(0.5 * ((double)asap[v] + (double)alap[v]));
+  }
+}
+
+/* Alg. GauS: "s = round(mu); mu, sigma <- legalize(s) if s is illegal"; App. A:
+ * when the legalized schedule does not improve on the running best, the
+ * optimizer is reset to the prior best.  A legalized schedule is a candidate when
+ * legalization succeeded and it has no dependency, latency or recurrence
+ * violation (and no resource overflow when the ReLU resource term is on); its
+ * score is the discrete objective of the active terms. */
+int32_t orc_outer_step(int32_t V, int32_t leg_ok, const int32_t *s_legal, const orc_report *r, uint32_t terms,
+                       int32_t II, double w_res, double alpha, double w_mem, int32_t iter, const int32_t *asap,
+                       const int32_t *alap, const float *sigma_init, int32_t *best_sched, double *best_score,
+                       int32_t *best_iter, float *mu, float *sigma, float *m_mu, float *v_mu, float *m_sg,
+                       float *v_sg, int32_t *step) {
+  int32_t moved = 0;
+  for (int32_t v = 0; v < V; ++v) {
+    const double m = (double)mu[v];
+    if (!isfinite(m) || floor(m + 0.5) != (double)s_legal[v]) ++moved;
+  }
+  const int cand = leg_ok && r->feasible && (!(terms & ORC_RES_VIOL) || r->res_ok);
+  double score = 0.0;
+  if (terms & ORC_RES_OBJ) score += w_res * (double)r->L_res;
+  if (terms & ORC_COM) score += alpha * (double)r->L_com;
+  if (terms & ORC_REG_OBJ) score += w_mem * (double)(II > 0 ? r->L_mmem : r->L_mem);
+  const int had_best = *best_iter >= 0;
+  const int improved = cand && score < *best_score;
+  const int illegal = !leg_ok || moved > 0;
+  if (improved) {
+    for (int32_t v = 0; v < V; ++v) best_sched[v] = s_legal[v];
+    *best_score = score;
+    *best_iter = iter;
+  }
+  if (illegal) {
+    for (int32_t v = 0; v < V; ++v) {
+      if (improved) mu[v] = (float)s_legal[v];
+      else if (had_best) mu[v] = (float)best_sched[v];
+      else mu[v] = (float)(0.5 * ((double)asap[v] + (double)alap[v]));
+      sigma[v] = sigma_init[v];
+      m_mu[v] = v_mu[v] = m_sg[v] = v_sg[v] = 0.0f;
+    }
+    *step = 0;
+  }
+  return leg_ok ? moved : -1;
+}

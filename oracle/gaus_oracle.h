@@ -107,6 +107,23 @@ int orc_legalize_modulo(const orc_problem *p, const int32_t *order, int32_t *s);
 /* Discrete objectives and constraint checks (Sec. 2.1) of one schedule. */
 void orc_verify(const orc_problem *p, const int32_t *s, orc_report *r);
 
+/* Sec. 3.3 Initialization for one restart: sigma_v = kappa (ALAP_v - ASAP_v),
+ * floored at sigma_min, and mu_v = (ASAP_v + ALAP_v) / 2 (or mu0[v] when given);
+ * computed in double, stored as the float32 state. */
+void orc_init_state(int32_t V, const int32_t *asap, const int32_t *alap, double kappa, float sigma_min,
+                    const float *mu0, float *mu, float *sigma);
+
+/* One outer step of Alg. GauS for one restart (sampling, "legalize if illegal";
+ * App. A: reset to the prior best).  s_legal = legalization of round(mu), leg_ok
+ * its success, r its report.  Updates the best (sched, score, iter) and, when the
+ * rounded schedule was illegal, resets mu, sigma, the Adam moments and step.
+ * Returns the number of nodes legalization moved, or -1 when it failed. */
+int32_t orc_outer_step(int32_t V, int32_t leg_ok, const int32_t *s_legal, const orc_report *r, uint32_t terms,
+                       int32_t II, double w_res, double alpha, double w_mem, int32_t iter, const int32_t *asap,
+                       const int32_t *alap, const float *sigma_init, int32_t *best_sched, double *best_score,
+                       int32_t *best_iter, float *mu, float *sigma, float *m_mu, float *v_mu, float *m_sg,
+                       float *v_sg, int32_t *step);
+
 #ifdef __cplusplus
 }
 #endif
