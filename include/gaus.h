@@ -181,10 +181,11 @@ gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st);
 /* Kernel-level timing of gaus_iterate: runs n_iters iterations exactly as
  * gaus_iterate does, but launched without a graph and with CUDA events between
  * the phases, and adds the mean duration in milliseconds of each phase of an
- * iteration to ms_out[0..3] (host array of 4): [0] window table, [1] node/edge
- * pass (k_fwd alone), [2] storage pass + usage reduction + per-restart finalize,
- * [3] gradient gather + Adam.  Synchronises the context's stream.  Library
- * feature for measurement; not on the hot path. */
+ * iteration to ms_out[0..3] (host array of 4): [0] node pass (windows, CDF table,
+ * usage histograms), [1] edge pass (the usage reduction runs beside it on a second
+ * stream), [2] storage pass + per-restart finalize, [3] gradient gather + Adam.
+ * Synchronises the context's stream.  Library feature for measurement; not on the
+ * hot path. */
 gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st, double *ms_out);
 
 /* Round every mean to s = floor(mu + 1/2) (Sec. 3.3 Sampling; exact for every
@@ -201,6 +202,54 @@ gaus_status gaus_round(gaus_ctx *ctx, const float *mu, int32_t *sched);
 /* Verify B schedules (Sec. 2.1): sched (V, B) int32 device; rep (B) device array
  * of gaus_report, written.  Integer arithmetic only. */
 gaus_status gaus_verify(gaus_ctx *ctx, const int32_t *sched, gaus_report *rep);
+
+/* ---- Outer loop of Alg. GauS: initialization, sampling, legalization, best ---- */
+
+/* Best legal schedule found per restart; device arrays owned by the caller. */
+typedef struct {
+  int32_t *sched;   /* (V, B) best legal schedule (caller node ids)               */
+  double *score;    /* (B) its score; +inf while none was found                   */
+  int32_t *iter;    /* (B) iteration count when it was found; -1 while none       */
+} gaus_best;
+
+/* Initialization of Alg. GauS (Sec. 3.3 Initialization): per node
+ * sigma = max(kappa (ALAP - ASAP), sigma_min) (computed in double, rounded to
+ * float) and mu = mu0 (device (V, B)) or, when mu0 is NULL, the midpoint
+ * (ASAP + ALAP) / 2; Adam moments and step zeroed, lambda = lambda0, status OK.
+ * sigma_init (V, B) device, written with that sigma (the value a reset returns
+ * to), or NULL.  best (optional): score = +inf, iter = -1.  EINVAL on NULL state
+ * pointers or kappa not finite and > 0. */
+gaus_status gaus_init_state(gaus_ctx *ctx, const float *mu0, float kappa, const gaus_state *st, float *sigma_init,
+                            const gaus_best *best);
+
+/* One outer step of Alg. GauS on all B restarts (sampling and "legalize if
+ * illegal"; App. A: the optimizer is reset to the prior best when the legalized
+ * schedule does not improve on it).  Inputs (device): sched (V, B) = the
+ * legalization of round(st->mu) and leg_status (B) from gaus_legalize, rep (B)
+ * from gaus_verify of sched, sigma_init (V, B) from gaus_init_state; iter is
+ * recorded with a new best.  Per restart:
+ *   candidate: leg_status OK, rep.feasible, and rep.res_ok if GAUS_RES_VIOL is on;
+ *     score = w_res L_res [RES_OBJ] + alpha L_com [COM] + w_mem (II > 0 ? L_mmem
+ *     : L_mem) [REG_OBJ] (double);
+ *   improved: a candidate with score < best score: best sched, score, iter set;
+ *   illegal: some node of sched differs from round(mu), or legalization failed:
+ *     reset mu to sched if improved, else to the best schedule if there is one,
+ *     else to (ASAP + ALAP) / 2; sigma to sigma_init; Adam moments and step to 0;
+ *     lambda kept.
+ * moved (B) device, written: nodes legalization moved (-1 if it failed).
+ * Asynchronous on the context's stream. */
+gaus_status gaus_outer_step(gaus_ctx *ctx, const int32_t *sched, const int32_t *leg_status, const gaus_report *rep,
+                            int32_t iter, const float *sigma_init, const gaus_state *st, const gaus_best *best,
+                            int32_t *moved);
+
+/* n_periods periods of Alg. GauS on the device, with no host synchronisation:
+ * each runs `period` fused iterations (gaus_iterate), then gaus_legalize,
+ * gaus_verify and gaus_outer_step (iteration count iter0 + (p + 1) period).
+ * Work buffers (device, caller-owned, overwritten): sched (V, B) int32,
+ * leg_status (B), rep (B), moved (B).  EINVAL on NULL pointers or counts < 1. */
+gaus_status gaus_solve(gaus_ctx *ctx, int32_t n_periods, int32_t period, int32_t iter0, const gaus_state *st,
+                       const float *sigma_init, const gaus_best *best, int32_t *sched, int32_t *leg_status,
+                       gaus_report *rep, int32_t *moved);
 
 /* Expected usage per resource class without allocating device memory.
  *

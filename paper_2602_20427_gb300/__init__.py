@@ -57,6 +57,10 @@ class Report(C.Structure):
                 ("feasible", C.c_int32), ("res_ok", C.c_int32)]
 
 
+class Best(C.Structure):
+    _fields_ = [("sched", C.c_void_p), ("score", C.c_void_p), ("iter", C.c_void_p)]
+
+
 class State(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("mu", "sigma", "m_mu", "v_mu", "m_sigma", "v_sigma",
                                           "lambda_", "step", "loss", "terms", "status")]
@@ -243,6 +247,78 @@ class Gaus:
         ms = (C.c_double * 4)(0.0, 0.0, 0.0, 0.0)
         self._check(lib().gaus_profile_iterate(self._ctx, C.c_int32(n), C.byref(s), ms))
         return list(ms)
+
+    def _state(self, state):
+        torch = self.torch
+        VB, f32 = (self.V, self.B), torch.float32
+        return State(*(self._dev(state[k], f32, VB).value for k in ("mu", "sigma", "m_mu", "v_mu", "m_sigma",
+                                                                     "v_sigma")),
+                     self._dev(state["lambda_"], f32, (self.B, K)).value,
+                     self._dev(state["step"], torch.int32, (self.B,)).value,
+                     self._dev(state["loss"], f32, (self.B,)).value,
+                     self._dev(state["terms"], f32, (self.B, NT)).value,
+                     self._dev(state["status"], torch.int32, (self.B,)).value)
+
+    def _best(self, best):
+        torch = self.torch
+        return Best(self._dev(best["sched"], torch.int32, (self.V, self.B)).value,
+                    self._dev(best["score"], torch.float64, (self.B,)).value,
+                    self._dev(best["iter"], torch.int32, (self.B,)).value)
+
+    def init_state(self, kappa=1.0 / 6.0, mu0=None, device="cuda"):
+        """Alg. GauS initialization (gaus_init_state): a fresh state (mu = mu0 or the
+        ASAP/ALAP midpoint, sigma = max(kappa (ALAP - ASAP), sigma_min)), the
+        sigma a reset returns to, and an empty best."""
+        torch = self.torch
+        VB = (self.V, self.B)
+        z = lambda: torch.empty(VB, dtype=torch.float32, device=device)
+        state = dict(mu=z(), sigma=z(), m_mu=z(), v_mu=z(), m_sigma=z(), v_sigma=z(),
+                     lambda_=torch.empty((self.B, K), dtype=torch.float32, device=device),
+                     step=torch.empty(self.B, dtype=torch.int32, device=device),
+                     loss=torch.zeros(self.B, dtype=torch.float32, device=device),
+                     terms=torch.zeros((self.B, NT), dtype=torch.float32, device=device),
+                     status=torch.empty(self.B, dtype=torch.int32, device=device))
+        sigma_init = z()
+        best = dict(sched=torch.zeros(VB, dtype=torch.int32, device=device),
+                    score=torch.empty(self.B, dtype=torch.float64, device=device),
+                    iter=torch.empty(self.B, dtype=torch.int32, device=device))
+        s, bst = self._state(state), self._best(best)
+        m0 = None if mu0 is None else self._dev(mu0, torch.float32, VB)
+        self._check(lib().gaus_init_state(self._ctx, m0, C.c_float(kappa), C.byref(s),
+                                          self._dev(sigma_init, torch.float32, VB), C.byref(bst)))
+        return state, sigma_init, best
+
+    def outer_step(self, state, sched, leg_status, rep, it, sigma_init, best, moved=None):
+        """One outer step (gaus_outer_step); returns the nodes legalization moved per restart."""
+        torch = self.torch
+        if moved is None:
+            moved = torch.empty(self.B, dtype=torch.int32, device=sched.device)
+        s, bst = self._state(state), self._best(best)
+        self._check(lib().gaus_outer_step(self._ctx, self._dev(sched, torch.int32, (self.V, self.B)),
+                                          self._dev(leg_status, torch.int32, (self.B,)),
+                                          C.c_void_p(rep.data_ptr()), C.c_int32(it),
+                                          self._dev(sigma_init, torch.float32, (self.V, self.B)), C.byref(s),
+                                          C.byref(bst), self._dev(moved, torch.int32, (self.B,))))
+        return moved
+
+    def solve(self, n_periods, period, state, sigma_init, best, iter0=0, work=None):
+        """n_periods periods of Alg. GauS on the device (gaus_solve); returns the work
+        buffers (last legalized schedules, their status and reports, nodes moved)."""
+        torch = self.torch
+        dev = state["mu"].device
+        if work is None:
+            work = dict(sched=torch.empty((self.V, self.B), dtype=torch.int32, device=dev),
+                        leg_status=torch.empty(self.B, dtype=torch.int32, device=dev),
+                        rep=torch.empty(C.sizeof(Report) * self.B, dtype=torch.uint8, device=dev),
+                        moved=torch.empty(self.B, dtype=torch.int32, device=dev))
+        s, bst = self._state(state), self._best(best)
+        self._check(lib().gaus_solve(self._ctx, C.c_int32(n_periods), C.c_int32(period), C.c_int32(iter0),
+                                     C.byref(s), self._dev(sigma_init, torch.float32, (self.V, self.B)),
+                                     C.byref(bst), self._dev(work["sched"], torch.int32, (self.V, self.B)),
+                                     self._dev(work["leg_status"], torch.int32, (self.B,)),
+                                     C.c_void_p(work["rep"].data_ptr()),
+                                     self._dev(work["moved"], torch.int32, (self.B,))))
+        return work
 
     def round(self, mu, sched=None):
         torch = self.torch

@@ -346,6 +346,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_coef, (size_t)P.B * 4));
   TRY(scratch(ctx, &ctx->d_wstat, (size_t)P.B * 2));
   TRY(scratch(ctx, &ctx->d_thr, (size_t)P.B));
+  TRY(scratch(ctx, &ctx->d_decision, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_nonfinite, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_status_tmp, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_loss_tmp, (size_t)P.B));
@@ -612,6 +613,72 @@ gaus_status gaus_verify(gaus_ctx *ctx, const int32_t *sched, gaus_report *rep) {
   A.succ_ptr = ctx->d_csucc_ptr; A.succ_dst = ctx->d_csucc_dst; A.limit = ctx->d_limit;
   k_verify<<<P.B, 256, ctx->smem_ver, ctx->stream>>>(A);
   CK(cudaGetLastError(), "k_verify launch");
+  return GAUS_OK;
+}
+
+gaus_status gaus_init_state(gaus_ctx *ctx, const float *mu0, float kappa, const gaus_state *S, float *sigma_init,
+                            const gaus_best *best) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!S || !S->mu || !S->sigma || !S->m_mu || !S->v_mu || !S->m_sigma || !S->v_sigma || !S->lambda || !S->step ||
+      !S->status || !std::isfinite(kappa) || !(kappa > 0.0f)) {
+    ctx->err = "gaus_init_state: NULL state pointer or kappa not finite and > 0";
+    return GAUS_EINVAL;
+  }
+  const Plan &P = ctx->plan;
+  const size_t n = (size_t)P.V * P.B;
+  k_init_state<<<(int)std::min<size_t>((n + 255) / 256, 4096), 256, 0, ctx->stream>>>(
+      mu0, S->mu, S->sigma, sigma_init, S->m_mu, S->v_mu, S->m_sigma, S->v_sigma, ctx->d_asap, ctx->d_alap, P.V, P.B,
+      (double)kappa, ctx->hp.sigma_min);
+  CK(cudaGetLastError(), "k_init_state launch");
+  k_init_restart<<<(P.B + 127) / 128, 128, 0, ctx->stream>>>(S->lambda, S->step, S->status,
+                                                                best ? best->score : nullptr,
+                                                                best ? best->iter : nullptr, P.B, ctx->hp.lambda0);
+  CK(cudaGetLastError(), "k_init_restart launch");
+  return GAUS_OK;
+}
+
+gaus_status gaus_outer_step(gaus_ctx *ctx, const int32_t *sched, const int32_t *leg_status, const gaus_report *rep,
+                            int32_t iter, const float *sigma_init, const gaus_state *S, const gaus_best *best,
+                            int32_t *moved) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!sched || !leg_status || !rep || !sigma_init || !S || !S->mu || !S->sigma || !S->m_mu || !S->v_mu ||
+      !S->m_sigma || !S->v_sigma || !S->step || !best || !best->sched || !best->score || !best->iter || !moved) {
+    ctx->err = "gaus_outer_step: NULL pointer";
+    return GAUS_EINVAL;
+  }
+  const Plan &P = ctx->plan;
+  OuterArgs O;
+  O.sched = sched; O.leg_status = leg_status; O.rep = rep; O.mu = S->mu;
+  O.V = P.V; O.B = P.B; O.II = P.II; O.iter = iter; O.terms = ctx->hp.terms;
+  O.w_res = ctx->hp.w_res; O.alpha = ctx->hp.alpha; O.w_mem = ctx->hp.w_mem;
+  O.best_score = best->score; O.best_iter = best->iter; O.step = S->step; O.moved = moved;
+  O.decision = ctx->d_decision;
+  k_outer_decide<<<P.B, 256, 0, ctx->stream>>>(O);
+  CK(cudaGetLastError(), "k_outer_decide launch");
+  const size_t n = (size_t)P.V * P.B;
+  k_outer_apply<<<(int)std::min<size_t>((n + 255) / 256, 4096), 256, 0, ctx->stream>>>(
+      ctx->d_decision, sched, best->sched, S->mu, S->sigma, sigma_init, S->m_mu, S->v_mu, S->m_sigma, S->v_sigma,
+      ctx->d_asap, ctx->d_alap, P.V, P.B);
+  CK(cudaGetLastError(), "k_outer_apply launch");
+  return GAUS_OK;
+}
+
+gaus_status gaus_solve(gaus_ctx *ctx, int32_t n_periods, int32_t period, int32_t iter0, const gaus_state *S,
+                       const float *sigma_init, const gaus_best *best, int32_t *sched, int32_t *leg_status,
+                       gaus_report *rep, int32_t *moved) {
+  if (!ctx) return GAUS_EINVAL;
+  if (n_periods < 1 || period < 1 || !S || !sigma_init || !best || !sched || !leg_status || !rep || !moved) {
+    ctx->err = "gaus_solve: NULL pointer or n_periods, period < 1";
+    return GAUS_EINVAL;
+  }
+  for (int32_t p = 0; p < n_periods; ++p) {
+    gaus_status st = gaus_iterate(ctx, period, S);
+    if (st == GAUS_OK) st = gaus_legalize(ctx, S->mu, sched, leg_status);
+    if (st == GAUS_OK) st = gaus_verify(ctx, sched, rep);
+    if (st == GAUS_OK)
+      st = gaus_outer_step(ctx, sched, leg_status, rep, iter0 + (p + 1) * period, sigma_init, S, best, moved);
+    if (st != GAUS_OK) return st;
+  }
   return GAUS_OK;
 }
 

@@ -300,4 +300,103 @@ __global__ void k_lambda(float *lambda, const float *terms, int B, unsigned on, 
   if (on & GAUS_REC) lambda[b * GAUS_K + GAUS_K_REC] += rho * T[GAUS_T_VREC];
 }
 
+// ---- Outer loop of Alg. GauS ----
+
+// Initialization (Sec. 3.3): sigma = max(kappa (ALAP - ASAP), sigma_min) per node
+// (in double, then rounded to float), mu = mu0 or the midpoint (ASAP + ALAP) / 2;
+// Adam moments zeroed.  Caller-order (V, B) arrays.
+__global__ void k_init_state(const float *mu0, float *mu, float *sg, float *sg_init, float *m1, float *v1, float *m2,
+                             float *v2, const int32_t *asap, const int32_t *alap, int V, int B, double kappa,
+                             float sigma_min) {
+  const size_t n = (size_t)V * B;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+    const int v = (int)(i / B);
+    const float s0 = fmaxf((float)(kappa * (double)(alap[v] - asap[v])), sigma_min);
+    mu[i] = mu0 ? mu0[i] : 0.5f * (float)(asap[v] + alap[v]);
+    sg[i] = s0;
+    if (sg_init) sg_init[i] = s0;
+    m1[i] = 0.f; v1[i] = 0.f; m2[i] = 0.f; v2[i] = 0.f;
+  }
+}
+
+__global__ void k_init_restart(float *lambda, int32_t *step, int32_t *status, double *best_score,
+                               int32_t *best_iter, int B, float lambda0) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  for (int k = 0; k < GAUS_K; ++k) lambda[b * GAUS_K + k] = lambda0;
+  step[b] = 0;
+  status[b] = GAUS_OK;
+  if (best_score) best_score[b] = __longlong_as_double(0x7ff0000000000000ll);  // +inf
+  if (best_iter) best_iter[b] = -1;
+}
+
+struct OuterArgs {
+  const int32_t *sched, *leg_status;
+  const gaus_report *rep;
+  const float *mu;
+  int V, B, II, iter;
+  unsigned terms;
+  double w_res, alpha, w_mem;
+  double *best_score;
+  int32_t *best_iter, *step, *moved, *decision;
+};
+
+// Outer-step decision of one restart (block b): the nodes legalization moved
+// (sched != round(mu)), the candidate's score and whether it improves the best
+// (App. A: the legalized schedule, or a reset to the prior best).  decision bits:
+// 1 improved, 2 illegal (reset), 4 a best existed before this step.
+__global__ void __launch_bounds__(256) k_outer_decide(const OuterArgs A) {
+  __shared__ int sh[8];
+  const int b = blockIdx.x, tid = threadIdx.x;
+  int moved = 0;
+  for (int v = tid; v < A.V; v += 256) {
+    bool bad = false;
+    const int r = round_half_up(A.mu[(size_t)v * A.B + b], bad);
+    if (bad || r != A.sched[(size_t)v * A.B + b]) ++moved;
+  }
+  for (int o = 16; o > 0; o >>= 1) moved += __shfl_xor_sync(0xffffffffu, moved, o);
+  if ((tid & 31) == 0) sh[tid >> 5] = moved;
+  __syncthreads();
+  if (tid != 0) return;
+  moved = 0;
+  for (int w = 0; w < 8; ++w) moved += sh[w];
+  const bool leg_ok = A.leg_status[b] == GAUS_OK;
+  const gaus_report &R = A.rep[b];
+  const bool cand = leg_ok && R.feasible && (!(A.terms & GAUS_RES_VIOL) || R.res_ok);
+  double score = 0.0;
+  if (A.terms & GAUS_RES_OBJ) score += A.w_res * (double)R.L_res;
+  if (A.terms & GAUS_COM) score += A.alpha * (double)R.L_com;
+  if (A.terms & GAUS_REG_OBJ) score += A.w_mem * (double)(A.II > 0 ? R.L_mmem : R.L_mem);
+  const bool had_best = A.best_iter[b] >= 0;
+  const bool improved = cand && score < A.best_score[b];
+  const bool illegal = !leg_ok || moved > 0;
+  if (improved) {
+    A.best_score[b] = score;
+    A.best_iter[b] = A.iter;
+  }
+  if (illegal) A.step[b] = 0;
+  A.moved[b] = leg_ok ? moved : -1;
+  A.decision[b] = (improved ? 1 : 0) | (illegal ? 2 : 0) | (had_best ? 4 : 0);
+}
+
+// Outer-step update of every (node, restart), coalesced: the improved restarts'
+// best schedules, and the resets of the illegal ones (mu from the legalized or the
+// prior best schedule, or the midpoint; sigma from sigma_init; moments zeroed).
+__global__ void k_outer_apply(const int32_t *decision, const int32_t *sched, int32_t *best_sched, float *mu,
+                              float *sg, const float *sg_init, float *m1, float *v1, float *m2, float *v2,
+                              const int32_t *asap, const int32_t *alap, int V, int B) {
+  const size_t n = (size_t)V * B;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+    const int v = (int)(i / B), b = (int)(i % B);
+    const int d = decision[b];
+    if (d & 1) best_sched[i] = sched[i];
+    if (d & 2) {
+      mu[i] = (d & 1) ? (float)sched[i]
+                      : ((d & 4) ? (float)best_sched[i] : 0.5f * (float)(asap[v] + alap[v]));
+      sg[i] = sg_init[i];
+      m1[i] = 0.f; v1[i] = 0.f; m2[i] = 0.f; v2[i] = 0.f;
+    }
+  }
+}
+
 }  // namespace gaus

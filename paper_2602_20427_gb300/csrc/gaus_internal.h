@@ -129,6 +129,7 @@ struct gaus_ctx {
   float *d_coef = nullptr;       // B * 4 (c_dep, c_rec, Adam bias corrections)
   unsigned long long *d_wstat = nullptr;  // B * 2 window statistics of the iteration
   int32_t *d_thr = nullptr;      // B long-window thresholds
+  int32_t *d_decision = nullptr; // B outer-step decisions
   int32_t *d_nonfinite = nullptr;  // B flags
   int32_t *d_status_tmp = nullptr; // B
   float *d_loss_tmp = nullptr, *d_terms_tmp = nullptr;

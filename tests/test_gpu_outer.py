@@ -1,0 +1,126 @@
+"""The outer loop of Alg. GauS on the GPU (gaus_init_state, gaus_outer_step,
+gaus_solve) against the oracle: initialization and every outer-step decision
+bit-exact on the same inputs; full solves whose best schedules the oracle
+verifies and scores identically."""
+import numpy as np
+import pytest
+
+import oracle
+import workloads as W
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def g():
+    import paper_2602_20427_gb300 as g
+    g.build()
+    g.lib()
+    return g
+
+
+def _np(state):
+    return {k: v.cpu().numpy().copy() for k, v in state.items()}
+
+
+def _score(r, terms, hp, II):
+    s = 0.0
+    if terms & W.RES_OBJ:
+        s += float(np.float32(hp.w_res)) * r["L_res"]
+    if terms & W.COM:
+        s += float(np.float32(hp.alpha)) * r["L_com"]
+    if terms & W.REG_OBJ:
+        s += float(np.float32(hp.w_mem)) * (r["L_mmem"] if II > 0 else r["L_mem"])
+    return s
+
+
+@pytest.mark.parametrize("mu0", [False, True])
+def test_init_state_matches_oracle(g, mu0):
+    p = W.random_layered(1)
+    B = 8
+    hp = g.default_hparams(terms=p.terms)
+    ctx = g.Gaus(p, B, hp)
+    m0 = W.init_state(p, B, 3)[0] if mu0 else None
+    state, sigma_init, best = ctx.init_state(kappa=1.0 / 6.0, mu0=None if m0 is None else torch.from_numpy(m0).cuda())
+    torch.cuda.synchronize()
+    op = oracle.OracleProblem(p)
+    mu, sg = oracle.init_state(op, B, 1.0 / 6.0, hp.sigma_min, mu0=m0)
+    np.testing.assert_array_equal(state["mu"].cpu().numpy(), mu)
+    np.testing.assert_array_equal(state["sigma"].cpu().numpy(), sg)
+    np.testing.assert_array_equal(sigma_init.cpu().numpy(), sg)
+    for k in ("m_mu", "v_mu", "m_sigma", "v_sigma"):
+        assert not state[k].cpu().numpy().any()
+    assert np.all(state["step"].cpu().numpy() == 0)
+    np.testing.assert_array_equal(state["lambda_"].cpu().numpy(), np.float32(hp.lambda0))
+    assert np.all(np.isinf(best["score"].cpu().numpy())) and np.all(best["iter"].cpu().numpy() == -1)
+    ctx.close()
+
+
+@pytest.mark.parametrize("maker", ["random_layered", "modulo_loop"])
+def test_outer_steps_match_oracle(g, maker):
+    # several outer steps with iterations between them; each step is checked on the
+    # GPU's own inputs (state, legalized schedules), so every decision is compared
+    p = getattr(W, maker)(1)
+    B = 16
+    hp = g.default_hparams(terms=p.terms, lr=0.05)
+    ctx = g.Gaus(p, B, hp)
+    state, sigma_init, best = ctx.init_state(kappa=1.0 / 6.0)
+    # spread the restarts: some rounded schedules legal, some not
+    rng = np.random.default_rng(5)
+    state["mu"] += torch.from_numpy(rng.normal(0, 1.5, size=(p.V, B)).astype(np.float32)).cuda()
+    op = oracle.OracleProblem(p)
+    seen = set()
+    for step in range(4):
+        ctx.iterate(15, state)
+        sched, lst = ctx.legalize(state["mu"])
+        rep = ctx.verify_raw(sched)
+        torch.cuda.synchronize()
+        before_state, before_best = _np(state), _np(best)
+        s_np, l_np = sched.cpu().numpy(), lst.cpu().numpy()
+        moved = ctx.outer_step(state, sched, lst, rep, 100 * (step + 1), sigma_init, best)
+        torch.cuda.synchronize()
+        o_state = {k: before_state[k].copy() for k in ("mu", "sigma", "m_mu", "v_mu", "m_sigma", "v_sigma",
+                                                         "step")}
+        o_best = {k: before_best[k].copy() for k in ("sched", "score", "iter")}
+        o_moved = oracle.outer_step(op, p.terms, hp.w_res, hp.alpha, hp.w_mem, 100 * (step + 1), s_np,
+                                    l_np == 0, sigma_init.cpu().numpy(), o_best, o_state)
+        np.testing.assert_array_equal(moved.cpu().numpy(), o_moved)
+        after = _np(state)
+        for k in o_state:
+            np.testing.assert_array_equal(after[k], o_state[k], err_msg=k)
+        np.testing.assert_array_equal(best["sched"].cpu().numpy(), o_best["sched"])
+        np.testing.assert_array_equal(best["score"].cpu().numpy(), o_best["score"])
+        np.testing.assert_array_equal(best["iter"].cpu().numpy(), o_best["iter"])
+        m = o_moved
+        seen.update({"legal" if x == 0 else ("illegal" if x > 0 else "failed") for x in m})
+    assert "illegal" in seen          # the resets were exercised
+    ctx.close()
+
+
+@pytest.mark.parametrize("maker", ["tiny_layered", "random_layered", "logic_network"])
+def test_solve_best_schedules_verify(g, maker):
+    # without the ReLU resource term a candidate needs dependency feasibility only,
+    # which Alg. 1 gives within the horizon, so most restarts find one; the resource
+    # rule of the candidates is checked bit for bit by test_outer_steps_match_oracle
+    p = getattr(W, maker)(2) if maker != "logic_network" else W.logic_network(2, V=2000, depth=40)
+    B = 32
+    hp = g.default_hparams(terms=p.terms & ~W.RES_VIOL)
+    ctx = g.Gaus(p, B, hp)
+    state, sigma_init, best = ctx.init_state(kappa=1.0 / 6.0)
+    work = ctx.solve(6, 50, state, sigma_init, best)
+    torch.cuda.synchronize()
+    op = oracle.OracleProblem(p)
+    it = best["iter"].cpu().numpy()
+    sc = best["score"].cpu().numpy()
+    bs = best["sched"].cpu().numpy()
+    assert np.all(np.isin(it, [-1] + [50 * (k + 1) for k in range(6)]))
+    assert np.sum(it >= 0) >= B // 2
+    for b in np.nonzero(it >= 0)[0]:
+        r = oracle.verify(op, bs[:, b])
+        assert r["feasible"] == 1
+        assert sc[b] == _score(r, hp.terms, hp, p.II)
+    assert np.all(np.isfinite(state["mu"].cpu().numpy())) and np.all(state["status"].cpu().numpy() == 0)
+    mv = work["moved"].cpu().numpy()
+    assert np.all(mv >= -1)
+    ctx.close()
