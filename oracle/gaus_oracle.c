@@ -526,8 +526,11 @@ int32_t orc_outer_step(int32_t V, int32_t leg_ok, const int32_t *s_legal, const 
     *best_iter = iter;
   }
   if (illegal) {
+    /* "mu, sigma <- legalize(s)": the legalized schedule, unless it does not improve
+     * on a prior best (then that best); the midpoint only when legalization failed
+     * and there is no best */
     for (int32_t v = 0; v < V; ++v) {
-      if (improved) mu[v] = (float)s_legal[v];
+      if (improved || (leg_ok && !had_best)) mu[v] = (float)s_legal[v];
       else if (had_best) mu[v] = (float)best_sched[v];
       else mu[v] = (float)(0.5 * ((double)asap[v] + (double)alap[v]));
       sigma[v] = sigma_init[v];

@@ -122,3 +122,27 @@ def test_score_weights_and_terms():
     state, best, si = fresh(op, mu)
     oracle.outer_step(op, W.RES_OBJ | W.RES_VIOL, 1.0, 1.0, 1.0, 10, np.int32([[0], [0]]), [1], si, best, state)
     assert best["iter"][0] == -1
+
+
+def test_illegal_without_best_takes_the_legalized_schedule():
+    # Alg. GauS: mu <- legalize(s) when s is illegal; with no prior best to return to,
+    # the legalized schedule is taken even when it is no candidate.  Nodes 0 -> 1 and
+    # an independent node 2, one step per class of limit 1, D = 4:
+    # ASAP = (0, 1, 0), ALAP = (2, 3, 3).  round(mu) = (1, 1, 2) violates 0 -> 1;
+    # Alg. 1 gives (1, 2, 2), where nodes 1 and 2 share step 2: usage 2 > 1.
+    i32 = lambda x: np.asarray(x, np.int32)
+    p = W.Problem(name="tri", V=3, src=i32([0]), dst=i32([1]), lat=i32([1, 1, 1]), cls=i32([0, 0, 0]), C=1,
+                  limit=np.array([1.0]), demand=i32([1, 1, 1]), bits=i32([1, 1, 1]), D=4)
+    op = oracle.OracleProblem(p)
+    rc, order, asap, alap, cp = oracle.asap_alap(op)
+    np.testing.assert_array_equal(asap, [0, 1, 0])
+    np.testing.assert_array_equal(alap, [2, 3, 3])
+    s_legal = oracle.legalize_regular(op, order, asap, alap, np.int32([1, 1, 2]))
+    np.testing.assert_array_equal(s_legal, [1, 2, 2])
+    state, best, si = fresh(op, np.float32([[1.2], [0.6], [2.4]]))      # rounds to (1, 1, 2)
+    terms = W.DEP | W.RES_OBJ | W.RES_VIOL
+    moved = oracle.outer_step(op, terms, 1.0, 1.0, 1.0, 100, s_legal[:, None], [1], si, best, state)
+    assert moved[0] == 1
+    assert best["iter"][0] == -1                                         # over the limit: no candidate
+    np.testing.assert_array_equal(state["mu"][:, 0], np.float32([1, 2, 2]))
+    assert state["step"][0] == 0
