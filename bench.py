@@ -50,6 +50,7 @@ def parse():
                     help="run N iterations kernel by kernel, then one more, print the phase times and exit "
                          "(a fixed launch sequence for ncu captures at iteration N)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-solver", action="store_true", help="skip the complete-solver run (gaus_solve)")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
 
@@ -311,6 +312,32 @@ def gpu_arm(args):
               "note": "initial state of the same workload with lr = 1e-20, so every iteration has the "
                       "initial +-6 sigma windows (the most expensive point of the run)"}
 
+    # ---- the complete solver: the outer loop of Alg. GauS on the device (gaus_solve)
+    # from the kappa initialization, one solve of the same length; anytime quality
+    solver = None
+    if not args.no_solver:
+        ctxS = g.Gaus(p, B, hp)
+        bufs = ctxS.init_state(kappa=1.0 / 6.0)
+        work = ctxS.solve(1, period, *bufs)                    # captures the graphs
+        ctxS.init_state(kappa=1.0 / 6.0, out=bufs)
+        evS = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+        torch.cuda.synchronize()
+        evS[0].record()
+        ctxS.solve(iters // period, period, *bufs, work=work)
+        evS[1].record()
+        torch.cuda.synchronize()
+        sms = evS[0].elapsed_time(evS[1])
+        bsc = bufs[2]["score"].cpu().numpy()
+        found = np.isfinite(bsc)
+        solver = {"value": iters * B / (sms / 1e3), "unit": UNIT, "ms": sms,
+                  "init": "kappa = 1/6: sigma = max(kappa (ALAP - ASAP), sigma_min), mu = (ASAP + ALAP) / 2",
+                  "periods": iters // period, "period": period,
+                  "restarts_with_feasible_best": int(found.sum()),
+                  "best_score_min": float(bsc[found].min()) if found.any() else None,
+                  "best_score_mean": float(bsc[found].mean()) if found.any() else None,
+                  "score": "L_res + alpha L_com of the best legal schedule (no resource overflow)"}
+        ctxS.close()
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -368,6 +395,7 @@ def gpu_arm(args):
                                            "k_edges_first_period": fwd_first, "k_edges_last_period": fwd_last},
                 "legalize_verify_ms": legalize_verify_ms,
                 "steady_fixed_sigma": steady,
+                "solver": solver,
                 "step_ms": step_ms,
                 "status_ok": status_ok, "legalized_ok": feasible, "wall_s": wall,
                 "cpu_baseline": cpu}

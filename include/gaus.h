@@ -233,9 +233,10 @@ gaus_status gaus_init_state(gaus_ctx *ctx, const float *mu0, float kappa, const 
  *     : L_mem) [REG_OBJ] (double);
  *   improved: a candidate with score < best score: best sched, score, iter set;
  *   illegal: some node of sched differs from round(mu), or legalization failed:
- *     reset mu to sched if improved, else to the best schedule if there is one,
- *     else to (ASAP + ALAP) / 2; sigma to sigma_init; Adam moments and step to 0;
- *     lambda kept.
+ *     reset mu to sched (Alg. GauS: mu <- legalize(s)) unless sched does not
+ *     improve on an existing best (then that best), or legalization failed (then
+ *     the best if any, else (ASAP + ALAP) / 2); sigma to sigma_init; Adam moments
+ *     and step to 0; lambda kept.
  * moved (B) device, written: nodes legalization moved (-1 if it failed).
  * Asynchronous on the context's stream. */
 gaus_status gaus_outer_step(gaus_ctx *ctx, const int32_t *sched, const int32_t *leg_status, const gaus_report *rep,

@@ -265,12 +265,20 @@ class Gaus:
                     self._dev(best["score"], torch.float64, (self.B,)).value,
                     self._dev(best["iter"], torch.int32, (self.B,)).value)
 
-    def init_state(self, kappa=1.0 / 6.0, mu0=None, device="cuda"):
+    def init_state(self, kappa=1.0 / 6.0, mu0=None, device="cuda", out=None):
         """Alg. GauS initialization (gaus_init_state): a fresh state (mu = mu0 or the
         ASAP/ALAP midpoint, sigma = max(kappa (ALAP - ASAP), sigma_min)), the
-        sigma a reset returns to, and an empty best."""
+        sigma a reset returns to, and an empty best.  out = (state, sigma_init,
+        best) re-initialises those buffers in place."""
         torch = self.torch
         VB = (self.V, self.B)
+        if out is not None:
+            state, sigma_init, best = out
+            s, bst = self._state(state), self._best(best)
+            m0 = None if mu0 is None else self._dev(mu0, torch.float32, VB)
+            self._check(lib().gaus_init_state(self._ctx, m0, C.c_float(kappa), C.byref(s),
+                                              self._dev(sigma_init, torch.float32, VB), C.byref(bst)))
+            return out
         z = lambda: torch.empty(VB, dtype=torch.float32, device=device)
         state = dict(mu=z(), sigma=z(), m_mu=z(), v_mu=z(), m_sigma=z(), v_sigma=z(),
                      lambda_=torch.empty((self.B, K), dtype=torch.float32, device=device),

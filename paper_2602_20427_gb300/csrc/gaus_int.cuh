@@ -344,7 +344,8 @@ struct OuterArgs {
 // Outer-step decision of one restart (block b): the nodes legalization moved
 // (sched != round(mu)), the candidate's score and whether it improves the best
 // (App. A: the legalized schedule, or a reset to the prior best).  decision bits:
-// 1 improved, 2 illegal (reset), 4 a best existed before this step.
+// 1 improved, 2 illegal (reset), 4 a best existed before this step, 8 legalization
+// succeeded.
 __global__ void __launch_bounds__(256) k_outer_decide(const OuterArgs A) {
   __shared__ int sh[8];
   const int b = blockIdx.x, tid = threadIdx.x;
@@ -376,7 +377,7 @@ __global__ void __launch_bounds__(256) k_outer_decide(const OuterArgs A) {
   }
   if (illegal) A.step[b] = 0;
   A.moved[b] = leg_ok ? moved : -1;
-  A.decision[b] = (improved ? 1 : 0) | (illegal ? 2 : 0) | (had_best ? 4 : 0);
+  A.decision[b] = (improved ? 1 : 0) | (illegal ? 2 : 0) | (had_best ? 4 : 0) | (leg_ok ? 8 : 0);
 }
 
 // Outer-step update of every (node, restart), coalesced: the improved restarts'
@@ -391,8 +392,11 @@ __global__ void k_outer_apply(const int32_t *decision, const int32_t *sched, int
     const int d = decision[b];
     if (d & 1) best_sched[i] = sched[i];
     if (d & 2) {
-      mu[i] = (d & 1) ? (float)sched[i]
-                      : ((d & 4) ? (float)best_sched[i] : 0.5f * (float)(asap[v] + alap[v]));
+      // the legalized schedule (Alg. GauS), unless it does not improve on a prior
+      // best (App. A: then that best); the midpoint only when legalization failed
+      // and there is no best
+      mu[i] = ((d & 1) || ((d & 8) && !(d & 4))) ? (float)sched[i]
+                                                 : ((d & 4) ? (float)best_sched[i] : 0.5f * (float)(asap[v] + alap[v]));
       sg[i] = sg_init[i];
       m1[i] = 0.f; v1[i] = 0.f; m2[i] = 0.f; v2[i] = 0.f;
     }
