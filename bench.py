@@ -50,7 +50,7 @@ def parse():
                     help="run N iterations kernel by kernel, then one more, print the phase times and exit "
                          "(a fixed launch sequence for ncu captures at iteration N)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-solver", action="store_true", help="skip the complete-solver run (gaus_solve)")
+    ap.add_argument("--no-solver", action="store_true", help="skip the complete-solver runs (gaus_solve)")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
 
@@ -338,6 +338,52 @@ def gpu_arm(args):
                   "score": "L_res + alpha L_com of the best legal schedule (no resource overflow)"}
         ctxS.close()
 
+    # ---- Formulation C (modulo scheduling) sweep: II in {MII, 1.25 MII, 1.5 MII} on the
+    # loop-body workload, the complete solver from that workload's initialization
+    # (mu = ASAP + N(0, 2), sigma = 1.5; the kappa initialization spans the whole
+    # horizon here, D = 3 II)
+    sweep = None
+    if not args.no_solver and rank == 0:
+        sweep = []
+        for factor in (1.0, 1.25, 1.5):
+            pm = W.modulo_loop(1, ii_factor=factor)
+            Bm = 32
+            mu_m, sg_m = W.init_state(pm, Bm, seed=1)
+            mu_m = torch.from_numpy(mu_m).cuda()
+            hpm = g.default_hparams(terms=pm.terms)
+            cm = g.Gaus(pm, Bm, hpm)
+
+            def init_m(out=None):
+                bufs_m = cm.init_state(kappa=1.0 / 6.0, mu0=mu_m, out=out)
+                bufs_m[0]["sigma"].fill_(float(sg_m[0, 0]))
+                bufs_m[1].fill_(float(sg_m[0, 0]))
+                return bufs_m
+
+            bm = init_m()
+            wm = cm.solve(1, period, *bm)
+            init_m(out=bm)
+            evm = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            n_per = 10
+            torch.cuda.synchronize()
+            evm[0].record()
+            cm.solve(n_per, period, *bm, work=wm)
+            evm[1].record()
+            torch.cuda.synchronize()
+            mms = evm[0].elapsed_time(evm[1])
+            sc = bm[2]["score"].cpu().numpy()
+            fnd = np.isfinite(sc)
+            ls = wm["leg_status"].cpu().numpy()
+            sweep.append({"ii_factor": factor, "II": pm.II, "D": pm.D, "V": pm.V, "E": pm.E, "back_edges": pm.NB,
+                          "B": Bm, "iterations": n_per * period,
+                          "restart_iterations_per_s": n_per * period * Bm / (mms / 1e3),
+                          "restarts_with_feasible_best": int(fnd.sum()),
+                          "best_score_min": float(sc[fnd].min()) if fnd.any() else None,
+                          "best_score_mean": float(sc[fnd].mean()) if fnd.any() else None,
+                          "last_legalize_not_converged": int((ls == 7).sum()),
+                          "init": "mu = ASAP + N(0, 2), sigma = 1.5 (seeded)",
+                          "score": "w_mem L_mmem of the best legal schedule (no resource overflow)"})
+            cm.close()
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -396,6 +442,7 @@ def gpu_arm(args):
                 "legalize_verify_ms": legalize_verify_ms,
                 "steady_fixed_sigma": steady,
                 "solver": solver,
+                "formulation_c_sweep": sweep,
                 "step_ms": step_ms,
                 "status_ok": status_ok, "legalized_ok": feasible, "wall_s": wall,
                 "cpu_baseline": cpu}

@@ -188,21 +188,22 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   return GAUS_OK;
 }
 
+// The dynamic shared-memory limit is a per-kernel attribute of the process, not of
+// a context: set it to the device maximum once per kernel, so that contexts of
+// different sizes can be used side by side (each launch still requests its own size).
 gaus_status set_smem_attrs(gaus_ctx *ctx) {
-  CK(cudaFuncSetAttribute((const void *)k_nodes, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_nodes),
-     "smem attr nodes");
-  CK(cudaFuncSetAttribute((const void *)k_finalize, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_fin),
-     "smem attr fin");
-  CK(cudaFuncSetAttribute((const void *)k_reg_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_rfwd),
-     "smem attr reg fwd");
-  CK(cudaFuncSetAttribute((const void *)k_reg_bwd, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_rbwd),
-     "smem attr reg bwd");
-  CK(cudaFuncSetAttribute((const void *)k_verify, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ctx->smem_ver),
-     "smem attr ver");
-  if (ctx->smem_leg)
-    CK(cudaFuncSetAttribute((const void *)k_legalize_regular_smem, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                            (int)ctx->smem_leg),
-       "smem attr legalize");
+  const void *fns[] = {(const void *)k_nodes, (const void *)k_finalize, (const void *)k_reg_fwd,
+                       (const void *)k_reg_bwd, (const void *)k_verify, (const void *)k_legalize_regular_smem};
+  int dev = 0, optin = 0;
+  CK(cudaGetDevice(&dev), "cudaGetDevice");
+  CK(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev), "smem opt-in");
+  for (const void *f : fns) {
+    cudaFuncAttributes fa;
+    CK(cudaFuncGetAttributes(&fa, f), "cudaFuncGetAttributes");
+    CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes),
+       "smem attr");
+  }
+  (void)ctx;
   return GAUS_OK;
 }
 

@@ -185,3 +185,23 @@ def test_iterate_tracks_oracle_trajectory(g):
     np.testing.assert_allclose(gl[0], ol[0], rtol=1e-4)
     np.testing.assert_allclose(gl, ol, rtol=2e-2)
     ctx.close()
+
+
+def test_two_live_contexts_of_different_sizes(g):
+    # kernel launch limits are per process: a second, smaller context must not break
+    # the first one's launches (legalize, verify, iterate interleaved)
+    big, small = W.random_layered(1), W.tiny_layered(1)
+    ctxs = []
+    for p, B in ((big, 16), (small, 4)):
+        c = g.Gaus(p, B, g.default_hparams(terms=p.terms))
+        mu, sg = W.init_state(p, B, 1)
+        st = c.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), 1e-6)
+        ctxs.append((c, st, p))
+    for c, st, p in ctxs * 2:
+        c.iterate(2, st)
+        sched, status = c.legalize(st["mu"])
+        c.verify(sched)
+        torch.cuda.synchronize()
+        assert np.all(status.cpu().numpy() == 0)
+    for c, _, _ in ctxs:
+        c.close()
