@@ -23,6 +23,8 @@ _LIB = os.path.join(_HERE, "_build", "liboracle.so")
 DEP, COM, RES_OBJ, RES_VIOL, REG_OBJ, REC = 1, 2, 4, 8, 16, 32
 K_DEP, K_RES, K_REC, K = 0, 1, 2, 3
 T_RES, T_COM, T_REG, T_VDEP, T_VRES, T_VREC, NT = 0, 1, 2, 3, 4, 5, 6
+# CDF families of the relaxation (Sec. 3.2; App. D)
+GAUSSIAN, LOGISTIC, LAPLACE, CAUCHY = 0, 1, 2, 3
 
 
 def build(force: bool = False) -> str:
@@ -50,7 +52,8 @@ class _Problem(C.Structure):
 
 class _Hparams(C.Structure):
     _fields_ = [("tau", C.c_double), ("rho", C.c_double), ("alpha", C.c_double),
-                ("w_res", C.c_double), ("w_mem", C.c_double), ("terms", C.c_uint32)]
+                ("w_res", C.c_double), ("w_mem", C.c_double), ("terms", C.c_uint32),
+                ("family", C.c_int32)]
 
 
 class _Report(C.Structure):
@@ -72,6 +75,10 @@ def lib():
         _lib.orc_Phi.argtypes = [C.c_double]
         _lib.orc_phi.restype = C.c_double
         _lib.orc_phi.argtypes = [C.c_double]
+        _lib.orc_F.restype = C.c_double
+        _lib.orc_F.argtypes = [C.c_int32, C.c_double]
+        _lib.orc_f.restype = C.c_double
+        _lib.orc_f.argtypes = [C.c_int32, C.c_double]
         _lib.orc_asap_alap.restype = C.c_int
         _lib.orc_legalize_modulo.restype = C.c_int
         _lib.orc_outer_step.restype = C.c_int32
@@ -113,10 +120,20 @@ def phi(z: float) -> float:
     return lib().orc_phi(float(z))
 
 
-def bin_masses(D: int, mu: float, sigma: float) -> np.ndarray:
+def F(family: int, z: float) -> float:
+    """CDF of a family in z = (x - mu) / sigma, scale-matched to N(0, 1) (App. D)."""
+    return lib().orc_F(int(family), float(z))
+
+
+def f(family: int, z: float) -> float:
+    """Density of a family in z = (x - mu) / sigma (App. D)."""
+    return lib().orc_f(int(family), float(z))
+
+
+def bin_masses(D: int, mu: float, sigma: float, family: int = GAUSSIAN) -> np.ndarray:
     """Eq. round over d = 0..D-1 with open boundary bins."""
     P = np.zeros(D, dtype=np.float64)
-    lib().orc_bin_masses(C.c_int32(D), C.c_double(mu), C.c_double(sigma), _p(P))
+    lib().orc_bin_masses(C.c_int32(D), C.c_int32(family), C.c_double(mu), C.c_double(sigma), _p(P))
     return P
 
 
@@ -132,8 +149,9 @@ def asap_alap(op: OracleProblem):
     return rc, order, asap, alap, cp.value
 
 
-def hparams(tau=1e-2, rho=1e-4, alpha=1.0, w_res=1.0, w_mem=1.0, terms=DEP | COM | RES_OBJ):
-    return _Hparams(tau, rho, alpha, w_res, w_mem, terms)
+def hparams(tau=1e-2, rho=1e-4, alpha=1.0, w_res=1.0, w_mem=1.0, terms=DEP | COM | RES_OBJ,
+            family=GAUSSIAN):
+    return _Hparams(tau, rho, alpha, w_res, w_mem, terms, family)
 
 
 def loss_grad(op: OracleProblem, hp, mu, sigma, lam):
@@ -155,13 +173,13 @@ def loss_grad(op: OracleProblem, hp, mu, sigma, lam):
     return loss, terms, np.ascontiguousarray(gmu.T), np.ascontiguousarray(gsg.T)
 
 
-def expected_hist(op: OracleProblem, mu, sigma):
+def expected_hist(op: OracleProblem, mu, sigma, family: int = GAUSSIAN):
     """Expected usage U (C, Dh) and storage Reg (Dh,) of one restart."""
     mu = np.ascontiguousarray(np.asarray(mu, np.float64))
     sigma = np.ascontiguousarray(np.asarray(sigma, np.float64))
     U = np.zeros((op.C, op.Dh))
     R = np.zeros(op.Dh)
-    lib().orc_expected_hist(C.byref(op.c), _p(mu), _p(sigma), _p(U), _p(R))
+    lib().orc_expected_hist(C.byref(op.c), C.c_int32(family), _p(mu), _p(sigma), _p(U), _p(R))
     return U, R
 
 

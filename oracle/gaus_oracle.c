@@ -34,18 +34,64 @@
 double orc_Phi(double z) { return 0.5 * erfc(-z / sqrt(2.0)); }
 double orc_phi(double z) { return exp(-0.5 * z * z) / sqrt(2.0 * M_PI); }
 
-/* Eq. round: P^d = Phi((d + 1/2 - mu)/sigma) - Phi((d - 1/2 - mu)/sigma), the
- * lower limit of bin 0 at -inf and the upper limit of bin D-1 at +inf
- * (Sec. 3.2 footnote).  Also returns dP/dmu and dP/dsigma when asked. */
-static void bin_masses_and_derivs(int32_t D, double mu, double sigma, double *P,
+/* App. D: the family's standard CDF replaces Phi in Eq. round, its scale matched
+ * to N(mu, sigma^2) so that one sigma means a comparable spread:
+ *   logistic  s     = sigma sqrt(3) / pi   (same variance)
+ *   Laplace   b     = sigma / sqrt(2)      (same variance)
+ *   Cauchy    gamma = sigma sqrt(2 ln 2)   (same full width at half maximum)
+ * In z = (x - mu) / sigma each family is G(z / c) for its standard CDF G and
+ * c = s / sigma, b / sigma or gamma / sigma; the density in z is g(z / c) / c. */
+static double family_scale(int32_t fam) {
+  switch (fam) {
+    case ORC_LOGISTIC: return sqrt(3.0) / M_PI;
+    case ORC_LAPLACE: return 1.0 / sqrt(2.0);
+    case ORC_CAUCHY: return sqrt(2.0 * log(2.0));
+    default: return 1.0;
+  }
+}
+
+double orc_F(int32_t fam, double z) {
+  const double y = z / family_scale(fam);
+  switch (fam) {
+    case ORC_LOGISTIC: {  /* 1 / (1 + e^-y), written with e^-|y| so that no exp overflows */
+      const double e = exp(-fabs(y));
+      return y >= 0.0 ? 1.0 / (1.0 + e) : e / (1.0 + e);
+    }
+    case ORC_LAPLACE:     /* 1/2 e^y below the centre, 1 - 1/2 e^-y above it */
+      return y < 0.0 ? 0.5 * exp(y) : 1.0 - 0.5 * exp(-y);
+    case ORC_CAUCHY:      /* 1/2 + atan(y) / pi */
+      return 0.5 + atan(y) / M_PI;
+    default:
+      return orc_Phi(z);
+  }
+}
+
+double orc_f(int32_t fam, double z) {
+  const double c = family_scale(fam), y = z / c;
+  switch (fam) {
+    case ORC_LOGISTIC: {  /* e^-y / (1 + e^-y)^2, even in y */
+      const double e = exp(-fabs(y));
+      return e / ((1.0 + e) * (1.0 + e)) / c;
+    }
+    case ORC_LAPLACE: return 0.5 * exp(-fabs(y)) / c;
+    case ORC_CAUCHY: return 1.0 / (M_PI * (1.0 + y * y)) / c;
+    default: return orc_phi(z);
+  }
+}
+
+/* Eq. round: P^d = F((d + 1/2 - mu)/sigma) - F((d - 1/2 - mu)/sigma), F = Phi for
+ * the Gaussian (App. D for the other families), the lower limit of bin 0 at -inf
+ * and the upper limit of bin D-1 at +inf (Sec. 3.2 footnote).  Also returns
+ * dP/dmu and dP/dsigma when asked. */
+static void bin_masses_and_derivs(int32_t D, int32_t fam, double mu, double sigma, double *P,
                                   double *dPdmu, double *dPdsig) {
   for (int32_t d = 0; d < D; ++d) {
     double z_lo = (d - 0.5 - mu) / sigma, z_hi = (d + 0.5 - mu) / sigma;
-    double F_lo = (d == 0) ? 0.0 : orc_Phi(z_lo);
-    double F_hi = (d == D - 1) ? 1.0 : orc_Phi(z_hi);
-    /* dPhi((x - mu)/sigma)/dmu = -phi(z)/sigma ; d/dsigma = -z phi(z)/sigma */
-    double f_lo = (d == 0) ? 0.0 : orc_phi(z_lo);
-    double f_hi = (d == D - 1) ? 0.0 : orc_phi(z_hi);
+    double F_lo = (d == 0) ? 0.0 : orc_F(fam, z_lo);
+    double F_hi = (d == D - 1) ? 1.0 : orc_F(fam, z_hi);
+    /* dF((x - mu)/sigma)/dmu = -f(z)/sigma ; d/dsigma = -z f(z)/sigma */
+    double f_lo = (d == 0) ? 0.0 : orc_f(fam, z_lo);
+    double f_hi = (d == D - 1) ? 0.0 : orc_f(fam, z_hi);
     double zf_lo = (d == 0) ? 0.0 : z_lo * f_lo;
     double zf_hi = (d == D - 1) ? 0.0 : z_hi * f_hi;
     P[d] = F_hi - F_lo;
@@ -54,8 +100,8 @@ static void bin_masses_and_derivs(int32_t D, double mu, double sigma, double *P,
   }
 }
 
-void orc_bin_masses(int32_t D, double mu, double sigma, double *P) {
-  bin_masses_and_derivs(D, mu, sigma, P, NULL, NULL);
+void orc_bin_masses(int32_t D, int32_t fam, double mu, double sigma, double *P) {
+  bin_masses_and_derivs(D, fam, mu, sigma, P, NULL, NULL);
 }
 
 static int32_t fold_len(const orc_problem *p) { return p->II > 0 ? p->II : p->D; }
@@ -152,14 +198,14 @@ static void expected_reg(const orc_problem *p, const adj_list *succ, const doubl
   }
 }
 
-void orc_expected_hist(const orc_problem *p, const double *mu, const double *sigma,
+void orc_expected_hist(const orc_problem *p, int32_t fam, const double *mu, const double *sigma,
                        double *U, double *Reg) {
   int32_t V = p->V, D = p->D, Dh = fold_len(p);
   double *P = malloc(sizeof(double) * (size_t)V * D);
   double *Cum = malloc(sizeof(double) * (size_t)V * D);
   double *R = malloc(sizeof(double) * (size_t)D);
   for (int32_t v = 0; v < V; ++v) {
-    bin_masses_and_derivs(D, mu[v], sigma[v], P + (size_t)v * D, NULL, NULL);
+    bin_masses_and_derivs(D, fam, mu[v], sigma[v], P + (size_t)v * D, NULL, NULL);
     cumulative(P + (size_t)v * D, D, Cum + (size_t)v * D);
   }
   for (int32_t i = 0; i < p->C * Dh; ++i) U[i] = 0.0;
@@ -195,7 +241,7 @@ static void loss_grad_one(const orc_problem *p, const orc_hparams *h, const doub
   double *gMReg = calloc((size_t)Dh, sizeof(double));
 
   for (int32_t v = 0; v < V; ++v) {
-    bin_masses_and_derivs(D, mu[v], sigma[v], P + (size_t)v * D, dPm + (size_t)v * D,
+    bin_masses_and_derivs(D, h->family, mu[v], sigma[v], P + (size_t)v * D, dPm + (size_t)v * D,
                           dPs + (size_t)v * D);
     cumulative(P + (size_t)v * D, D, Cum + (size_t)v * D);
   }

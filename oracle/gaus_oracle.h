@@ -54,9 +54,16 @@ typedef struct {
   int32_t D, II;                /* horizon; initiation interval (0 = regular)       */
 } orc_problem;
 
+/* CDF family of the relaxation (Sec. 3.2 with Phi; App. D for the others) */
+#define ORC_GAUSSIAN 0
+#define ORC_LOGISTIC 1
+#define ORC_LAPLACE  2
+#define ORC_CAUCHY   3
+
 typedef struct {
   double tau, rho, alpha, w_res, w_mem;
   uint32_t terms;
+  int32_t family;               /* ORC_GAUSSIAN .. ORC_CAUCHY                        */
 } orc_hparams;
 
 typedef struct {
@@ -70,8 +77,13 @@ typedef struct {
 double orc_Phi(double z);
 double orc_phi(double z);
 
+/* CDF F and density f of a family in the standardized z = (x - mu) / sigma,
+ * scale-matched to N(0, 1) (App. D); F = Phi, f = phi for ORC_GAUSSIAN. */
+double orc_F(int32_t fam, double z);
+double orc_f(int32_t fam, double z);
+
 /* Bin masses of Eq. round over d = 0..D-1, with open first and last bins. */
-void orc_bin_masses(int32_t D, double mu, double sigma, double *P);
+void orc_bin_masses(int32_t D, int32_t fam, double mu, double sigma, double *P);
 
 /* Topological order (Kahn), ASAP, ALAP, critical path.
  * returns 0 ok, 1 cycle, 2 critical path longer than D. */
@@ -81,7 +93,7 @@ int orc_asap_alap(int32_t V, int32_t E, const int32_t *src, const int32_t *dst,
 
 /* Expected histograms for one restart: usage U[c*Dh + t] and storage Reg[t],
  * folded modulo II when II > 0 (Dh = II), else Dh = D. */
-void orc_expected_hist(const orc_problem *p, const double *mu, const double *sigma,
+void orc_expected_hist(const orc_problem *p, int32_t fam, const double *mu, const double *sigma,
                        double *U, double *Reg);
 
 /* Loss, term values and gradient for B restarts (OpenMP over restarts). */

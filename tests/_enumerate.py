@@ -1,20 +1,35 @@
 """Brute-force enumeration over every discrete schedule of a tiny DAG.
 
-Independent of the oracle: bin masses come from scipy's ``ndtr`` and the
+Independent of the oracle: bin masses come from scipy's ``ndtr`` (or, for the
+other CDF families of App. D, scipy.stats' distributions) and the
 discrete objectives are evaluated per schedule from the definitions of
 Sec. 2.1 (Dep, Res, Mem, Rec) and App. B.1 (Com), then weighted by the
 product of independent bin probabilities (Sec. 3.1-3.2).
 """
 import itertools
 
+import math
+
 import numpy as np
+from scipy import stats
 from scipy.special import ndtr
 
+# App. D scale matching, as the scipy `scale` of each family for sigma = 1:
+# logistic s = sqrt(3)/pi and Laplace b = 1/sqrt(2) (unit variance), Cauchy
+# gamma = sqrt(2 ln 2) (the normal's half width at half maximum)
+FAMILY_CDF = {
+    0: ndtr,
+    1: lambda z: stats.logistic.cdf(z, scale=math.sqrt(3.0) / math.pi),
+    2: lambda z: stats.laplace.cdf(z, scale=1.0 / math.sqrt(2.0)),
+    3: lambda z: stats.cauchy.cdf(z, scale=math.sqrt(2.0 * math.log(2.0))),
+}
 
-def bin_probs(D, mu, sigma):
-    """P{floor(X + 1/2) = d} for X ~ N(mu, sigma^2), d = 0..D-1, open end bins."""
+
+def bin_probs(D, mu, sigma, family=0):
+    """P{floor(X + 1/2) = d}, d = 0..D-1, open end bins, for X = mu + sigma Z with
+    Z of the given family (0 normal, 1 logistic, 2 Laplace, 3 Cauchy)."""
     edges = (np.arange(D + 1) - 0.5 - mu) / sigma
-    cdf = ndtr(edges)
+    cdf = np.asarray(FAMILY_CDF[family](edges), dtype=np.float64)
     cdf[0] = 0.0
     cdf[-1] = 1.0
     return np.diff(cdf)
@@ -43,9 +58,9 @@ def discrete_metrics(p, s):
     return dep, com, use, mem, rec
 
 
-def expectations(p, mu, sigma):
+def expectations(p, mu, sigma, family=0):
     """Exact expectations by summing over all D^V schedules."""
-    P = [bin_probs(p.D, mu[v], sigma[v]) for v in range(p.V)]
+    P = [bin_probs(p.D, mu[v], sigma[v], family) for v in range(p.V)]
     E = {"dep": 0.0, "com": 0.0, "use": np.zeros((p.C, p.D)), "mem": np.zeros(p.D), "rec": 0.0}
     for s in itertools.product(range(p.D), repeat=p.V):
         w = 1.0
