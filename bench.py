@@ -52,6 +52,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-solver", action="store_true", help="skip the complete-solver runs (gaus_solve)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-families", action="store_true", help="skip the CDF-family timings")
     return ap.parse_args()
 
 
@@ -384,6 +385,33 @@ def gpu_arm(args):
                           "score": "w_mem L_mmem of the best legal schedule (no resource overflow)"})
             cm.close()
 
+    # ---- CDF families (App. D): the first 100 fused iterations of the same workload
+    # from the same initialization with the normal, logistic, Laplace and Cauchy
+    # relaxations (heavier tails: wider windows)
+    families = None
+    if not args.no_families and rank == 0:
+        families = []
+        for fam, name in ((g.GAUSSIAN, "gaussian"), (g.LOGISTIC, "logistic"), (g.LAPLACE, "laplace"),
+                          (g.CAUCHY, "cauchy")):
+            hpf = g.default_hparams(terms=p.terms, family=fam)
+            cf = g.Gaus(p, B, hpf)
+            sf = cf.new_state(dmu0, dsg0, hpf.lambda0)
+            cf.iterate(10, sf)
+            sf = cf.new_state(dmu0, dsg0, hpf.lambda0)
+            evf = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            n_f = 100
+            torch.cuda.synchronize()
+            evf[0].record()
+            cf.iterate(n_f, sf)
+            evf[1].record()
+            torch.cuda.synchronize()
+            fms = evf[0].elapsed_time(evf[1])
+            families.append({"family": name, "iterations": n_f,
+                             "restart_iterations_per_s": n_f * B / (fms / 1e3),
+                             "ms_per_iteration": fms / n_f,
+                             "mean_loss_after": float(sf["loss"].mean().item())})
+            cf.close()
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -443,6 +471,7 @@ def gpu_arm(args):
                 "steady_fixed_sigma": steady,
                 "solver": solver,
                 "formulation_c_sweep": sweep,
+                "cdf_families": families,
                 "step_ms": step_ms,
                 "status_ok": status_ok, "legalized_ok": feasible, "wall_s": wall,
                 "cpu_baseline": cpu}

@@ -65,6 +65,16 @@ typedef enum {
 #define GAUS_T_VREC 5   /* expected recurrence violations */
 #define GAUS_NT     6
 
+/* CDF family that rounds X_v to a step (gaus_hparams.family).  The normal of
+ * Sec. 3.2 or, in its place (App. D), a logistic, Laplace or Cauchy CDF whose
+ * scale is matched to sigma: logistic s = sigma sqrt(3)/pi and Laplace
+ * b = sigma/sqrt(2) have the variance sigma^2; Cauchy gamma = sigma sqrt(2 ln 2)
+ * has the normal's full width at half maximum. */
+#define GAUS_GAUSSIAN 0
+#define GAUS_LOGISTIC 1
+#define GAUS_LAPLACE  2
+#define GAUS_CAUCHY   3
+
 /* Scheduling problem (Sec. 2.1).  All pointers are HOST pointers, read during
  * gaus_create and not kept.  Node ids are 0..V-1. */
 typedef struct {
@@ -95,9 +105,13 @@ typedef struct {
   float w_mem;      /* weight of the storage LSE objective                              */
   float lr;         /* Adam learning rate; paper 1e-2                                   */
   float beta1, beta2, eps;   /* Adam; 0.9, 0.999, 1e-8                                  */
-  float window_k;   /* bins further than window_k * sigma from mu carry no mass; 6     */
+  float window_k;   /* bins further than window_k * sigma from mu carry no mass; 6.
+                       Other families widen the window to the point whose tail mass
+                       equals the normal's beyond window_k (logistic ~1.9x, Laplace
+                       ~2.4x, Cauchy: the whole horizon for any practical D)       */
   float sigma_min;  /* sigma is clamped to >= sigma_min after each Adam step; 0.05     */
   uint32_t terms;   /* GAUS_* bit mask                                                  */
+  int32_t family;   /* GAUS_GAUSSIAN (default) .. GAUS_CAUCHY                           */
 } gaus_hparams;
 
 /* Discrete verdict on one schedule (Sec. 2.1; App. B.1 for L_com). */
@@ -128,7 +142,8 @@ typedef struct {
 
 /* Paper defaults (Sec. 3.3, App. C.1): tau 1e-2, rho 1e-4, lambda0 1e-6, lr 1e-2;
  * Adam betas (0.9, 0.999), eps 1e-8; alpha = w_res = w_mem = 1; window 6 sigma;
- * sigma_min 0.05; terms = DEP | COM | RES_OBJ.  Returns GAUS_EINVAL on NULL. */
+ * sigma_min 0.05; terms = DEP | COM | RES_OBJ; family GAUSSIAN.  Returns GAUS_EINVAL
+ * on NULL. */
 gaus_status gaus_default_hparams(gaus_hparams *hp);
 
 /* Validate the problem, sort it topologically (Kahn), compute ASAP/ALAP and the

@@ -18,10 +18,14 @@ from .build import LIB as _LIB_PATH
 from .build import build
 
 __all__ = ["build", "lib", "Gaus", "default_hparams", "symbols_declared",
-           "DEP", "COM", "RES_OBJ", "RES_VIOL", "REG_OBJ", "REC", "K", "NT", "STATUS"]
+           "DEP", "COM", "RES_OBJ", "RES_VIOL", "REG_OBJ", "REC", "K", "NT", "STATUS",
+           "GAUSSIAN", "LOGISTIC", "LAPLACE", "CAUCHY"]
 
 DEP, COM, RES_OBJ, RES_VIOL, REG_OBJ, REC = 1, 2, 4, 8, 16, 32
 K, NT = 3, 6
+# CDF families (gaus_hparams.family): the normal, or in its place a scale-matched
+# logistic, Laplace or Cauchy CDF (App. D)
+GAUSSIAN, LOGISTIC, LAPLACE, CAUCHY = 0, 1, 2, 3
 STATUS = {0: "OK", 1: "EINVAL", 2: "ECYCLE", 3: "EHORIZON", 4: "ENOMEM", 5: "ECUDA",
           6: "ENONFINITE", 7: "ENOTCONV"}
 
@@ -47,7 +51,7 @@ class Problem(C.Structure):
 class Hparams(C.Structure):
     _fields_ = [(n, C.c_float) for n in ("tau", "rho", "lambda0", "alpha", "w_res", "w_mem", "lr",
                                          "beta1", "beta2", "eps", "window_k", "sigma_min")] + \
-               [("terms", C.c_uint32)]
+               [("terms", C.c_uint32), ("family", C.c_int32)]
 
 
 class Report(C.Structure):

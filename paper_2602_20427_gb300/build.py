@@ -12,7 +12,9 @@ CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libgaus.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["gaus_api.cu", "gaus_plan.cpp", "gaus_noalloc.cu"]
+# (source, object tag, extra defines): gaus_family.cu once per non-normal CDF family
+SOURCES = [("gaus_api.cu", "api", []), ("gaus_plan.cpp", "plan", []), ("gaus_noalloc.cu", "noalloc", [])] + [
+    ("gaus_family.cu", f"family{k}", [f"-DGAUS_FAMILY_ID={k}", "-DGAUS_FAMILY_KERNELS_ONLY"]) for k in (1, 2, 3)]
 
 
 def _nvcc() -> str:
@@ -37,11 +39,11 @@ def build(force: bool = False, verbose: bool = False) -> str:
     nvcc = _nvcc()
     common = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include")]
     objs, cmds = [], []
-    for src in SOURCES:
-        obj = os.path.join(OUT_DIR, src + f".{os.getpid()}.o")
+    for src, tag, defs in SOURCES:
+        obj = os.path.join(OUT_DIR, f"{tag}.{os.getpid()}.o")
         objs.append(obj)
         extra = ARCH if src.endswith(".cu") else []
-        cmds.append([nvcc, *common, *extra, "-c", os.path.join(CSRC, src), "-o", obj])
+        cmds.append([nvcc, *common, *extra, *defs, "-c", os.path.join(CSRC, src), "-o", obj])
 
     def run(cmd):
         r = subprocess.run(cmd, capture_output=True, text=True)

@@ -13,7 +13,7 @@
 #include "gaus.h"
 #include "gaus_int.cuh"
 #include "gaus_internal.h"
-#include "gaus_kernels.cuh"
+#include "gaus_kernel_set.cuh"
 
 using namespace gaus;
 
@@ -62,7 +62,7 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   A.mu = mu; A.sg = sg;
   A.V = P.V; A.B = P.B; A.D = P.D; A.II = P.II; A.Dh = P.Dh; A.C = P.C; A.RB = ctx->RB; A.G = ctx->G;
   A.W = ctx->W;
-  A.k_win = ctx->hp.window_k; A.alpha = ctx->hp.alpha;
+  A.k_win = ctx->k_win; A.alpha = ctx->hp.alpha;
   A.perm = ctx->d_perm; A.w = ctx->d_w; A.lat = ctx->d_lat;
   A.in_ptr = ctx->d_in_ptr; A.in_src = ctx->d_in_src; A.in_lat = ctx->d_in_lat;
   A.out_ptr = ctx->d_out_ptr; A.out_dst = ctx->d_out_dst;
@@ -75,24 +75,12 @@ IterArgs iter_args(gaus_ctx *ctx, const float *mu, const float *sg) {
   return A;
 }
 
-using EdgeKernel = void (*)(const IterArgs);
-
-EdgeKernel pick_edges(unsigned terms, int II, bool unit) {
-  const bool dep = terms & GAUS_DEP, com = terms & GAUS_COM, rec = (terms & GAUS_REC) && II > 0;
-  if (dep && com && rec) return k_edges<true, true, true, false>;
-  if (dep && rec) return k_edges<true, false, true, false>;
-  if (com && rec) return k_edges<false, true, true, false>;
-  if (rec) return k_edges<false, false, true, false>;
-  if (unit) {
-    if (dep && com) return k_edges<true, true, false, true>;
-    if (dep) return k_edges<true, false, false, true>;
-    if (com) return k_edges<false, true, false, true>;
-    return k_edges<false, false, false, true>;
-  }
-  if (dep && com) return k_edges<true, true, false, false>;
-  if (dep) return k_edges<true, false, false, false>;
-  if (com) return k_edges<false, true, false, false>;
-  return k_edges<false, false, false, false>;
+// The family-dependent kernels of a context's CDF family (the normal's are
+// instantiated here, the others in their own translation units).
+const KernelSet &kernels(int family) {
+  static const KernelSet sets[4] = {make_kernel_set<GAUS_GAUSSIAN>(), kernel_set_logistic(), kernel_set_laplace(),
+                                    kernel_set_cauchy()};
+  return sets[(family >= GAUS_GAUSSIAN && family <= GAUS_CAUCHY) ? family : GAUS_GAUSSIAN];
 }
 
 // Enqueue loss + gradient (adam == false: gradient written to grad_*), or the
@@ -105,7 +93,8 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   const Plan &P = ctx->plan;
   const unsigned on = ctx->hp.terms;
   IterArgs A = iter_args(ctx, mu, sg);
-  k_nodes<<<ctx->nblk, kFwdThreads, ctx->smem_nodes, st>>>(A);
+  const KernelSet &ks = kernels(ctx->hp.family);
+  ks.nodes<<<ctx->nblk, kFwdThreads, ctx->smem_nodes, st>>>(A);
   CK(cudaGetLastError(), "k_nodes launch");
   if (ev) CK(cudaEventRecord(ev[1], st), "event");
   // usage reduction (needs only the node pass) on the side stream, beside the edge pass
@@ -119,7 +108,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
     CK(cudaGetLastError(), "k_reduce launch");
   }
   CK(cudaEventRecord(ctx->ev_join, ctx->side), "join record");
-  EdgeKernel ke = pick_edges(on, P.II, P.unit_lat != 0);
+  EdgeKernel ke = ks.edges[edge_variant(on, P.II, P.unit_lat != 0)];
   ke<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
   CK(cudaGetLastError(), "k_edges launch");
   if (ev) CK(cudaEventRecord(ev[2], st), "event");
@@ -128,10 +117,10 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   if (reg) {
     RA.mu = mu; RA.sg = sg;
     RA.V = P.V; RA.B = P.B; RA.D = P.D; RA.II = P.II; RA.Dh = P.Dh; RA.RB = ctx->RBr; RA.G = ctx->Gr;
-    RA.k_win = ctx->hp.window_k; RA.perm = ctx->d_perm; RA.bits = ctx->d_bits;
+    RA.k_win = ctx->k_win; RA.perm = ctx->d_perm; RA.bits = ctx->d_bits;
     RA.out_ptr = ctx->d_out_ptr; RA.out_dst = ctx->d_out_dst; RA.seg = ctx->d_seg; RA.win = ctx->d_win;
     RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gown = ctx->d_gown; RA.eslot = ctx->d_eslot;
-    k_reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
+    ks.reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_fwd launch");
     k_reduce_reg<<<ctx->Gr * P.Dh, 256, 0, st>>>(ctx->d_rpart, ctx->d_Ureg, P.B, P.Dh, ctx->RBr, ctx->Gr,
                                                  P.nseg);
@@ -155,7 +144,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   k_finalize<<<P.B, 256, ctx->smem_fin, st>>>(F);
   CK(cudaGetLastError(), "k_finalize launch");
   if (reg) {
-    k_reg_bwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rbwd, st>>>(RA);
+    ks.reg_bwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rbwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_bwd launch");
   }
   if (ev) CK(cudaEventRecord(ev[3], st), "event");
@@ -167,7 +156,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   U.eslot = reg ? ctx->d_eslot : nullptr; U.gown = reg ? ctx->d_gown : nullptr;
   U.mu = const_cast<float *>(mu); U.sg = const_cast<float *>(sg);
   U.V = P.V; U.B = P.B; U.D = P.D; U.II = P.II; U.Dh = P.Dh; U.C = P.C; U.RB = ctx->RB; U.G = ctx->G;
-  U.k_win = ctx->hp.window_k; U.W = ctx->W; U.perm = ctx->d_perm; U.cls = ctx->d_cls; U.w = ctx->d_w;
+  U.k_win = ctx->k_win; U.W = ctx->W; U.perm = ctx->d_perm; U.cls = ctx->d_cls; U.w = ctx->d_w;
   U.H = ctx->d_H; U.coef = ctx->d_coef; U.thr = ctx->d_thr;
   U.grad_mu = grad_mu; U.grad_sg = grad_sg;
   U.m_mu = adam ? S->m_mu : nullptr; U.v_mu = adam ? S->v_mu : nullptr;
@@ -176,13 +165,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   U.lr = ctx->hp.lr; U.beta1 = ctx->hp.beta1; U.beta2 = ctx->hp.beta2; U.eps = ctx->hp.eps;
   U.sigma_min = ctx->hp.sigma_min;
   const bool hist = on & (GAUS_RES_OBJ | GAUS_RES_VIOL);
-  if (adam) {
-    if (hist) k_update<true, true><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
-    else k_update<true, false><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
-  } else {
-    if (hist) k_update<false, true><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
-    else k_update<false, false><<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
-  }
+  ks.update[2 * (adam ? 1 : 0) + (hist ? 1 : 0)]<<<ctx->nblk_u, kUpdThreads, 0, st>>>(U);
   CK(cudaGetLastError(), "k_update launch");
   if (ev) CK(cudaEventRecord(ev[4], st), "event");
   return GAUS_OK;
@@ -192,8 +175,9 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
 // a context: set it to the device maximum once per kernel, so that contexts of
 // different sizes can be used side by side (each launch still requests its own size).
 gaus_status set_smem_attrs(gaus_ctx *ctx) {
-  const void *fns[] = {(const void *)k_nodes, (const void *)k_finalize, (const void *)k_reg_fwd,
-                       (const void *)k_reg_bwd, (const void *)k_verify, (const void *)k_legalize_regular_smem};
+  const KernelSet &ks = kernels(ctx->hp.family);
+  const void *fns[] = {(const void *)ks.nodes, (const void *)k_finalize, (const void *)ks.reg_fwd,
+                       (const void *)ks.reg_bwd, (const void *)k_verify, (const void *)k_legalize_regular_smem};
   int dev = 0, optin = 0;
   CK(cudaGetDevice(&dev), "cudaGetDevice");
   CK(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev), "smem opt-in");
@@ -203,7 +187,6 @@ gaus_status set_smem_attrs(gaus_ctx *ctx) {
     CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes),
        "smem attr");
   }
-  (void)ctx;
   return GAUS_OK;
 }
 
@@ -441,6 +424,7 @@ gaus_status gaus_default_hparams(gaus_hparams *hp) {
   hp->window_k = 6.0f;
   hp->sigma_min = 0.05f;
   hp->terms = GAUS_DEP | GAUS_COM | GAUS_RES_OBJ;
+  hp->family = GAUS_GAUSSIAN;
   return GAUS_OK;
 }
 
@@ -456,6 +440,7 @@ gaus_status gaus_create(const gaus_problem *prob, const gaus_hparams *hp, void *
   gaus_ctx *ctx = new (std::nothrow) gaus_ctx();
   if (!ctx) return GAUS_ENOMEM;
   ctx->hp = *hp;
+  ctx->k_win = family_window_k(hp->window_k, hp->family);
   ctx->stream = (cudaStream_t)cuda_stream;
   st = build_ctx(ctx, prob);
   if (st != GAUS_OK) {
@@ -476,8 +461,11 @@ gaus_status gaus_set_hparams(gaus_ctx *ctx, const gaus_hparams *hp) {
     gaus_status st2 = alloc_storage_scratch(ctx);
     if (st2 != GAUS_OK) return st2;
   }
+  const int old_family = ctx->hp.family;
   ctx->hp = *hp;
+  ctx->k_win = family_window_k(hp->window_k, hp->family);
   drop_graph(ctx);
+  if (hp->family != old_family) return set_smem_attrs(ctx);
   return GAUS_OK;
 }
 

@@ -42,6 +42,71 @@ __device__ __forceinline__ float tail_fast(float z) {
   return e * __fdividef(num, den);
 }
 
+// CDF families of the relaxation: the standard normal (Sec. 3.2) and, in its
+// place (App. D), the logistic, Laplace and Cauchy CDFs with the scale matched to
+// sigma -- logistic s = sigma sqrt(3)/pi and Laplace b = sigma/sqrt(2) (equal
+// variance), Cauchy gamma = sigma sqrt(2 ln 2) (equal full width at half
+// maximum).  In z = (x - mu)/sigma each is G(c z) for its standard CDF G, with
+// c = sigma/s, sigma/b or sigma/gamma; every family is symmetric, so one upper
+// tail Q(|z|) = 1 - F(|z|) gives F on both sides.  Fam<k>::tail(z) = Q(|z|),
+// Fam<k>::pdf(z) = F'(z), Fam<k>::cdf(z) = F(z).
+template <int kFam>
+struct Fam;
+
+template <>
+struct Fam<GAUS_GAUSSIAN> {
+  static __device__ __forceinline__ float tail(float z) { return tail_fast(z); }
+  static __device__ __forceinline__ float pdf(float z) { return 0.3989422804014327f * __expf(-0.5f * z * z); }
+  static __device__ __forceinline__ float cdf(float z) { return cdf_fast(z); }
+};
+
+template <>
+struct Fam<GAUS_LOGISTIC> {
+  static constexpr float kC = 1.8137993642342178f;  // pi / sqrt(3)
+  // Q = e / (1 + e) with e = exp(-c |z|): relative accuracy in both tails
+  static __device__ __forceinline__ float tail(float z) {
+    const float e = __expf(-kC * fabsf(z));
+    return __fdividef(e, 1.0f + e);
+  }
+  static __device__ __forceinline__ float pdf(float z) {
+    const float e = __expf(-kC * fabsf(z));
+    const float r = __fdividef(1.0f, 1.0f + e);
+    return kC * e * r * r;
+  }
+  static __device__ __forceinline__ float cdf(float z) {
+    const float q = tail(z);
+    return z <= 0.f ? q : 1.0f - q;
+  }
+};
+
+template <>
+struct Fam<GAUS_LAPLACE> {
+  static constexpr float kC = 1.4142135623730951f;  // sqrt(2)
+  static __device__ __forceinline__ float tail(float z) { return 0.5f * __expf(-kC * fabsf(z)); }
+  static __device__ __forceinline__ float pdf(float z) { return 0.5f * kC * __expf(-kC * fabsf(z)); }
+  static __device__ __forceinline__ float cdf(float z) {
+    const float q = tail(z);
+    return z <= 0.f ? q : 1.0f - q;
+  }
+};
+
+template <>
+struct Fam<GAUS_CAUCHY> {
+  static constexpr float kC = 0.8493218002880191f;   // 1 / sqrt(2 ln 2)
+  static constexpr float kInvPi = 0.3183098861837907f;
+  // Q = atan(1 / (c |z|)) / pi: the complement of 1/2 + atan(y)/pi without the
+  // cancellation in the far tail; 1 / 0 = inf gives Q(0) = 1/2
+  static __device__ __forceinline__ float tail(float z) { return kInvPi * atanf(1.0f / (kC * fabsf(z))); }
+  static __device__ __forceinline__ float pdf(float z) {
+    const float y = kC * z;
+    return __fdividef(kC * kInvPi, 1.0f + y * y);
+  }
+  static __device__ __forceinline__ float cdf(float z) {
+    const float q = tail(z);
+    return z <= 0.f ? q : 1.0f - q;
+  }
+};
+
 // One Adam step of a parameter (torch.optim.Adam semantics): m, v updated in
 // place; inv_bc1 = 1 / (1 - beta1^t), rs_bc2 = 1 / sqrt(1 - beta2^t).
 __device__ __forceinline__ float adam_update(float th, float g, float &m, float &v, float lr, float beta1,

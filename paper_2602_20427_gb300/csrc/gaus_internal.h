@@ -73,12 +73,14 @@ struct Plan {
 // Returns GAUS_OK or an error with a message.
 gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err);
 gaus_status check_hparams(const gaus_hparams *hp, std::string *err);
+float family_window_k(float window_k, int family);
 
 }  // namespace gaus
 
 struct gaus_ctx {
   gaus::Plan plan;
   gaus_hparams hp;
+  float k_win = 6.0f;            // window half-width in sigma for the CDF family (family_window_k)
   cudaStream_t stream = nullptr;
   cudaStream_t side = nullptr;                     // usage reduction beside the edge pass
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;

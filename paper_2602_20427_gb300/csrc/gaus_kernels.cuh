@@ -161,6 +161,7 @@ __device__ __forceinline__ float warp_sum(float x) {
 // A neighbour's windowed CDF C_u(x): 0 below its window, 1 above it, inside it
 // the table value written by k_nodes, or -- for a window the table row cannot
 // hold -- evaluated from its mean and sigma.
+template <int kFam>
 struct Nb {
   const float *row;  // table row of (u, b): [0, C(a), ..., C(b), 1, ...]
   int a, b;          // window points [a, b]
@@ -170,7 +171,7 @@ struct Nb {
   __device__ __forceinline__ float at(int x) const {
     if (x < a) return 0.0f;
     if (x > b) return 1.0f;
-    return tab ? __ldg(row + (x - a + 1)) : cdf_fast(((float)x + 0.5f - mu) * inv);
+    return tab ? __ldg(row + (x - a + 1)) : Fam<kFam>::cdf(((float)x + 0.5f - mu) * inv);
   }
   // a tabled window: the sentinels make the clamped index exact everywhere
   __device__ __forceinline__ float at_tab(int x) const {
@@ -178,7 +179,7 @@ struct Nb {
   }
   // a window the table row cannot hold: direct evaluation
   __device__ __forceinline__ float at_direct(int x) const {
-    return x < a ? 0.0f : (x > b ? 1.0f : cdf_fast(((float)x + 0.5f - mu) * inv));
+    return x < a ? 0.0f : (x > b ? 1.0f : Fam<kFam>::cdf(((float)x + 0.5f - mu) * inv));
   }
   template <bool kTab>
   __device__ __forceinline__ float val(int x) const {
@@ -193,6 +194,7 @@ struct Nb {
 // accuracy) written to its table row for the edge pass, and its bin masses added
 // to the block's histogram as round(w P 2^32) in two exact 16-bit halves.  The
 // span of bins the block touched goes to the partials read by k_reduce.
+template <int kFam>
 __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
   extern __shared__ __align__(16) unsigned char smem[];
   constexpr int T = kFwdThreads;
@@ -251,7 +253,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
     for (int j = 0; j <= nmax; ++j) {
       const bool pt = j < nl;  // point a+j exists
       const float zc = ((float)(a + j) + 0.5f - mu) * inv_s;
-      const float qc = pt ? tail_fast(zc) : 0.f;
+      const float qc = pt ? Fam<kFam>::tail(zc) : 0.f;
       if (tabled && j <= nl) row[j + 1] = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;
       if (j <= nl) hist_add(hlo, hhi, fold_bin(a + j, A.II) * RB + r, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
       zp = zc;
@@ -275,7 +277,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
         const int p = p0 + lane;
         const bool pt = p < l_n;
         const float z = ((float)(l_a + p) + 0.5f - l_mu) * l_inv;
-        const float q = pt ? tail_fast(z) : 0.f;
+        const float q = pt ? Fam<kFam>::tail(z) : 0.f;
         if (l_tabled && p <= l_n) l_row[p + 1] = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
         float zpv = __shfl_up_sync(FULL, z, 1), qpv = __shfl_up_sync(FULL, q, 1);
         if (lane == 0) { zpv = z_carry; qpv = q_carry; }
@@ -331,8 +333,8 @@ __global__ void __launch_bounds__(kFwdThreads) k_nodes(const IterArgs A) {
 // Same terms and formulas as the per-lane path, with the own values evaluated
 // directly.  Returns the warp-reduced sums on every lane: the producer's and the
 // consumer's partials and the edge's forward sums.
-template <bool kDep, bool kCom>
-__device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, const Nb &Vn, float4 &su, float4 &sv,
+template <int kFam, bool kDep, bool kCom>
+__device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb<kFam> &U, const Nb<kFam> &Vn, float4 &su, float4 &sv,
                           float &fd, float &fc, float &fr) {
   const int lane = threadIdx.x & 31;
   float s[11] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // su, sv, fd, fc, fr
@@ -343,9 +345,9 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
     const bool pt = pidx < nv;
     const int t = Vn.a + pidx;
     const float z = ((float)t + 0.5f - Vn.mu) * Vn.inv;
-    const float q = pt ? tail_fast(z) : 0.f;
+    const float q = pt ? Fam<kFam>::tail(z) : 0.f;
     const float Cv = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
-    const float f = pt ? kInvSqrt2Pi * __expf(-0.5f * z * z) : 0.f;
+    const float f = pt ? Fam<kFam>::pdf(z) : 0.f;
     const float zf = z * f;
     if (!back) {
       if (pt) {
@@ -375,9 +377,9 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
     const bool pt = pidx < nu;
     const int x = U.a + pidx;
     const float z = ((float)x + 0.5f - U.mu) * U.inv;
-    const float q = pt ? tail_fast(z) : 0.f;
+    const float q = pt ? Fam<kFam>::tail(z) : 0.f;
     const float Cu = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
-    const float f = pt ? kInvSqrt2Pi * __expf(-0.5f * z * z) : 0.f;
+    const float f = pt ? Fam<kFam>::pdf(z) : 0.f;
     const float zf = z * f;
     if (!back) {
       if (pt) {
@@ -409,17 +411,17 @@ __device__ void coop_edge(const IterArgs &A, bool back, int L, const Nb &U, cons
 // points where a term can be nonzero.  kTab: both rows are in the table (clamped
 // reads against the sentinels); otherwise the values are evaluated directly.
 // All lanes of the warp call it (warp-wide trip counts).
-template <bool kDep, bool kCom, bool kUnit, bool kTab>
-__device__ __forceinline__ void edge_sides(const IterArgs &A, bool fw, bool bk, int L, const Nb &U, const Nb &Vn,
+template <int kFam, bool kDep, bool kCom, bool kUnit, bool kTab>
+__device__ __forceinline__ void edge_sides(const IterArgs &A, bool fw, bool bk, int L, const Nb<kFam> &U, const Nb<kFam> &Vn,
                                            float4 &su, float4 &sv, float &fd, float &fc, float &fr) {
   constexpr unsigned FULL = 0xffffffffu;
   const int nu = U.b - U.a + 1, nv = Vn.b - Vn.a + 1;
   const bool back = bk;
   // own point j of the consumer (v) / producer (u): C from the table, phi, z phi
-  auto own = [&](const Nb &o, int j, float &C, float &f, float &zf) {
+  auto own = [&](const Nb<kFam> &o, int j, float &C, float &f, float &zf) {
     const float z = ((float)(o.a + j) + 0.5f - o.mu) * o.inv;
-    C = kTab ? __ldg(o.row + j + 1) : cdf_fast(z);
-    f = kInvSqrt2Pi * __expf(-0.5f * z * z);
+    C = kTab ? __ldg(o.row + j + 1) : Fam<kFam>::cdf(z);
+    f = Fam<kFam>::pdf(z);
     zf = z * f;
   };
 
@@ -527,7 +529,7 @@ __device__ __forceinline__ void edge_sides(const IterArgs &A, bool fw, bool bk, 
 // directly; an edge with an endpoint window longer than the restart's threshold
 // is done by the whole warp (coop_edge).  kUnit: every edge has latency 1 (no
 // back edges), so C_u(t) is the bin mass's upper value.
-template <bool kDep, bool kCom, bool kRec, bool kUnit>
+template <int kFam, bool kDep, bool kCom, bool kRec, bool kUnit>
 __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   constexpr int T = kFwdThreads;
   constexpr unsigned FULL = 0xffffffffu;
@@ -552,7 +554,7 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
     const float mu_v = present ? A.mu[iv] : 0.f, sg_v = present ? A.sg[iv] : 1.f;
     const unsigned wu = present ? __ldg(A.win + iu) : 0u, wv = present ? __ldg(A.win + iv) : 0u;
     const bool on = present && usable(mu_u, sg_u) && usable(mu_v, sg_v);
-    Nb U, Vn;
+    Nb<kFam> U, Vn;
     U.a = (int)(wu & 0xFFFFu); U.b = (int)(wu >> 16) - 1; U.row = A.tab + iu * A.W;
     Vn.a = (int)(wv & 0xFFFFu); Vn.b = (int)(wv >> 16) - 1; Vn.row = A.tab + iv * A.W;
     U.mu = on ? mu_u : 0.f; U.inv = on ? __frcp_rn(sg_u) : 1.f;
@@ -570,16 +572,16 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
     // ---- per-lane terms: both rows in the table (branch-free reads), then, if any
     // lane needs it, the lanes with a window the table cannot hold ----
     const bool tabbed = U.tab && Vn.tab;
-    edge_sides<kDep, kCom, kUnit, true>(A, fw && tabbed, bk && tabbed, L, U, Vn, su, sv, fd, fc, fr);
+    edge_sides<kFam, kDep, kCom, kUnit, true>(A, fw && tabbed, bk && tabbed, L, U, Vn, su, sv, fd, fc, fr);
     if (__any_sync(FULL, (fw || bk) && !tabbed))
-      edge_sides<kDep, kCom, kUnit, false>(A, fw && !tabbed, bk && !tabbed, L, U, Vn, su, sv, fd, fc, fr);
+      edge_sides<kFam, kDep, kCom, kUnit, false>(A, fw && !tabbed, bk && !tabbed, L, U, Vn, su, sv, fd, fc, fr);
 
     // ---- cooperative pass over this warp's long (edge, restart) items ----
     unsigned longmask = __ballot_sync(FULL, is_long);
     while (longmask) {
       const int src = __ffs(longmask) - 1;
       longmask &= longmask - 1;
-      Nb lu, lv;
+      Nb<kFam> lu, lv;
       lu.a = __shfl_sync(FULL, U.a, src); lu.b = __shfl_sync(FULL, U.b, src);
       lu.tab = __shfl_sync(FULL, (int)U.tab, src) != 0;
       lu.mu = __shfl_sync(FULL, U.mu, src); lu.inv = __shfl_sync(FULL, U.inv, src);
@@ -593,8 +595,8 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
       lv.row = A.tab + ((size_t)l_vc * A.B + l_b) * A.W;
       float4 csu, csv;
       float cfd, cfc, cfr;
-      if (!l_back) coop_edge<kDep, kCom>(A, false, l_L, lu, lv, csu, csv, cfd, cfc, cfr);
-      else coop_edge<true, false>(A, true, l_L, lu, lv, csu, csv, cfd, cfc, cfr);
+      if (!l_back) coop_edge<kFam, kDep, kCom>(A, false, l_L, lu, lv, csu, csv, cfd, cfc, cfr);
+      else coop_edge<kFam, true, false>(A, true, l_L, lu, lv, csu, csv, cfd, cfc, cfr);
       if (lane == src) {
         su = csu; sv = csv;
         fd = cfd; fc = cfc; fr = cfr;
@@ -624,6 +626,7 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   }
 }
 
+#ifndef GAUS_FAMILY_KERNELS_ONLY
 // Usage per (restart, class, bin) from the partials of every block of the class:
 // block = (group g, class c, bin d).  The class's segment spans are staged in
 // shared memory first, so that every thread then issues its partial loads
@@ -658,6 +661,7 @@ __global__ void __launch_bounds__(256) k_reduce(const RedArgs A) {
     A.U[((size_t)b * A.C + c) * Dh + d] = tot;
   }
 }
+#endif  // GAUS_FAMILY_KERNELS_ONLY
 
 // x * 2^-32 of a 2^32 fixed-point value as float, through two 32-bit halves
 // (64-bit integer to floating-point conversions run at the FP64 rate).
@@ -697,6 +701,7 @@ __device__ __forceinline__ long long block_max_ll(long long x, long long *sh) {
   return t;
 }
 
+#ifndef GAUS_FAMILY_KERNELS_ONLY
 // One block (256 threads) per restart.  Usage and storage stay exact 2^32 fixed
 // point (max and ReLU excess in integers); the softmax runs in fp32 on exact
 // differences from the max, and only thread 0 assembles the loss in fp64.
@@ -840,6 +845,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
       A.Hreg[(size_t)b * Dh + t] = A.w_mem * expf(fix_to_float(U[A.C * Dh + t] - s_m[A.C]) / A.tau) / s_s[A.C];
   (void)kInvFixF;
 }
+#endif  // GAUS_FAMILY_KERNELS_ONLY
 
 // Gradient and Adam step (Sec. 3.3).  Warp-item = 32 / RB internal nodes x one
 // restart group (lanes are restarts), taken grid-stride.  Per (node, restart):
@@ -849,7 +855,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
 //   dL/dmu = -(c_dep Ad + Ao + c_rec Ar + Ah) / sigma, same with B.. for sigma,
 // and, in Adam mode, the Adam step with the per-restart bias corrections.
 // Windows longer than the restart's threshold are done by the whole warp.
-template <bool kAdam, bool kHist>
+template <int kFam, bool kAdam, bool kHist>
 __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
   constexpr unsigned FULL = 0xffffffffu;
   const int lane = threadIdx.x & 31, RB = A.RB, npw = 32 / RB, Dh = A.Dh;
@@ -879,7 +885,7 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
         if (j < n) {
           const int t = a + j;
           const float z = ((float)t + 0.5f - mu) * inv_s;
-          const float f = kInvSqrt2Pi * __expf(-0.5f * z * z);
+          const float f = Fam<kFam>::pdf(z);
           const float gh = wv * (Hc[(size_t)fold_bin(t, A.II) * A.B + b] - Hc[(size_t)fold_bin(t + 1, A.II) * A.B + b]);
           Ah += gh * f;
           Bh += gh * z * f;
@@ -901,7 +907,7 @@ __global__ void __launch_bounds__(kUpdThreads) k_update(const UpdArgs A) {
           if (j < l_n) {
             const int t = l_a + j;
             const float z = ((float)t + 0.5f - l_mu) * l_inv;
-            const float f = kInvSqrt2Pi * __expf(-0.5f * z * z);
+            const float f = Fam<kFam>::pdf(z);
             const float gh = l_w * (l_H[(size_t)fold_bin(t, A.II) * A.B + l_b] -
                                     l_H[(size_t)fold_bin(t + 1, A.II) * A.B + l_b]);
             pa += gh * f;

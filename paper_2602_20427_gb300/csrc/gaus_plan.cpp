@@ -28,7 +28,26 @@ gaus_status check_hparams(const gaus_hparams *hp, std::string *err) {
   if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f && hp->beta2 >= 0.0f && hp->beta2 < 1.0f))
     return fail(err, GAUS_EINVAL, "Adam betas must lie in [0, 1)");
   if (hp->terms & ~63u) return fail(err, GAUS_EINVAL, "unknown term bits");
+  if (hp->family < GAUS_GAUSSIAN || hp->family > GAUS_CAUCHY) return fail(err, GAUS_EINVAL, "unknown CDF family");
   return GAUS_OK;
+}
+
+// Window half-width (in sigma) of a family: the point beyond which its tail mass
+// equals the normal's beyond window_k, Q = Phi(-window_k), and at least window_k.  Logistic
+// (s = sigma sqrt(3)/pi): Q = 1 / (1 + e^{k pi/sqrt 3}); Laplace (b = sigma/sqrt 2):
+// Q = e^{-k sqrt 2} / 2; Cauchy (gamma = sigma sqrt(2 ln 2)):
+// Q = atan(gamma / (k sigma)) / pi.  Capped at FLT_MAX (a window of every step).
+float family_window_k(float window_k, int family) {
+  if (family == GAUS_GAUSSIAN) return window_k;
+  const double q = 0.5 * std::erfc((double)window_k / std::sqrt(2.0));
+  const double pi = 3.14159265358979323846;
+  double k = HUGE_VAL;
+  if (q > 0.0) {
+    if (family == GAUS_LOGISTIC) k = std::sqrt(3.0) / pi * std::log(1.0 / q - 1.0);
+    else if (family == GAUS_LAPLACE) k = std::log(0.5 / q) / std::sqrt(2.0);
+    else k = std::sqrt(2.0 * std::log(2.0)) / std::tan(pi * q);
+  }
+  return (std::isfinite(k) && k < 3.0e38) ? (float)std::max(k, (double)window_k) : 3.4028234663852886e38f;
 }
 
 static bool valid_csr(int V, int E, const int32_t *ptr, const int32_t *idx) {

@@ -45,12 +45,26 @@ struct RegArgs {
   float2 *eslot;                     // (E, B) per out-edge slot (CSR position)
 };
 
+// Upper tail Q(|z|) and density of the storage terms: the normal through erfcf
+// and expf, the other families through Fam<kFam>.
+template <int kFam>
+__device__ __forceinline__ float reg_tail(float z) {
+  if constexpr (kFam == GAUS_GAUSSIAN) return 0.5f * erfcf(fabsf(z) * kInvSqrt2);
+  else return Fam<kFam>::tail(z);
+}
+template <int kFam>
+__device__ __forceinline__ float reg_pdf(float z) {
+  if constexpr (kFam == GAUS_GAUSSIAN) return kInvSqrt2Pi * expf(-0.5f * z * z);
+  else return Fam<kFam>::pdf(z);
+}
+
 // C and Q = 1 - C of a windowed CDF at integer point d, both tails accurate.
+template <int kFam>
 __device__ __forceinline__ void cdf_pair(int d, float mu, float inv_s, int a, int b, float &C, float &Q) {
   if (d < a) { C = 0.f; Q = 1.f; return; }
   if (d > b) { C = 1.f; Q = 0.f; return; }
   const float z = ((float)d + 0.5f - mu) * inv_s;
-  const float q = 0.5f * erfcf(fabsf(z) * kInvSqrt2);
+  const float q = reg_tail<kFam>(z);
   C = z <= 0.f ? q : 1.0f - q;
   Q = z <= 0.f ? 1.0f - q : q;
 }
@@ -92,6 +106,7 @@ __device__ __forceinline__ void succ_bounds(const RegArgs &A, int e0, int deg, i
 }
 
 // 1 - M_i(d): 1 when some successor certainly has not started by d.
+template <int kFam>
 __device__ __forceinline__ float one_minus_m(const RegArgs &A, int e0, int deg, int dmax, int b, int d, int Amax) {
   if (deg == 0 || d < Amax) return 1.0f;
   float t = 0.f;
@@ -103,13 +118,14 @@ __device__ __forceinline__ float one_minus_m(const RegArgs &A, int e0, int deg, 
       float C, Q;
       const float mj = (d >= aj && d <= bj) ? A.mu[(size_t)jc * A.B + b] : 0.f;
       const float ij = (d >= aj && d <= bj) ? 1.0f / A.sg[(size_t)jc * A.B + b] : 1.f;
-      cdf_pair(d, mj, ij, aj, bj, C, Q);
+      cdf_pair<kFam>(d, mj, ij, aj, bj, C, Q);
       t = t + (1.0f - t) * Q;
     }
   }
   return t;
 }
 
+template <int kFam>
 __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
   extern __shared__ __align__(16) unsigned char smem_r[];
   constexpr int T = kFwdThreads;
@@ -163,8 +179,8 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
       const bool own = k < n_own;
       const int d = own ? a + k : tail_lo + (k - n_own);
       float Ci = 1.f, Qi;
-      if (on && own) cdf_pair(d, mu, inv_s, a, bw, Ci, Qi);
-      const float L = one_minus_m(A, e0, on ? deg : 0, dmax, b, d, Amax);
+      if (on && own) cdf_pair<kFam>(d, mu, inv_s, a, bw, Ci, Qi);
+      const float L = one_minus_m<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
       if (on && bits != 0.f) hist_add(hlo, hhi, fold_bin(d, A.II) * RB + r, bits * Ci * L);
     }
     __syncwarp();
@@ -183,6 +199,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
   }
 }
 
+#ifndef GAUS_FAMILY_KERNELS_ONLY
 // Reg per (restart, bin) from every block's partials: block = (group, bin),
 // threads = restarts x slices of the segment list, slices combined in order.
 __global__ void __launch_bounds__(256) k_reduce_reg(const long long *rpart, long long *Ureg, int B, int Dh, int RB,
@@ -201,7 +218,9 @@ __global__ void __launch_bounds__(256) k_reduce_reg(const long long *rpart, long
     Ureg[(size_t)b * Dh + d] = tot;
   }
 }
+#endif  // GAUS_FAMILY_KERNELS_ONLY
 
+template <int kFam>
 __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
   extern __shared__ __align__(16) unsigned char smem_rb[];
   constexpr int T = kFwdThreads;
@@ -244,10 +263,10 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
     for (int k = 0; k < nmax; ++k) {
       const bool on = k < n_own;
       const int d = a + k;
-      const float L = one_minus_m(A, e0, on ? deg : 0, dmax, b, d, Amax);
+      const float L = one_minus_m<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
       if (on) {
         const float z = ((float)d + 0.5f - mu) * inv_s;
-        const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
+        const float f = reg_pdf<kFam>(z);
         const float gg = Hs[fold_bin(d, A.II) * RB + r] * bits * L;
         Ao += gg * f;
         Bo += gg * z * f;
@@ -271,7 +290,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
         const bool on = k < cnt;
         const int d = lo + k;
         float Ci = 1.f, Qi;
-        if (on) cdf_pair(d, mu, inv_s, a, bw, Ci, Qi);
+        if (on) cdf_pair<kFam>(d, mu, inv_s, a, bw, Ci, Qi);
         // product of the other successors' CDFs at d
         float prod = 1.f;
         for (int q2 = 0; q2 < dmax; ++q2) {
@@ -283,13 +302,13 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
             const float m2 = in2 ? A.mu[(size_t)kc2 * A.B + b] : 0.f;
             const float i2 = in2 ? 1.0f / A.sg[(size_t)kc2 * A.B + b] : 1.f;
             float C2, Q2;
-            cdf_pair(d, m2, i2, a2, b2, C2, Q2);
+            cdf_pair<kFam>(d, m2, i2, a2, b2, C2, Q2);
             prod *= C2;
           }
         }
         if (on) {
           const float z = ((float)d + 0.5f - mj) * ij;
-          const float f = kInvSqrt2Pi * expf(-0.5f * z * z);
+          const float f = reg_pdf<kFam>(z);
           const float adj = -Hs[fold_bin(d, A.II) * RB + r] * bits * Ci * prod;
           Aj += adj * f;
           Bj += adj * z * f;

@@ -33,6 +33,7 @@ def test_default_hparams_are_the_paper_values(L):
     assert h.lambda0 == pytest.approx(1e-6) and h.lr == pytest.approx(1e-2)
     assert (h.beta1, h.beta2) == (pytest.approx(0.9), pytest.approx(0.999))
     assert h.terms == g.DEP | g.COM | g.RES_OBJ
+    assert h.family == g.GAUSSIAN
     assert L.gaus_default_hparams(None) == 1
 
 
@@ -94,6 +95,8 @@ def test_create_validation_errors_without_gpu(L):
     # hparams out of range
     assert _create(L, pr, g.default_hparams(tau=0.0))[0] == 1
     assert _create(L, pr, g.default_hparams(beta1=1.0))[0] == 1
+    assert _create(L, pr, g.default_hparams(family=4))[0] == 1
+    assert _create(L, pr, g.default_hparams(family=-1))[0] == 1
 
 
 def test_valid_problem_reaches_the_device_check(L):

@@ -27,7 +27,7 @@ def g():
 
 def _ohp(hp, terms):
     return oracle.hparams(tau=hp.tau, rho=hp.rho, alpha=hp.alpha, w_res=hp.w_res, w_mem=hp.w_mem,
-                          terms=terms)
+                          terms=terms, family=hp.family)
 
 
 def check_loss_grad(p, g, B, mu, sg, lam, hp, restarts=None, rtol=1e-4):
