@@ -21,6 +21,9 @@ _SRC = os.path.join(_HERE, "gaus_oracle.c")
 _LIB = os.path.join(_HERE, "_build", "liboracle.so")
 
 DEP, COM, RES_OBJ, RES_VIOL, REG_OBJ, REC = 1, 2, 4, 8, 16, 32
+# not the paper's Eq. dep: sum_e Phi((mu_u + Lat(u) - mu_v) / sqrt(sigma_u^2 + sigma_v^2)),
+# the continuous dependency penalty, a variant with the same multiplier as DEP
+DEP_CF = 64
 K_DEP, K_RES, K_REC, K = 0, 1, 2, 3
 T_RES, T_COM, T_REG, T_VDEP, T_VRES, T_VREC, NT = 0, 1, 2, 3, 4, 5, 6
 # CDF families of the relaxation (Sec. 3.2; App. D)

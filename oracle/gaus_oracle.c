@@ -390,6 +390,30 @@ static void loss_grad_one(const orc_problem *p, const orc_hparams *h, const doub
     gmu[v] = gm;
     gsig[v] = gs;
   }
+  /* ---- continuous dependency penalty (a variant, not the paper's binned Eq. dep):
+   *      X_u + Lat(u) - X_v ~ N(mu_u + Lat(u) - mu_v, sigma_u^2 + sigma_v^2) for the
+   *      independent unrounded normals, so P(X_u + Lat(u) > X_v) = Phi(m / s) ---- */
+  if (on & ORC_DEP_CF) {
+    double vdep = 0.0;
+    for (int32_t e = 0; e < E; ++e) {
+      int32_t u = p->src[e], v = p->dst[e];
+      double m = mu[u] + p->lat[u] - mu[v], s = sqrt(sigma[u] * sigma[u] + sigma[v] * sigma[v]);
+      vdep += orc_Phi(m / s);
+    }
+    terms[ORC_T_VDEP] = vdep;
+    L += lambda[ORC_K_DEP] * vdep + 0.5 * h->rho * vdep * vdep;
+    double coef = lambda[ORC_K_DEP] + h->rho * vdep;
+    for (int32_t e = 0; e < E; ++e) {
+      int32_t u = p->src[e], v = p->dst[e];
+      double m = mu[u] + p->lat[u] - mu[v], s = sqrt(sigma[u] * sigma[u] + sigma[v] * sigma[v]);
+      double f = orc_phi(m / s);
+      /* d Phi(m/s) = f (dm / s - m ds / s^2), ds/dsigma_x = sigma_x / s */
+      gmu[u] += coef * f / s;
+      gmu[v] -= coef * f / s;
+      gsig[u] -= coef * f * m * sigma[u] / (s * s * s);
+      gsig[v] -= coef * f * m * sigma[v] / (s * s * s);
+    }
+  }
   *loss = L;
 #undef PP
   free(P); free(dPm); free(dPs); free(gP); free(Cum); free(gCum); free(U); free(gU);

@@ -24,6 +24,10 @@ extern "C" {
 #define ORC_RES_VIOL 8u   /* ReLU resource violation (App. B.2, Eq. relu)          */
 #define ORC_REG_OBJ 16u   /* LogSumExp of expected live storage (Eq. active, max)  */
 #define ORC_REC     32u   /* expected recurrence violations (App. B.3)             */
+/* NOT the paper's Eq. dep: the continuous dependency penalty
+ * sum_e Phi((mu_u + Lat(u) - mu_v) / sqrt(sigma_u^2 + sigma_v^2)) = sum_e P(X_u + Lat(u) > X_v)
+ * of the unrounded normals, a variant kept apart from ORC_DEP (same multiplier). */
+#define ORC_DEP_CF  64u
 
 /* constraint slots of the augmented Lagrangian (Sec. 3.3) */
 #define ORC_K_DEP 0

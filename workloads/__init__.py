@@ -23,6 +23,7 @@ import numpy as np
 
 # term bits, mirrored from the public header
 DEP, COM, RES_OBJ, RES_VIOL, REG_OBJ, REC = 1, 2, 4, 8, 16, 32
+DEP_CF = 64  # continuous dependency penalty (a variant, not the paper's Eq. dep)
 
 
 @dataclass
