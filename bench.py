@@ -387,13 +387,16 @@ def gpu_arm(args):
 
     # ---- CDF families (App. D): the first 100 fused iterations of the same workload
     # from the same initialization with the normal, logistic, Laplace and Cauchy
-    # relaxations (heavier tails: wider windows)
+    # relaxations (heavier tails: wider windows), and the normal with the continuous
+    # dependency penalty in place of the binned Eq. dep
     families = None
     if not args.no_families and rank == 0:
         families = []
-        for fam, name in ((g.GAUSSIAN, "gaussian"), (g.LOGISTIC, "logistic"), (g.LAPLACE, "laplace"),
-                          (g.CAUCHY, "cauchy")):
-            hpf = g.default_hparams(terms=p.terms, family=fam)
+        cf_terms = (p.terms & ~g.DEP) | g.DEP_CF
+        for fam, name, terms_f in ((g.GAUSSIAN, "gaussian", p.terms), (g.LOGISTIC, "logistic", p.terms),
+                                   (g.LAPLACE, "laplace", p.terms), (g.CAUCHY, "cauchy", p.terms),
+                                   (g.GAUSSIAN, "gaussian, continuous dependency penalty (DEP_CF)", cf_terms)):
+            hpf = g.default_hparams(terms=terms_f, family=fam)
             cf = g.Gaus(p, B, hpf)
             sf = cf.new_state(dmu0, dsg0, hpf.lambda0)
             cf.iterate(10, sf)

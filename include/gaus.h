@@ -51,6 +51,12 @@ typedef enum {
 #define GAUS_RES_VIOL 8u  /* constraint: sum_c sum_t ReLU(usage - R_c), Eq. relu                 */
 #define GAUS_REG_OBJ 16u  /* objective:  w_mem * LSE_tau(expected live storage), Eq. active/max  */
 #define GAUS_REC     32u  /* constraint: expected recurrence violations, App. B.3 (II > 0)       */
+/* constraint, a VARIANT that is not the paper's Eq. dep: the continuous dependency
+ * penalty sum_e Phi((mu_u + Lat(u) - mu_v) / sqrt(sigma_u^2 + sigma_v^2)), i.e.
+ * P(X_u + Lat(u) > X_v) of the unrounded normals, O(1) per edge; it takes the
+ * dependency multiplier and term slot (GAUS_K_DEP, GAUS_T_VDEP).  Excludes GAUS_DEP;
+ * needs family GAUS_GAUSSIAN. */
+#define GAUS_DEP_CF  64u
 
 /* Constraint slots (lambda, multiplier update) and per-restart term values. */
 #define GAUS_K_DEP 0
@@ -151,8 +157,10 @@ gaus_status gaus_default_hparams(gaus_hparams *hp);
  * upload the graph to the device on `cuda_stream` (a cudaStream_t; NULL = the
  * legacy default stream).  Errors: EINVAL (arrays missing or inconsistent,
  * CSR/CSC disagree, duplicate edge, ids out of range, C outside 1..16, D < 1,
- * II < 0, B < 1, sizes beyond the library's limits), ECYCLE, EHORIZON, ENOMEM,
- * ECUDA.  On success *out owns device memory until gaus_destroy. */
+ * II < 0, B < 1, sizes beyond the library's limits; hparams out of range, unknown
+ * term bits or family, GAUS_REC without II, GAUS_DEP with GAUS_DEP_CF, GAUS_DEP_CF
+ * with a family other than the normal), ECYCLE, EHORIZON, ENOMEM, ECUDA.  On
+ * success *out owns device memory until gaus_destroy. */
 gaus_status gaus_create(const gaus_problem *prob, const gaus_hparams *hp, void *cuda_stream,
                         gaus_ctx **out);
 

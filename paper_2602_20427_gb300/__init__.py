@@ -18,10 +18,11 @@ from .build import LIB as _LIB_PATH
 from .build import build
 
 __all__ = ["build", "lib", "Gaus", "default_hparams", "symbols_declared",
-           "DEP", "COM", "RES_OBJ", "RES_VIOL", "REG_OBJ", "REC", "K", "NT", "STATUS",
+           "DEP", "COM", "RES_OBJ", "RES_VIOL", "REG_OBJ", "REC", "DEP_CF", "K", "NT", "STATUS",
            "GAUSSIAN", "LOGISTIC", "LAPLACE", "CAUCHY"]
 
 DEP, COM, RES_OBJ, RES_VIOL, REG_OBJ, REC = 1, 2, 4, 8, 16, 32
+DEP_CF = 64  # continuous dependency penalty: a variant, not the paper's Eq. dep
 K, NT = 3, 6
 # CDF families (gaus_hparams.family): the normal, or in its place a scale-matched
 # logistic, Laplace or Cauchy CDF (App. D)

@@ -111,6 +111,10 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   EdgeKernel ke = ks.edges[edge_variant(on, P.II, P.unit_lat != 0)];
   ke<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
   CK(cudaGetLastError(), "k_edges launch");
+  if (on & GAUS_DEP_CF) {
+    k_dep_cf<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
+    CK(cudaGetLastError(), "k_dep_cf launch");
+  }
   if (ev) CK(cudaEventRecord(ev[2], st), "event");
   const bool reg = on & GAUS_REG_OBJ;
   RegArgs RA;

@@ -295,7 +295,7 @@ __global__ void k_lambda(float *lambda, const float *terms, int B, unsigned on, 
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   const float *T = terms + (size_t)b * GAUS_NT;
-  if (on & GAUS_DEP) lambda[b * GAUS_K + GAUS_K_DEP] += rho * T[GAUS_T_VDEP];
+  if (on & (GAUS_DEP | GAUS_DEP_CF)) lambda[b * GAUS_K + GAUS_K_DEP] += rho * T[GAUS_T_VDEP];
   if (on & GAUS_RES_VIOL) lambda[b * GAUS_K + GAUS_K_RES] += rho * T[GAUS_T_VRES];
   if (on & GAUS_REC) lambda[b * GAUS_K + GAUS_K_REC] += rho * T[GAUS_T_VREC];
 }

@@ -627,6 +627,52 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
 }
 
 #ifndef GAUS_FAMILY_KERNELS_ONLY
+// Continuous dependency penalty (term GAUS_DEP_CF; a variant, not the paper's
+// binned Eq. dep): per forward edge u -> v and restart, Phi(z) with
+// z = m / s, m = mu_u + Lat(u) - mu_v, s = sqrt(sigma_u^2 + sigma_v^2), the
+// probability that X_u + Lat(u) > X_v for the unrounded independent normals.
+// Same blocks and lanes as the edge pass (a chunk of the edge list x a restart
+// group, lane = (edge, restart)), run after it: it overwrites the dependency
+// halves (.x, .y) of the edge's two slots in the edge pass's convention
+// (dV/dmu = -A / sigma, dV/dsigma = -B / sigma of the slot's node) and adds the
+// exact fixed-point sum to the restart's dependency total.
+__global__ void __launch_bounds__(kFwdThreads) k_dep_cf(const IterArgs A) {
+  constexpr int T = kFwdThreads;
+  __shared__ long long s_red[T];
+  const int tid = threadIdx.x, RB = A.RB;
+  const int blk = blockIdx.x, ch = blk / A.G, g = blk % A.G;
+  const int e_begin = ch * A.ce, e_end = min(A.E, e_begin + A.ce);
+  const int r = tid % RB, b = g * RB + r;
+  const bool bok = b < A.B;
+  long long xdep = 0;
+  for (int e = e_begin + tid / RB; bok && e < e_end; e += T / RB) {
+    const int4 ed = __ldg(A.ed + e);
+    const size_t iu = (size_t)ed.x * A.B + b, iv = (size_t)ed.y * A.B + b;
+    const float mu_u = A.mu[iu], sg_u = A.sg[iu], mu_v = A.mu[iv], sg_v = A.sg[iv];
+    float2 pu = make_float2(0.f, 0.f), pv = make_float2(0.f, 0.f);
+    if (usable(mu_u, sg_u) && usable(mu_v, sg_v)) {
+      const float m = mu_u + (float)ed.z - mu_v;
+      const float rs = rsqrtf(sg_u * sg_u + sg_v * sg_v);
+      const float z = m * rs;
+      const float q = tail_fast(z);
+      xdep += to_fix(z <= 0.f ? q : 1.0f - q);
+      const float f = kInvSqrt2Pi * __expf(-0.5f * z * z);
+      // dPhi/dmu_u = f / s, dPhi/dmu_v = -f / s, dPhi/dsigma_x = -f m sigma_x / s^3
+      pu = make_float2(-sg_u * f * rs, f * z * sg_u * sg_u * rs * rs);
+      pv = make_float2(sg_v * f * rs, f * z * sg_v * sg_v * rs * rs);
+    }
+    *reinterpret_cast<float2 *>(&A.eslot4[(size_t)e * A.B + b]) = pu;
+    *reinterpret_cast<float2 *>(&A.eslot4[((size_t)A.nEt + (ed.w >> 1)) * A.B + b]) = pv;
+  }
+  s_red[tid] = xdep;
+  __syncthreads();
+  if (tid < RB && bok) {
+    long long acc = 0;
+    for (int row = 0; row < T / RB; ++row) acc += s_red[row * RB + tid];
+    if (acc) atomicAdd(&A.fwdtot[3 * b], (unsigned long long)acc);
+  }
+}
+
 // Usage per (restart, class, bin) from the partials of every block of the class:
 // block = (group g, class c, bin d).  The class's segment spans are staged in
 // shared memory first, so that every thread then issues its partial loads
@@ -784,7 +830,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   const float vdep = s_f3[0], lcom = s_f3[1], vrec = s_f3[2];
   ex = s_ex;
 
-  const bool on_dep = A.terms & GAUS_DEP, on_com = A.terms & GAUS_COM;
+  const bool on_dep = A.terms & (GAUS_DEP | GAUS_DEP_CF), on_com = A.terms & GAUS_COM;
   const bool on_robj = A.terms & GAUS_RES_OBJ, on_rv = A.terms & GAUS_RES_VIOL;
   const bool on_rec = A.terms & GAUS_REC;
   const float *lam = A.lambda + (size_t)b * GAUS_K;

@@ -27,7 +27,11 @@ gaus_status check_hparams(const gaus_hparams *hp, std::string *err) {
     if (!(x >= 0.0f) || !std::isfinite(x)) return fail(err, GAUS_EINVAL, "rho, alpha, w_res, w_mem, eps, lambda0 must be finite and >= 0");
   if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f && hp->beta2 >= 0.0f && hp->beta2 < 1.0f))
     return fail(err, GAUS_EINVAL, "Adam betas must lie in [0, 1)");
-  if (hp->terms & ~63u) return fail(err, GAUS_EINVAL, "unknown term bits");
+  if (hp->terms & ~127u) return fail(err, GAUS_EINVAL, "unknown term bits");
+  if ((hp->terms & GAUS_DEP) && (hp->terms & GAUS_DEP_CF))
+    return fail(err, GAUS_EINVAL, "GAUS_DEP and GAUS_DEP_CF are two forms of one constraint: choose one");
+  if ((hp->terms & GAUS_DEP_CF) && hp->family != GAUS_GAUSSIAN)
+    return fail(err, GAUS_EINVAL, "GAUS_DEP_CF is the normal's closed form: it needs family GAUS_GAUSSIAN");
   if (hp->family < GAUS_GAUSSIAN || hp->family > GAUS_CAUCHY) return fail(err, GAUS_EINVAL, "unknown CDF family");
   return GAUS_OK;
 }

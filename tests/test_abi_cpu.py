@@ -97,6 +97,10 @@ def test_create_validation_errors_without_gpu(L):
     assert _create(L, pr, g.default_hparams(beta1=1.0))[0] == 1
     assert _create(L, pr, g.default_hparams(family=4))[0] == 1
     assert _create(L, pr, g.default_hparams(family=-1))[0] == 1
+    # the two forms of the dependency constraint exclude each other; the closed form is the normal's
+    assert _create(L, pr, g.default_hparams(terms=g.DEP | g.DEP_CF))[0] == 1
+    assert _create(L, pr, g.default_hparams(terms=g.DEP_CF, family=g.LOGISTIC))[0] == 1
+    assert _create(L, pr, g.default_hparams(terms=128))[0] == 1
 
 
 def test_valid_problem_reaches_the_device_check(L):
