@@ -109,7 +109,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   }
   CK(cudaEventRecord(ctx->ev_join, ctx->side), "join record");
   EdgeKernel ke = ks.edges[edge_variant(on, P.II, P.unit_lat != 0)];
-  ke<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
+  ke<<<ctx->nblk_e, kFwdThreads, 0, st>>>(A);
   CK(cudaGetLastError(), "k_edges launch");
   if (on & GAUS_DEP_CF) {
     k_dep_cf<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
@@ -212,30 +212,46 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     return GAUS_ECUDA;
   }
   ctx->RB = 1;
-  while (ctx->RB < P.B && ctx->RB < 32) ctx->RB <<= 1;
+  while (ctx->RB < P.B && ctx->RB < kMaxRB) ctx->RB <<= 1;
   ctx->G = (P.B + ctx->RB - 1) / ctx->RB;
-  ctx->nblk = P.nseg * ctx->G;
-  // edge pass: about 8 blocks per SM over all restart groups, whole warp passes per block
-  {
-    const int nEt = P.E + P.NB, per_pass = (kFwdThreads / 32) * (32 / ctx->RB);
-    const long want = std::max(1L, (long)8 * nsm / ctx->G);
-    long ce = std::max<long>(per_pass, ((long)nEt + want - 1) / want);
-    ce = (ce + per_pass - 1) / per_pass * per_pass;
-    ctx->ce = (int)ce;
-    ctx->nchunk = std::max(1, (int)((nEt + ce - 1) / ce));
-  }
-  // k_update: one warp-item (32 / RB nodes x one restart group) per warp
-  {
-    const long nwi = ((long)P.V + (32 / ctx->RB) - 1) / (32 / ctx->RB) * ctx->G;
-    ctx->nblk_u = (int)std::max(1L, (nwi + kUpdThreads / 32 - 1) / (kUpdThreads / 32));
-  }
-  ctx->red_blocks = ctx->G * P.C * P.Dh;
   // k_nodes shared memory: the two halves of the usage histogram
   ctx->smem_nodes = 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned);
   if (ctx->smem_nodes > kMaxSmem - 1024) {
     ctx->err = "usage histogram of this horizon/II does not fit in shared memory";
     return GAUS_EINVAL;
   }
+  TRY(set_smem_attrs(ctx));
+  // Grids of the node, edge and update passes sized to one wave: the blocks the
+  // device holds at once (occupancy calculator x SMs), so that no pass ends with a
+  // partly filled second wave.
+  const KernelSet &ks = kernels(ctx->hp.family);
+  auto resident = [&](const void *fn, int threads, size_t smem) {
+    int occ = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fn, threads, smem) != cudaSuccess) {
+      cudaGetLastError();
+      occ = 0;
+    }
+    return std::max(1, occ) * nsm;
+  };
+  plan_segments(P, resident((const void *)ks.nodes, kFwdThreads, ctx->smem_nodes));
+  ctx->nblk = P.nseg * ctx->G;
+  // edge pass: one wave of blocks, the same number per restart group (rows of
+  // edges grid-stride); k_dep_cf: one block per chunk of a warp pass per group
+  {
+    const int nEt = P.E + P.NB, per_pass = (kFwdThreads / 32) * (32 / ctx->RB);
+    const void *ke = (const void *)ks.edges[edge_variant(ctx->hp.terms, P.II, P.unit_lat != 0)];
+    ctx->ce = per_pass;
+    ctx->nchunk = std::max(1, (nEt + per_pass - 1) / per_pass);
+    const int per_group = std::max(1, std::min(ctx->nchunk, resident(ke, kFwdThreads, 0) / ctx->G));
+    ctx->nblk_e = per_group * ctx->G;
+  }
+  // k_update: one warp-item (32 / RB nodes x one restart group) per warp
+  {
+    const long nwi = ((long)P.V + (32 / ctx->RB) - 1) / (32 / ctx->RB) * ctx->G;
+    ctx->nblk_u = (int)std::max(1L, (nwi + kUpdThreads / 32 - 1) / (kUpdThreads / 32));
+    ctx->nblk_u = std::min(ctx->nblk_u, resident((const void *)ks.update[3], kUpdThreads, 0));
+  }
+  ctx->red_blocks = ctx->G * P.C * P.Dh;
   // CDF table rows: up to kTableMax points per (node, restart), a multiple of 4,
   // with the table kept under kTableBytes (longer windows are evaluated directly)
   {
@@ -267,7 +283,6 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     ctx->err = "histogram of this horizon/II does not fit in shared memory";
     return GAUS_EINVAL;
   }
-  TRY(set_smem_attrs(ctx));
   CK(cudaStreamCreateWithFlags(&ctx->side, cudaStreamNonBlocking), "side stream");
   CK(cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming), "event");
   CK(cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming), "event");

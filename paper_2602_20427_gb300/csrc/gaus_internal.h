@@ -18,6 +18,10 @@ constexpr int kThreads = 128;
 constexpr int kUpdThreads = 256;               // threads per k_update block
 constexpr int kGraphUnroll = 10;               // iterations per captured graph
 constexpr int kReduceSpans = 1024;             // segment spans staged per k_reduce pass
+// Restarts per warp row of the node, edge and update passes (a power of two <= 32):
+// lanes = (item, restart), 32 / kMaxRB items per warp.  Fewer restarts per row
+// means each warp's loops run to the longest window of fewer restarts.
+constexpr int kMaxRB = 16;
 constexpr int kTableMax = 32;                    // points per CDF table row, at most
 constexpr size_t kTableBytes = (size_t)64 << 20;  // CDF table size bound
 // Fixed-point scale of the usage histograms: P * 2^32 accumulated in int64.
@@ -72,6 +76,7 @@ struct Plan {
 
 // Returns GAUS_OK or an error with a message.
 gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err);
+void plan_segments(Plan &P, int target_blocks);
 gaus_status check_hparams(const gaus_hparams *hp, std::string *err);
 float family_window_k(float window_k, int family);
 
@@ -86,7 +91,8 @@ struct gaus_ctx {
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   std::string err;
   int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per node pass
-  int ce = 0, nchunk = 0;        // edge pass: edges per block, edge chunks (blocks = nchunk * G)
+  int ce = 0, nchunk = 0;        // k_dep_cf: edges per block, chunks per restart group
+  int nblk_e = 0;                // edge pass blocks (one wave, a multiple of G)
   int nblk_u = 0;                // k_update blocks
   int W = 0;                     // points per CDF table row
   int red_blocks = 0;

@@ -49,7 +49,7 @@ struct IterArgs {
   int32_t *nonfinite;
   unsigned *win;  // (V, B) packed windows a | (b + 1) << 16, written by k_nodes
   float *tab;     // (V, B, W) CDF values at the window points, written by k_nodes
-  const int4 *ed; // edge list of the edge pass (nEt = E + NB edges, ce per block)
+  const int4 *ed; // edge list of the edge pass (nEt = E + NB edges; k_dep_cf: ce per block)
   int nEt, ce, E;
   unsigned long long *wstat;  // (B, 2) window points / valid items of this iteration
   float4 *eslot4; // per-edge partials [side][position][restart]: producer side at
@@ -535,16 +535,17 @@ __global__ void __launch_bounds__(kFwdThreads, 4) k_edges(const IterArgs A) {
   constexpr unsigned FULL = 0xffffffffu;
   __shared__ long long s_red[3 * T];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, RB = A.RB, epw = 32 / RB;
-  const int blk = blockIdx.x, ch = blk / A.G, g = blk % A.G;
-  const int e_begin = ch * A.ce, e_end = min(A.nEt, e_begin + A.ce);
+  // block = one restart group; its warps take rows of epw edges grid-stride over
+  // the group's blocks, so each warp's rows are spread over the whole edge list
+  const int g = blockIdx.x % A.G, nbg = gridDim.x / A.G;
   const int r = tid % RB, b = g * RB + r;
   const bool bok = b < A.B;
   const int thr = bok ? long_threshold(A.wstat, b) : A.W;
   long long xdep = 0, xcom = 0, xrec = 0;  // forward sums, exact (order-free) fixed point
-  const int per_pass = (T / 32) * epw;
-  for (int e0 = e_begin + warp * epw; e0 < e_end; e0 += per_pass) {
-    const int e = e0 + lane / RB;
-    const bool present = bok && e < e_end;
+  const int nrows = (A.nEt + epw - 1) / epw, rstride = nbg * (T / 32);
+  for (int row = (blockIdx.x / A.G) * (T / 32) + warp; row < nrows; row += rstride) {
+    const int e = row * epw + lane / RB;
+    const bool present = bok && e < A.nEt;
     const int4 ed = present ? __ldg(A.ed + e) : make_int4(0, 0, 0, 0);
     const int uc = ed.x, vc = ed.y, L = kUnit ? 1 : ed.z;
     const bool back = (ed.w & 1) != 0;

@@ -64,6 +64,45 @@ static bool valid_csr(int V, int E, const int32_t *ptr, const int32_t *idx) {
   return true;
 }
 
+// Segments: contiguous internal nodes of one class, sized so that the per-node
+// kernels launch about target_blocks blocks over all restart groups.
+void plan_segments(Plan &P, int target_blocks) {
+  const int V = P.V, C = P.C;
+  P.seg.clear();
+  int RB = 1;
+  while (RB < P.B && RB < kMaxRB) RB <<= 1;
+  int G = (P.B + RB - 1) / RB;
+  long want = std::max(1L, (long)target_blocks / G);
+  int seglen = (int)std::max(1L, ((long)V + want - 1) / want);
+  // at least one row of nodes per block pass; and few enough nodes that the
+  // 16-bit halves of the shared-memory usage histogram cannot overflow:
+  // segment length * max demand * ceil(D / Dh) * 2^16 < 2^32
+  seglen = std::max(seglen, std::max(1, kFwdThreads / RB));
+  int maxw = 1;
+  for (int v = 0; v < V; ++v) maxw = std::max(maxw, P.c_dem[v]);
+  const long folds = (P.D + P.Dh - 1) / P.Dh;
+  const long cap = std::max(1L, 32768L / ((long)maxw * folds));
+  seglen = (int)std::max(1L, std::min<long>(seglen, cap));
+  // whole rows of the block: warps then claim equal shares
+  const int rows = kFwdThreads / RB;
+  if (seglen > rows) seglen = (seglen + rows - 1) / rows * rows;
+  if (seglen > cap) seglen = (int)std::max(1L, cap >= rows ? cap - cap % rows : cap);
+  P.cls_seg_ptr.assign(C + 1, 0);
+  int i0 = 0;
+  for (int c = 0; c < C; ++c) {
+    int i1 = i0;
+    while (i1 < V && P.cls[i1] == c) ++i1;
+    for (int s = i0; s < i1; s += seglen) {
+      P.seg.push_back(s);
+      P.seg.push_back(std::min(i1, s + seglen));
+      P.seg.push_back(c);
+    }
+    P.cls_seg_ptr[c + 1] = (int)P.seg.size() / 3;
+    i0 = i1;
+  }
+  P.nseg = (int)P.seg.size() / 3;
+}
+
 gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err) {
   if (!p) return fail(err, GAUS_EINVAL, "problem is NULL");
   const int V = p->V, E = p->E, C = p->C, NB = p->n_back;
@@ -316,40 +355,7 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
     P.lq_ptr[q + 1] = (int32_t)P.lq_src.size();
   }
 
-  // segments: contiguous internal nodes of one class, sized so that the per-node
-  // kernels launch about target_blocks blocks over all restart groups
-  int RB = 1;
-  while (RB < p->B && RB < 32) RB <<= 1;
-  int G = (p->B + RB - 1) / RB;
-  long want = std::max(1L, (long)target_blocks / G);
-  int seglen = (int)std::max(1L, ((long)V + want - 1) / want);
-  // at least one row of nodes per block pass; and few enough nodes that the
-  // 16-bit halves of the shared-memory usage histogram cannot overflow:
-  // segment length * max demand * ceil(D / Dh) * 2^16 < 2^32
-  seglen = std::max(seglen, std::max(1, kFwdThreads / RB));
-  int maxw = 1;
-  for (int v = 0; v < V; ++v) maxw = std::max(maxw, P.c_dem[v]);
-  const long folds = (p->D + P.Dh - 1) / P.Dh;
-  const long cap = std::max(1L, 32768L / ((long)maxw * folds));
-  seglen = (int)std::max(1L, std::min<long>(seglen, cap));
-  // whole rows of the block: warps then claim equal shares
-  const int rows = kFwdThreads / RB;
-  if (seglen > rows) seglen = (seglen + rows - 1) / rows * rows;
-  if (seglen > cap) seglen = (int)std::max(1L, cap >= rows ? cap - cap % rows : cap);
-  P.cls_seg_ptr.assign(C + 1, 0);
-  int i0 = 0;
-  for (int c = 0; c < C; ++c) {
-    int i1 = i0;
-    while (i1 < V && P.cls[i1] == c) ++i1;
-    for (int s = i0; s < i1; s += seglen) {
-      P.seg.push_back(s);
-      P.seg.push_back(std::min(i1, s + seglen));
-      P.seg.push_back(c);
-    }
-    P.cls_seg_ptr[c + 1] = (int)P.seg.size() / 3;
-    i0 = i1;
-  }
-  P.nseg = (int)P.seg.size() / 3;
+  plan_segments(P, target_blocks);
   return GAUS_OK;
 }
 
