@@ -109,8 +109,21 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   }
   CK(cudaEventRecord(ctx->ev_join, ctx->side), "join record");
   EdgeKernel ke = ks.edges[edge_variant(on, P.II, P.unit_lat != 0)];
-  ke<<<ctx->nblk_e, kFwdThreads, 0, st>>>(A);
-  CK(cudaGetLastError(), "k_edges launch");
+  {
+    // the edge pass at the device's greatest priority, so that its blocks start
+    // ahead of the usage reduction's (which has until the finalize to finish)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)ctx->nblk_e);
+    cfg.blockDim = dim3(kFwdThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributePriority;
+    at[0].val.priority = ctx->prio_hi;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    CK(cudaLaunchKernelEx(&cfg, ke, A), "k_edges launch");
+  }
   if (on & GAUS_DEP_CF) {
     k_dep_cf<<<ctx->nchunk * ctx->G, kFwdThreads, 0, st>>>(A);
     CK(cudaGetLastError(), "k_dep_cf launch");
@@ -284,6 +297,11 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     return GAUS_EINVAL;
   }
   CK(cudaStreamCreateWithFlags(&ctx->side, cudaStreamNonBlocking), "side stream");
+  {
+    int least = 0, greatest = 0;
+    CK(cudaDeviceGetStreamPriorityRange(&least, &greatest), "priority range");
+    ctx->prio_hi = greatest;
+  }
   CK(cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming), "event");
   CK(cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming), "event");
 
@@ -410,7 +428,7 @@ gaus_status capture_iterations(gaus_ctx *ctx, const gaus_state *S, int iters, cu
     return st;
   }
   if (e != cudaSuccess) return cuda_fail(ctx, e, "end capture");
-  e = cudaGraphInstantiate(out, graph, 0);
+  e = cudaGraphInstantiate(out, graph, cudaGraphInstantiateFlagUseNodePriority);
   cudaGraphDestroy(graph);
   if (e != cudaSuccess) {
     *out = nullptr;

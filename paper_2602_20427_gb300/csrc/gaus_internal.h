@@ -89,6 +89,7 @@ struct gaus_ctx {
   cudaStream_t stream = nullptr;
   cudaStream_t side = nullptr;                     // usage reduction beside the edge pass
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  int prio_hi = 0;                                 // greatest stream priority (the edge pass)
   std::string err;
   int RB = 32, G = 1, nblk = 0;  // restarts per block row, restart groups, blocks per node pass
   int ce = 0, nchunk = 0;        // k_dep_cf: edges per block, chunks per restart group

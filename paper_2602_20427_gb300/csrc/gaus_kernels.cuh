@@ -123,11 +123,13 @@ __device__ __forceinline__ long long to_fix(float x) {
 // twice the restart's mean window (over all its nodes, this iteration) plus 4,
 // at least 8.  It depends on restart b alone, so the
 // split -- and with it every rounding -- does not depend on the other restarts.
-__device__ __forceinline__ int long_threshold(const unsigned long long *ws, int b) {
-  const unsigned long long c = ws[2 * b + 1];
+__device__ __forceinline__ int threshold_of(unsigned long long sum, unsigned long long c) {
   if (c == 0) return 8;
-  const int mean = (int)(ws[2 * b] / c);
+  const int mean = (int)(sum / c);
   return min(1 << 20, max(8, 2 * mean + 4));
+}
+__device__ __forceinline__ int long_threshold(const unsigned long long *ws, int b) {
+  return threshold_of(ws[2 * b], ws[2 * b + 1]);
 }
 
 // Mean window length (points) of restart b over the nodes s0..s1 of a segment,
@@ -760,6 +762,18 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   const int b = blockIdx.x, tid = threadIdx.x, Dh = A.Dh;
   const float kInvFixF = 2.3283064365386963e-10f;
 
+  // the restart's scalars, all loaded before any store (the stores below could
+  // alias them): forward sums of the edge pass, multipliers, window statistics,
+  // nonfinite flag, Adam step
+  __shared__ float s_f3[3];
+  __shared__ unsigned long long s_fw[3], s_ws[2];
+  __shared__ float s_lam[GAUS_K];
+  __shared__ int s_bad, s_step;
+  if (tid < 3) s_fw[tid] = A.fwdtot[3 * b + tid];
+  if (tid >= 32 && tid < 32 + GAUS_K) s_lam[tid - 32] = A.lambda[(size_t)b * GAUS_K + tid - 32];
+  if (tid >= 64 && tid < 66) s_ws[tid - 64] = A.wstat[2 * b + tid - 64];
+  if (tid == 96) s_bad = A.nonfinite[b];
+  if (tid == 128) s_step = A.step ? A.step[b] : 0;
   for (int i = tid; i < A.C * Dh; i += 256) U[i] = A.Ug[(size_t)b * A.C * Dh + i];
   if (A.Ureg)
     for (int t = tid; t < Dh; t += 256) U[A.C * Dh + t] = A.Ureg[(size_t)b * Dh + t];
@@ -772,14 +786,6 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   }
   __syncthreads();
 
-  // forward sums of the edge terms (per-restart totals of the edge pass)
-  __shared__ float s_f3[3];
-  if (tid == 0) {
-    for (int k = 0; k < 3; ++k) {
-      s_f3[k] = (float)((double)(long long)A.fwdtot[3 * b + k] * kInvFix);
-      A.fwdtot[3 * b + k] = 0ull;
-    }
-  }
 
   // per class: the max (Eq. max, max shifted out) and the exact ReLU excess over
   // finite limits (Eq. relu) in one pass, then the sums of exp; every class is
@@ -803,6 +809,10 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   for (int o = 16; o > 0; o >>= 1) ex += __shfl_xor_sync(0xffffffffu, ex, o);
   if (lane == 0) s_wx[wid] = ex;
   __syncthreads();
+  if (tid < 3) {
+    s_f3[tid] = (float)((double)(long long)s_fw[tid] * kInvFix);
+    A.fwdtot[3 * b + tid] = 0ull;
+  }
   if (tid < nh) {
     long long m = LLONG_MIN;
     for (int w = 0; w < 8; ++w) m = max(m, s_wm[tid][w]);
@@ -834,7 +844,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   const bool on_dep = A.terms & (GAUS_DEP | GAUS_DEP_CF), on_com = A.terms & GAUS_COM;
   const bool on_robj = A.terms & GAUS_RES_OBJ, on_rv = A.terms & GAUS_RES_VIOL;
   const bool on_rec = A.terms & GAUS_REC;
-  const float *lam = A.lambda + (size_t)b * GAUS_K;
+  const float *lam = s_lam;
   const double vres = (double)ex * kInvFix;
   const float c_res = on_rv ? (float)((double)lam[GAUS_K_RES] + (double)A.rho * vres) : 0.f;
   if (tid == 0) {
@@ -859,19 +869,19 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
     A.loss[b] = (float)L;
     A.coef[b * 4 + 0] = on_dep ? (float)((double)lam[GAUS_K_DEP] + (double)A.rho * Vk[0]) : 0.f;
     A.coef[b * 4 + 1] = on_rec ? (float)((double)lam[GAUS_K_REC] + (double)A.rho * Vk[2]) : 0.f;
-    A.thr[b] = long_threshold(A.wstat, b);
+    A.thr[b] = threshold_of(s_ws[0], s_ws[1]);
     A.wstat[2 * b] = 0ull;
     A.wstat[2 * b + 1] = 0ull;
-    const int bad = A.nonfinite[b];
+    const int bad = s_bad;
     if (A.status) A.status[b] = bad ? GAUS_ENONFINITE : GAUS_OK;
     A.nonfinite[b] = 0;
     if (A.update_lambda) {
       float *lw = A.lambda + (size_t)b * GAUS_K;
       for (int k = 0; k < 3; ++k)
-        if (act[k]) lw[k] = (float)((double)lw[k] + (double)A.rho * Vk[k]);
+        if (act[k]) lw[k] = (float)((double)lam[k] + (double)A.rho * Vk[k]);
     }
     if (A.step) {
-      const int st = A.step[b] + 1;
+      const int st = s_step + 1;
       A.step[b] = st;
       // Adam bias corrections of this step (torch.optim.Adam): 1 / (1 - beta1^t)
       // and 1 / sqrt(1 - beta2^t)
