@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--no-solver", action="store_true", help="skip the complete-solver runs (gaus_solve)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-families", action="store_true", help="skip the CDF-family timings")
+    ap.add_argument("--profile-range", action="store_true",
+                    help="bracket the timed steps with cudaProfilerStart/Stop (for ncu --profile-from-start off)")
     return ap.parse_args()
 
 
@@ -240,12 +242,16 @@ def gpu_arm(args):
         sampler.start()
         time.sleep(0.5)
     wall0 = time.perf_counter()
+    if args.profile_range:
+        torch.cuda.profiler.start()              # ncu --profile-from-start off: the timed steps only
     for k in range(args.steps):
         flush.fill_(k & 255)                     # L2 flush between steps (outside the events)
         evs[k][0].record()
         step()
         evs[k][1].record()
     torch.cuda.synchronize()
+    if args.profile_range:
+        torch.cuda.profiler.stop()
     wall = time.perf_counter() - wall0
     clocks = sampler.stop() if sampler else None
     step_ms = [a.elapsed_time(b) for a, b in evs]
