@@ -202,8 +202,10 @@ def gpu_arm(args):
     lstat = torch.empty(B, dtype=torch.int32, device="cuda")
     rep = torch.empty(B * 200, dtype=torch.uint8, device="cuda")
     reg = bool(p.terms & W.REG_OBJ)
-    launches_per_iter = 5 + (3 if reg else 0)   # windows, fwd, [reg fwd, reg reduce], reduce, finalize, [reg bwd], update
-    launches_per_step = iters * launches_per_iter + (iters // period) * 2
+    # per iteration: k_nodes, k_edges, k_reduce, k_finalize, k_update [+ k_reg_fwd, k_reduce_reg,
+    # k_reg_bwd]; per period: the legalization kernel and the verifier's two passes
+    launches_per_iter = 5 + (3 if reg else 0)
+    launches_per_step = iters * launches_per_iter + (iters // period) * 3
 
     def init_state(mu_src, sg_src):
         st["mu"].copy_(mu_src, non_blocking=True)

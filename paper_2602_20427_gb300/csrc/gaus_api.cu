@@ -194,7 +194,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
 gaus_status set_smem_attrs(gaus_ctx *ctx) {
   const KernelSet &ks = kernels(ctx->hp.family);
   const void *fns[] = {(const void *)ks.nodes, (const void *)k_finalize, (const void *)ks.reg_fwd,
-                       (const void *)ks.reg_bwd, (const void *)k_verify, (const void *)k_legalize_regular_smem};
+                       (const void *)ks.reg_bwd, (const void *)k_verify_fin, (const void *)k_legalize_regular_smem};
   int dev = 0, optin = 0;
   CK(cudaGetDevice(&dev), "cudaGetDevice");
   CK(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev), "smem opt-in");
@@ -360,6 +360,13 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   if (ctx->hp.terms & GAUS_REG_OBJ) TRY(alloc_storage_scratch(ctx));
   TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
   TRY(scratch(ctx, &ctx->d_fwdtot, (size_t)P.B * 3));
+  // verifier: per-restart counts, usage counts and storage difference arrays
+  ctx->vacc_words = (size_t)P.B * (4 + (size_t)P.C * P.Dh + (size_t)P.D + 1);
+  TRY(scratch(ctx, &ctx->d_vacc, ctx->vacc_words));
+  ctx->RBv = 1;
+  while (ctx->RBv < P.B && ctx->RBv < 32) ctx->RBv <<= 1;
+  ctx->Gv = (P.B + ctx->RBv - 1) / ctx->RBv;
+  ctx->nblk_v = std::max(1, resident((const void *)k_verify_scan, 256, 0) / ctx->Gv) * ctx->Gv;
   TRY(scratch(ctx, &ctx->d_eslot4, 2 * ((size_t)P.E + P.NB) * P.B));
   TRY(scratch(ctx, &ctx->d_win, VB));
   TRY(scratch(ctx, &ctx->d_tab, VB * ctx->W));
@@ -637,8 +644,15 @@ gaus_status gaus_verify(gaus_ctx *ctx, const int32_t *sched, gaus_report *rep) {
   A.dem = ctx->d_c_dem; A.bits = ctx->d_c_bits;
   A.b_src = ctx->d_b_src; A.b_dst = ctx->d_b_dst; A.b_dist = ctx->d_b_dist;
   A.succ_ptr = ctx->d_csucc_ptr; A.succ_dst = ctx->d_csucc_dst; A.limit = ctx->d_limit;
-  k_verify<<<P.B, 256, ctx->smem_ver, ctx->stream>>>(A);
-  CK(cudaGetLastError(), "k_verify launch");
+  A.RB = ctx->RBv; A.G = ctx->Gv;
+  A.vacc = ctx->d_vacc;
+  A.vcnt = A.vacc + (size_t)P.B * 4;
+  A.vdiff = A.vcnt + (size_t)P.B * P.C * P.Dh;
+  CK(cudaMemsetAsync(ctx->d_vacc, 0, ctx->vacc_words * sizeof(unsigned long long), ctx->stream), "verify memset");
+  k_verify_scan<<<ctx->nblk_v, 256, 0, ctx->stream>>>(A);
+  CK(cudaGetLastError(), "k_verify_scan launch");
+  k_verify_fin<<<P.B, 256, ctx->smem_ver, ctx->stream>>>(A);
+  CK(cudaGetLastError(), "k_verify_fin launch");
   return GAUS_OK;
 }
 

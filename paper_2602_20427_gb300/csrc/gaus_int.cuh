@@ -168,82 +168,103 @@ struct VerArgs {
   const int32_t *s;
   gaus_report *rep;
   int V, E, NB, B, C, D, II, Dh;
+  int RB, G;  // restarts per warp row, restart groups (pass 1)
   const int32_t *e_src, *e_dst, *lat, *cls, *dem, *bits;
   const int32_t *b_src, *b_dst, *b_dist;
   const int32_t *succ_ptr, *succ_dst;
   const float *limit;
+  // zeroed before pass 1: per restart the counts (dep, com, lat, rec), the usage
+  // counts (B, C, Dh) and the storage difference array (B, D + 1), exact int64
+  unsigned long long *vacc, *vcnt, *vdiff;
 };
 
-__device__ __forceinline__ long long block_sum_ll(long long x, long long *buf) {
-  const int tid = threadIdx.x;
-  buf[tid] = x;
+// Verifier pass 1 (Sec. 2.1 definitions; L_com of App. B.1): items are the edges,
+// the nodes and the back edges; lanes are restarts (32 / RB items per warp, rows
+// grid-stride over the blocks of the restart group), so every read of a schedule
+// is coalesced over restarts.  Per (item, restart): the dependency / latency /
+// recurrence violation and L_com counts in registers, then per restart in shared
+// memory and once per block in global memory; usage counts and the storage
+// difference array as global integer atomics (exact, order-free).
+__global__ void __launch_bounds__(256) k_verify_scan(const VerArgs A) {
+  __shared__ unsigned long long s_acc[4][32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, RB = A.RB, ipw = 32 / RB;
+  const int g = blockIdx.x % A.G, nbg = gridDim.x / A.G;
+  const int r = lane % RB, b = g * RB + r;
+  const bool bok = b < A.B;
+  if (tid < 4 * 32) s_acc[tid / 32][tid % 32] = 0ull;
   __syncthreads();
-  for (int s = 128; s > 0; s >>= 1) {
-    if (tid < s) buf[tid] += buf[tid + s];
-    __syncthreads();
+  const int nback = A.II > 0 ? A.NB : 0;
+  const long long nitems = (long long)A.E + A.V + nback;
+  const long long rows = (nitems + ipw - 1) / ipw;
+  long long ndep = 0, lcom = 0, nlat = 0, nrec = 0;
+  for (long long row = (long long)(blockIdx.x / A.G) * 8 + warp; row < rows; row += (long long)nbg * 8) {
+    const long long it = row * ipw + lane / RB;
+    if (!bok || it >= nitems) continue;
+    if (it < A.E) {
+      const int e = (int)it, u = A.e_src[e], v = A.e_dst[e];
+      const int su = A.s[(size_t)u * A.B + b], sv = A.s[(size_t)v * A.B + b];
+      if ((long long)sv < (long long)su + A.lat[u]) ++ndep;
+      lcom += (long long)sv - su;
+    } else if (it < (long long)A.E + A.V) {
+      const int v = (int)(it - A.E);
+      const int sv = A.s[(size_t)v * A.B + b];
+      if (sv < 0 || (long long)sv + A.lat[v] > A.D) ++nlat;
+      if (sv >= 0 && sv < A.D) {
+        const int t = A.II > 0 ? sv % A.II : sv;
+        atomicAdd(&A.vcnt[((size_t)b * A.C + A.cls[v]) * A.Dh + t], (unsigned long long)(long long)A.dem[v]);
+      }
+      // Mem: live on [s_v, max over successors of s_w) (leaves: until D), within [0, D)
+      long long last = A.D;
+      if (A.succ_ptr[v + 1] > A.succ_ptr[v]) {
+        last = LLONG_MIN;
+        for (int q = A.succ_ptr[v]; q < A.succ_ptr[v + 1]; ++q)
+          last = max(last, (long long)A.s[(size_t)A.succ_dst[q] * A.B + b]);
+      }
+      const long long lo = max((long long)sv, 0LL), hi = min(last, (long long)A.D);
+      if (lo < hi && A.bits[v] != 0) {
+        unsigned long long *row_d = A.vdiff + (size_t)b * (A.D + 1);
+        atomicAdd(&row_d[lo], (unsigned long long)(long long)A.bits[v]);
+        atomicAdd(&row_d[hi], (unsigned long long)(-(long long)A.bits[v]));
+      }
+    } else {
+      const int q = (int)(it - A.E - A.V), j = A.b_src[q], i = A.b_dst[q];
+      if ((long long)A.s[(size_t)i * A.B + b] + (long long)A.b_dist[q] * A.II <
+          (long long)A.s[(size_t)j * A.B + b] + A.lat[j])
+        ++nrec;
+    }
   }
-  const long long r = buf[0];
+  if (bok) {
+    if (ndep) atomicAdd(&s_acc[0][r], (unsigned long long)ndep);
+    if (lcom) atomicAdd(&s_acc[1][r], (unsigned long long)lcom);
+    if (nlat) atomicAdd(&s_acc[2][r], (unsigned long long)nlat);
+    if (nrec) atomicAdd(&s_acc[3][r], (unsigned long long)nrec);
+  }
   __syncthreads();
-  return r;
+  if (tid < 4 * RB) {
+    const int k = tid / RB, rr = tid % RB, bb = g * RB + rr;
+    if (bb < A.B && s_acc[k][rr]) atomicAdd(&A.vacc[(size_t)bb * 4 + k], s_acc[k][rr]);
+  }
 }
 
-// One block (256 threads) per restart.  Shared: usage counts C*Dh (int64),
-// storage difference array D+1 (int64), folded storage Dh (int64).
-__global__ void __launch_bounds__(256) k_verify(const VerArgs A) {
+// Verifier pass 2: one block (256 threads) per restart assembles its report from
+// pass 1's counts: per-class peaks and limit violations, the storage scan (Mem and
+// its fold modulo II).
+__global__ void __launch_bounds__(256) k_verify_fin(const VerArgs A) {
   extern __shared__ __align__(16) unsigned char smem_v[];
   long long *cnt = reinterpret_cast<long long *>(smem_v);
   long long *diff = cnt + (size_t)A.C * A.Dh;
   long long *mm = diff + (A.D + 1);
-  __shared__ long long buf[256];
   const int b = blockIdx.x, tid = threadIdx.x;
-  for (int i = tid; i < A.C * A.Dh; i += 256) cnt[i] = 0;
-  for (int i = tid; i <= A.D; i += 256) diff[i] = 0;
+  for (int i = tid; i < A.C * A.Dh; i += 256) cnt[i] = (long long)A.vcnt[(size_t)b * A.C * A.Dh + i];
+  for (int i = tid; i <= A.D; i += 256) diff[i] = (long long)A.vdiff[(size_t)b * (A.D + 1) + i];
   for (int i = tid; i < A.Dh; i += 256) mm[i] = 0;
   __syncthreads();
-  auto S = [&](int v) { return A.s[(size_t)v * A.B + b]; };
-  long long ndep = 0, lcom = 0, nlat = 0, nrec = 0;
-  for (int e = tid; e < A.E; e += 256) {
-    const int u = A.e_src[e], v = A.e_dst[e];
-    const int su = S(u), sv = S(v);
-    if ((long long)sv < (long long)su + A.lat[u]) ++ndep;
-    lcom += (long long)sv - su;
-  }
-  for (int v = tid; v < A.V; v += 256) {
-    const int sv = S(v);
-    if (sv < 0 || (long long)sv + A.lat[v] > A.D) ++nlat;
-    if (sv >= 0 && sv < A.D) {
-      const int t = A.II > 0 ? sv % A.II : sv;
-      atomicAdd(reinterpret_cast<unsigned long long *>(&cnt[A.cls[v] * A.Dh + t]),
-                (unsigned long long)(long long)A.dem[v]);
-    }
-    // Mem: live on [s_v, max over successors of s_w) (leaves: until D), within [0, D)
-    long long last = A.D;
-    if (A.succ_ptr[v + 1] > A.succ_ptr[v]) {
-      last = LLONG_MIN;
-      for (int q = A.succ_ptr[v]; q < A.succ_ptr[v + 1]; ++q) last = max(last, (long long)S(A.succ_dst[q]));
-    }
-    const long long lo = max((long long)sv, 0LL), hi = min(last, (long long)A.D);
-    if (lo < hi && A.bits[v] != 0) {
-      atomicAdd(reinterpret_cast<unsigned long long *>(&diff[lo]), (unsigned long long)(long long)A.bits[v]);
-      atomicAdd(reinterpret_cast<unsigned long long *>(&diff[hi]), (unsigned long long)(-(long long)A.bits[v]));
-    }
-  }
-  if (A.II > 0)
-    for (int q = tid; q < A.NB; q += 256) {
-      const int j = A.b_src[q], i = A.b_dst[q];
-      if ((long long)S(i) + (long long)A.b_dist[q] * A.II < (long long)S(j) + A.lat[j]) ++nrec;
-    }
-  __syncthreads();
-  ndep = block_sum_ll(ndep, buf);
-  lcom = block_sum_ll(lcom, buf);
-  nlat = block_sum_ll(nlat, buf);
-  nrec = block_sum_ll(nrec, buf);
   if (tid == 0) {
     gaus_report R;
-    R.n_dep_viol = ndep;
-    R.n_lat_viol = nlat;
-    R.n_rec_viol = nrec;
-    R.L_com = lcom;
+    R.n_dep_viol = (long long)A.vacc[(size_t)b * 4 + 0];
+    R.L_com = (long long)A.vacc[(size_t)b * 4 + 1];
+    R.n_lat_viol = (long long)A.vacc[(size_t)b * 4 + 2];
+    R.n_rec_viol = (long long)A.vacc[(size_t)b * 4 + 3];
     R.n_res_viol = 0;
     R.L_res = 0;
     for (int c = 0; c < 16; ++c) R.peak[c] = 0;
@@ -268,7 +289,7 @@ __global__ void __launch_bounds__(256) k_verify(const VerArgs A) {
     for (int t = 0; t < A.Dh; ++t) lmm = max(lmm, mm[t]);
     R.L_mem = lmem;
     R.L_mmem = lmm;
-    R.feasible = (ndep == 0 && nlat == 0 && nrec == 0);
+    R.feasible = (R.n_dep_viol == 0 && R.n_lat_viol == 0 && R.n_rec_viol == 0);
     R.res_ok = R.n_res_viol == 0;
     A.rep[b] = R;
   }

@@ -139,6 +139,9 @@ struct gaus_ctx {
   unsigned long long *d_wstat = nullptr;  // B * 2 window statistics of the iteration
   int32_t *d_thr = nullptr;      // B long-window thresholds
   int32_t *d_decision = nullptr; // B outer-step decisions
+  unsigned long long *d_vacc = nullptr;  // verifier counts, usage counts, storage differences
+  size_t vacc_words = 0;
+  int RBv = 32, Gv = 1, nblk_v = 1;      // verifier pass 1: restarts per row, groups, blocks
   int32_t *d_nonfinite = nullptr;  // B flags
   int32_t *d_status_tmp = nullptr; // B
   float *d_loss_tmp = nullptr, *d_terms_tmp = nullptr;
