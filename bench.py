@@ -155,6 +155,14 @@ def algorithmic_flops(torch, mu, sg, src, dst, k, D):
     return 20.0 * n_pt + 8.0 * n_eb, n_pt, n_eb
 
 
+def measured_hbm_gbs():
+    """HBM copy bandwidth from MEASURED_PEAKS.json, else the fallback of an earlier GB300 measurement."""
+    try:
+        return float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["hbm_gbs"])
+    except (OSError, KeyError, ValueError):
+        return 6800.0
+
+
 def profiled_traffic():
     """DRAM bytes per k_edges launch from the committed ncu summary, or None when the
     kernel sources changed since that capture."""
@@ -236,6 +244,10 @@ def gpu_arm(args):
         gpu_id = "GPU-" + str(torch.cuda.get_device_properties(local).uuid)
     except Exception:
         gpu_id = None
+    # this device's FP32 FMA and SFU exp2 throughput (the library's microbenchmark)
+    fp32_peak = g.measure_peak(g.PEAK_FP32)
+    ex2_peak = g.measure_peak(g.PEAK_EX2)
+    hbm_peak = measured_hbm_gbs() * 1e9
     sampler = ClockSampler(gpu_id) if rank == 0 else None
     if world > 1:
         dist.barrier()
@@ -282,6 +294,8 @@ def gpu_arm(args):
     dst = torch.from_numpy(np.asarray(p.dst, np.int64)).cuda()
     ph_ms = np.zeros(4)
     t_edges_total, t_nodes_total, npt_total, neb_total = 0.0, 0.0, 0.0, 0.0
+    t_star, t_star_by = 0.0, {"hbm": 0, "sfu": 0, "fp32": 0}
+    state_bytes = 48.0 * p.V * B + (2.0 * p.E + 6.0 * p.V) * 4.0   # per iteration, design-independent
     fwd_first = fwd_last = None
     nchunk = iters // period
     for k in range(nchunk):
@@ -291,6 +305,10 @@ def gpu_arm(args):
         ph_ms += kms / nchunk
         npt_total += period * 0.5 * (n0 + n1)
         neb_total += period * 0.5 * (e0 + e1)
+        pts, ebs = 0.5 * (n0 + n1), 0.5 * (e0 + e1)
+        bound = {"hbm": state_bytes / hbm_peak, "sfu": pts / ex2_peak, "fp32": (20.0 * pts + 8.0 * ebs) / fp32_peak}
+        t_star += period * max(bound.values())
+        t_star_by[max(bound, key=bound.get)] += period
         t_nodes_total += period * kms[0] * 1e-3
         t_edges_total += period * kms[1] * 1e-3
         fwd_first = kms[1] if fwd_first is None else fwd_first
@@ -475,6 +493,16 @@ def gpu_arm(args):
                                            "frac": nodes_achieved / peak,
                                            "cost_model": "20 flop per CDF point",
                                            "points_per_iter": npt_total / iters}},
+                "iteration_roofline": {
+                    "model": "per iteration T* = max(48 V B + (2E + 6V) 4 bytes / HBM, points / SFU exp2, "
+                             "(20 points + 8 edge-bins) flop / FP32), summed over the solve's iterations",
+                    "t_star_ms_per_step": t_star * 1e3,
+                    "t_measured_ms_per_step": ms / args.steps - nchunk * legalize_verify_ms,
+                    "frac": t_star * 1e3 / (ms / args.steps - nchunk * legalize_verify_ms),
+                    "binding_iterations": t_star_by,
+                    "peaks": {"fp32_tflops_measured": fp32_peak / 1e12, "sfu_ex2_per_s_measured": ex2_peak,
+                              "hbm_gbs": hbm_peak / 1e9,
+                              "fp32_tflops_nominal": peak}},
                 "phase_ms_per_iteration": {"k_nodes": ph_ms[0], "k_edges": ph_ms[1],
                                            "reduce_finalize": ph_ms[2], "k_update": ph_ms[3],
                                            "k_edges_first_period": fwd_first, "k_edges_last_period": fwd_last},

@@ -306,6 +306,18 @@ gaus_status gaus_expected_usage_noalloc(const float *mu, const float *sigma, con
                                         const int32_t *demand, int32_t V, int32_t B, int32_t C, int32_t D,
                                         int32_t II, float window_k, double *usage, void *cuda_stream);
 
+/* Measurement helper, not on the scheduling path: the throughput of this device's
+ * FP32 FMA pipe (what = GAUS_PEAK_FP32; FLOP/s, an FMA counted as 2) or of its
+ * special-function unit's exp2 (what = GAUS_PEAK_EX2; results/s), the two
+ * arithmetic bounds of the node and edge passes.  A microbenchmark of independent
+ * dependency chains on every SM (one wave of 256-thread blocks), best of three timed
+ * runs after a warm-up, with CUDA events on `cuda_stream` (a cudaStream_t; NULL =
+ * the legacy default stream), which it synchronises.  Allocates and frees 1 KiB of
+ * device memory.  Errors: EINVAL (NULL per_second or unknown what), ECUDA. */
+#define GAUS_PEAK_FP32 0
+#define GAUS_PEAK_EX2  1
+gaus_status gaus_measure_peak(int32_t what, double *per_second, void *cuda_stream);
+
 /* Message of the last error on this context ("" if none), or with ctx = NULL the
  * message of this thread's last failed gaus_create or gaus_expected_usage_noalloc.
  * Valid until the next call. */

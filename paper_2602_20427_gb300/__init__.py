@@ -19,7 +19,7 @@ from .build import build
 
 __all__ = ["build", "lib", "Gaus", "default_hparams", "symbols_declared",
            "DEP", "COM", "RES_OBJ", "RES_VIOL", "REG_OBJ", "REC", "DEP_CF", "K", "NT", "STATUS",
-           "GAUSSIAN", "LOGISTIC", "LAPLACE", "CAUCHY"]
+           "GAUSSIAN", "LOGISTIC", "LAPLACE", "CAUCHY", "PEAK_FP32", "PEAK_EX2", "measure_peak"]
 
 DEP, COM, RES_OBJ, RES_VIOL, REG_OBJ, REC = 1, 2, 4, 8, 16, 32
 DEP_CF = 64  # continuous dependency penalty: a variant, not the paper's Eq. dep
@@ -101,6 +101,21 @@ def lib():
                 getattr(L, name).restype = C.c_int
         _lib = L
     return _lib
+
+
+PEAK_FP32, PEAK_EX2 = 0, 1
+
+
+def measure_peak(what: int, stream=None) -> float:
+    """gaus_measure_peak: FP32 FMA FLOP/s (PEAK_FP32) or SFU exp2 results/s (PEAK_EX2)
+    of the current device, from the library's microbenchmark."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    v = C.c_double()
+    rc = lib().gaus_measure_peak(C.c_int32(what), C.byref(v), C.c_void_p(s.cuda_stream))
+    if rc != 0:
+        raise GausError(rc, "gaus_measure_peak failed")
+    return v.value
 
 
 def default_hparams(**kw) -> Hparams:

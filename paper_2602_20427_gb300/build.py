@@ -13,7 +13,8 @@ OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libgaus.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 # (source, object tag, extra defines): gaus_family.cu once per non-normal CDF family
-SOURCES = [("gaus_api.cu", "api", []), ("gaus_plan.cpp", "plan", []), ("gaus_noalloc.cu", "noalloc", [])] + [
+SOURCES = [("gaus_api.cu", "api", []), ("gaus_plan.cpp", "plan", []), ("gaus_noalloc.cu", "noalloc", []),
+           ("gaus_peaks.cu", "peaks", [])] + [
     ("gaus_family.cu", f"family{k}", [f"-DGAUS_FAMILY_ID={k}", "-DGAUS_FAMILY_KERNELS_ONLY"]) for k in (1, 2, 3)]
 
 

@@ -110,3 +110,10 @@ def test_valid_problem_reaches_the_device_check(L):
     pr, keep = _problem(W.tiny_layered(1))
     rc, msg = _create(L, pr)
     assert rc == 5 and "CUDA" in msg
+
+
+def test_measure_peak_rejects_bad_arguments_without_gpu(L):
+    import ctypes as C
+    v = C.c_double()
+    assert L.gaus_measure_peak(C.c_int32(7), C.byref(v), None) == 1
+    assert L.gaus_measure_peak(C.c_int32(g.PEAK_FP32), None, None) == 1
