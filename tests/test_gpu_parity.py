@@ -105,6 +105,17 @@ def test_ragged_restart_counts(g, B):
                     restarts=sorted({0, B // 2, B - 1}))
 
 
+def test_many_restart_groups(g):
+    # B = 200: thirteen groups of 16 restarts, the last one partly filled; the
+    # node, edge and update passes' one-wave grids then hold several groups each
+    p = W.random_layered(6)
+    p.terms = W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL
+    B = 200
+    mu, sg = W.init_state(p, B, 14)
+    hp = g.default_hparams(terms=p.terms)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, np.random.default_rng(14)), hp, restarts=[0, 15, 16, 99, 192, 199])
+
+
 def test_edge_cases_windows_and_bounds(g):
     # mu far outside [0, D), sigma at sigma_min, windows longer than the 32-point
     # cache, zero-latency (chaining) edges, an unlimited class, a high fan-out node
