@@ -94,7 +94,12 @@ static void bin_masses_and_derivs(int32_t D, int32_t fam, double mu, double sigm
     double f_hi = (d == D - 1) ? 0.0 : orc_f(fam, z_hi);
     double zf_lo = (d == 0) ? 0.0 : z_lo * f_lo;
     double zf_hi = (d == D - 1) ? 0.0 : z_hi * f_hi;
-    P[d] = F_hi - F_lo;
+    /* above the centre the mass is taken from the upper tails, F(-z_lo) - F(-z_hi)
+     * (every family is symmetric), so that far-tail bins keep relative accuracy */
+    if (d > 0 && z_lo >= 0.0)
+      P[d] = orc_F(fam, -z_lo) - ((d == D - 1) ? 0.0 : orc_F(fam, -z_hi));
+    else
+      P[d] = F_hi - F_lo;
     if (dPdmu) dPdmu[d] = -(f_hi - f_lo) / sigma;
     if (dPdsig) dPdsig[d] = -(zf_hi - zf_lo) / sigma;
   }

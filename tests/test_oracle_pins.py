@@ -365,3 +365,18 @@ def test_adam_matches_torch_and_first_step_closed_form():
         np.testing.assert_allclose(th, t.detach().numpy(), rtol=1e-14, atol=1e-15)
         if step == 1:
             np.testing.assert_allclose(th, th0 - 0.05 * g / (np.abs(g) + 1e-8), rtol=1e-13)
+
+
+def test_upper_tail_bin_masses_keep_relative_accuracy():
+    # far above the mean the masses come from the upper tails (1 - Phi loses them to
+    # cancellation): compare with scipy's survival function
+    from scipy.stats import norm
+    P = oracle.bin_masses(14, 0.0, 1.0)
+    for d in range(7, 13):
+        ref = norm.sf(d - 0.5) - norm.sf(d + 0.5)
+        assert P[d] == pytest.approx(ref, rel=1e-12)
+    assert P[13] == pytest.approx(norm.sf(12.5), rel=1e-12)
+    # and below the mean from the lower tails, by symmetry
+    Q = oracle.bin_masses(14, 13.0, 1.0)
+    for d in range(1, 7):
+        assert Q[d] == pytest.approx(norm.cdf(d + 0.5 - 13.0) - norm.cdf(d - 0.5 - 13.0), rel=1e-12)
