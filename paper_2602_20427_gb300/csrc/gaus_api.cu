@@ -288,11 +288,10 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   ctx->nblk_r = P.nseg * ctx->Gr;
   ctx->smem_rfwd = rfwd_bytes(ctx->RBr);
   ctx->smem_rbwd = (size_t)P.Dh * ctx->RBr * sizeof(float);
-  ctx->smem_upd = (size_t)ctx->RB * P.Dh * sizeof(float);
   ctx->smem_fin = (size_t)(P.C + 1) * P.Dh * sizeof(double);
   ctx->smem_ver = ((size_t)P.C * P.Dh + (P.D + 1) + P.Dh) * sizeof(long long);
   ctx->smem_leg = (size_t)P.V * sizeof(int) <= kMaxSmem - 1024 ? (size_t)P.V * sizeof(int) : 0;
-  if (ctx->smem_upd > kMaxSmem || ctx->smem_fin > kMaxSmem || ctx->smem_ver > kMaxSmem) {
+  if (ctx->smem_fin > kMaxSmem || ctx->smem_ver > kMaxSmem) {
     ctx->err = "histogram of this horizon/II does not fit in shared memory";
     return GAUS_EINVAL;
   }

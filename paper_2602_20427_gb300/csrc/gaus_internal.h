@@ -11,11 +11,9 @@
 
 namespace gaus {
 
-// Threads per block of the node/edge pass and of the update kernel.
+// Threads per block of the node and edge passes and of the update kernel.
 constexpr int kFwdThreads = 256;
-constexpr int kThreads = 128;
-// Most own-window points cached in shared memory per thread (longer windows recompute).
-constexpr int kUpdThreads = 256;               // threads per k_update block
+constexpr int kUpdThreads = 256;
 constexpr int kGraphUnroll = 10;               // iterations per captured graph
 constexpr int kReduceSpans = 1024;             // segment spans staged per k_reduce pass
 // Restarts per warp row of the node, edge and update passes (a power of two <= 32):
@@ -24,8 +22,7 @@ constexpr int kReduceSpans = 1024;             // segment spans staged per k_red
 constexpr int kMaxRB = 16;
 constexpr int kTableMax = 32;                    // points per CDF table row, at most
 constexpr size_t kTableBytes = (size_t)64 << 20;  // CDF table size bound
-// Fixed-point scale of the usage histograms: P * 2^32 accumulated in int64.
-constexpr float kFix = 4294967296.0f;
+// Fixed-point scale of the usage histograms and forward sums: values * 2^32 in int64.
 constexpr double kInvFix = 1.0 / 4294967296.0;
 // Limits checked by gaus_create.
 constexpr int kMaxClasses = 16;
@@ -99,7 +96,7 @@ struct gaus_ctx {
   int red_blocks = 0;
   int RBr = 32, Gr = 1, nblk_r = 0;  // storage-term kernels: restarts per row, groups, blocks
   size_t smem_rfwd = 0, smem_rbwd = 0;
-  size_t smem_nodes = 0, smem_upd = 0, smem_fin = 0, smem_ver = 0;
+  size_t smem_nodes = 0, smem_fin = 0, smem_ver = 0;
   // device graph
   int32_t *d_perm = nullptr;
   float *d_w = nullptr, *d_bits = nullptr, *d_limit = nullptr;
