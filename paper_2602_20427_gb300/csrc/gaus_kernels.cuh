@@ -712,12 +712,24 @@ __global__ void __launch_bounds__(256) k_reduce(const RedArgs A) {
 }
 #endif  // GAUS_FAMILY_KERNELS_ONLY
 
-// x * 2^-32 of a 2^32 fixed-point value as float, through two 32-bit halves
-// (64-bit integer to floating-point conversions run at the FP64 rate).
-__device__ __forceinline__ float fix_to_float(long long x) {
-  const int hi = (int)(x >> 32);
-  const unsigned lo = (unsigned)((unsigned long long)x & 0xffffffffull);
-  return (float)hi + (float)lo * 2.3283064365386963e-10f;
+// exp((U - m) / tau) of an exact 2^32 fixed-point difference du = U - m <= 0 (the
+// softmax weight of Eq. max), with the exponent kept as a pair of floats: du 2^-32
+// is hi + a + b exactly (hi its integer part, a and b the top 24 and the low 8 bits
+// of its fraction), x = (hi + a + b) / tau = xh + xl with the division's remainder
+// taken through an FMA, and exp(x) = exp(xh) (1 + xl).  Rounding du to one float
+// first would cost |x| ulps of relative error, large for a small tau.
+__device__ __forceinline__ float soft_exp(long long du, float tau) {
+  const int hi = (int)(du >> 32);
+  const unsigned lo = (unsigned)((unsigned long long)du & 0xffffffffull);
+  const float a = (float)(lo >> 8) * 5.9604644775390625e-08f;    // 2^-24
+  const float b = (float)(lo & 255u) * 2.3283064365386963e-10f;  // 2^-32
+  const float fh = (float)hi;
+  const float s = fh + a;  // two-sum: s + e1 = fh + a exactly
+  const float bv = s - fh;
+  const float e1 = (fh - (s - bv)) + (a - bv);
+  const float xh = s / tau;
+  const float xl = (fmaf(-xh, tau, s) + (e1 + b)) / tau;
+  return expf(xh) * (1.0f + xl);
 }
 
 // Deterministic block reductions over 256 threads: a fixed xor-shuffle tree per
@@ -827,7 +839,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   for (int c = 0; c < nh; ++c) {
     const long long m = s_m[c];
     float sacc = 0.f;
-    for (int t = tid; t < Dh; t += 256) sacc += expf(fix_to_float(U[c * Dh + t] - m) / A.tau);
+    for (int t = tid; t < Dh; t += 256) sacc += soft_exp(U[c * Dh + t] - m, A.tau);
     sacc = warp_sum(sacc);
     if (lane == 0) s_wsum[c][wid] = sacc;
   }
@@ -893,13 +905,13 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   for (int i = tid; i < A.C * Dh; i += 256) {
     const int c = i / Dh;
     float h = 0.f;
-    if (on_robj) h += A.w_res * expf(fix_to_float(U[i] - s_m[c]) / A.tau) / s_s[c];
+    if (on_robj) h += A.w_res * soft_exp(U[i] - s_m[c], A.tau) / s_s[c];
     if (on_rv && s_R[c] != LLONG_MAX && U[i] > s_R[c]) h += c_res;
     A.H[(size_t)i * A.B + b] = h;
   }
   if (A.Ureg)
     for (int t = tid; t < Dh; t += 256)
-      A.Hreg[(size_t)b * Dh + t] = A.w_mem * expf(fix_to_float(U[A.C * Dh + t] - s_m[A.C]) / A.tau) / s_s[A.C];
+      A.Hreg[(size_t)b * Dh + t] = A.w_mem * soft_exp(U[A.C * Dh + t] - s_m[A.C], A.tau) / s_s[A.C];
   (void)kInvFixF;
 }
 #endif  // GAUS_FAMILY_KERNELS_ONLY

@@ -84,6 +84,13 @@ def test_legalize_verify_modulo(g, factor):
     _legalize_and_verify(g, p, 16, mu)
 
 
+def test_legalize_verify_modulo_full_size(g):
+    # the loop-body workload at its full size (V = 5,000, 200 back edges, B = 32)
+    p = W.modulo_loop(1, ii_factor=1.25)
+    mu, _ = W.init_state(p, 32, 1)
+    _legalize_and_verify(g, p, 32, mu)
+
+
 def test_legalize_modulo_reports_infeasible_recurrence(g):
     p = W.random_small(5, V=6, D=12, p_edge=1.0, max_lat=1)
     p.lat[:] = 1
