@@ -196,9 +196,12 @@ gaus_status gaus_adam_step(gaus_ctx *ctx, float *mu, float *sigma, const float *
                            float *v_sigma, float *lambda, const float *terms, int32_t step);
 
 /* n_iters fused iterations of Alg. GauS's inner loop (loss, gradient, Adam,
- * multiplier update), each a replay of one captured CUDA graph.  Equivalent to
- * gaus_loss_grad + gaus_adam_step with step = st->step[b] + 1 per iteration.
- * Gradients are not materialised.  EINVAL on NULL state pointers or n_iters < 0. */
+ * multiplier update), enqueued on the context stream as replays of captured CUDA
+ * graphs (ten iterations per graph, one-iteration graphs for the remainder; the
+ * graphs are captured on first use and again after gaus_set_hparams or a change of
+ * state pointers).  Equivalent to gaus_loss_grad + gaus_adam_step with
+ * step = st->step[b] + 1 per iteration.  Gradients are not materialised.  EINVAL
+ * on NULL state pointers or n_iters < 0. */
 gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st);
 
 /* Kernel-level timing of gaus_iterate: runs n_iters iterations exactly as
