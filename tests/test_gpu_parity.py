@@ -287,3 +287,31 @@ def test_modulo_loop_full_size_sampled_usage_and_storage(g):
     lam = np.full((32, 3), 1e-6, np.float32)
     check_loss_grad(p, g, 32, mu, sg, lam, hp, restarts=[0, 17], comp_floor=5e-2)
 
+
+def test_set_hparams_turns_terms_on_and_off(g):
+    # one context: the storage term switched on later (its scratch is allocated then)
+    # and the weights changed; each call matches the oracle with the hparams in force
+    p = W.random_small(31, V=40, D=30, C=2, max_lat=2, p_edge=0.12)
+    rng = np.random.default_rng(33)
+    B = 8
+    mu = (p.start[:, None] + rng.normal(0, 2, size=(p.V, B))).astype(np.float32)
+    sg = rng.uniform(0.3, 2.5, size=(p.V, B)).astype(np.float32)
+    lam = _lam(B, rng)
+    ctx = g.Gaus(p, B, g.default_hparams(terms=W.DEP | W.COM))
+    op = oracle.OracleProblem(p)
+    for hp in (g.default_hparams(terms=W.DEP | W.COM),
+               g.default_hparams(terms=W.DEP | W.REG_OBJ | W.RES_VIOL, tau=0.3, w_mem=1.7, rho=0.05),
+               g.default_hparams(terms=W.COM | W.RES_OBJ, alpha=0.3, w_res=2.0)):
+        ctx.set_hparams(hp)
+        out = ctx.loss_grad(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(),
+                            torch.from_numpy(lam).cuda())
+        torch.cuda.synchronize()
+        loss, terms, gm, gs = oracle.loss_grad(op, _ohp(hp, hp.terms), mu.astype(np.float64),
+                                               sg.astype(np.float64), lam.astype(np.float64))
+        np.testing.assert_allclose(out["loss"].cpu().numpy(), loss, rtol=1e-4, atol=1e-5)
+        np.testing.assert_allclose(out["terms"].cpu().numpy(), terms, rtol=1e-4, atol=1e-5)
+        for ref, got in ((gm, out["grad_mu"].cpu().numpy()), (gs, out["grad_sigma"].cpu().numpy())):
+            for b in range(B):
+                assert np.max(np.abs(got[:, b] - ref[:, b])) <= 1e-4 * np.max(np.abs(ref[:, b])) + 1e-7
+    ctx.close()
+
