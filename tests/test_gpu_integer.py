@@ -84,6 +84,14 @@ def test_legalize_verify_modulo(g, factor):
     _legalize_and_verify(g, p, 16, mu)
 
 
+def test_legalize_verify_regular_global_memory_path(g):
+    # V = 60,000: a schedule (4 V bytes) no longer fits one block's shared memory, so
+    # Alg. 1 runs in its global-memory form
+    p = W.wide_layered(2, width=1200, levels=50)
+    mu, _ = W.init_state(p, 3, 2)
+    _legalize_and_verify(g, p, 3, mu)
+
+
 def test_legalize_verify_modulo_full_size(g):
     # the loop-body workload at its full size (V = 5,000, 200 back edges, B = 32)
     p = W.modulo_loop(1, ii_factor=1.25)
