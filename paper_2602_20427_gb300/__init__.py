@@ -241,31 +241,14 @@ class Gaus:
                     status=torch.zeros(self.B, dtype=torch.int32, device=dev))
 
     def iterate(self, n, state):
-        torch = self.torch
-        VB, f32 = (self.V, self.B), torch.float32
-        s = State(*(self._dev(state[k], f32, VB).value for k in ("mu", "sigma", "m_mu", "v_mu", "m_sigma",
-                                                                   "v_sigma")),
-                  self._dev(state["lambda_"], f32, (self.B, K)).value,
-                  self._dev(state["step"], torch.int32, (self.B,)).value,
-                  self._dev(state["loss"], f32, (self.B,)).value,
-                  self._dev(state["terms"], f32, (self.B, NT)).value,
-                  self._dev(state["status"], torch.int32, (self.B,)).value)
-        self._check(lib().gaus_iterate(self._ctx, C.c_int32(n), C.byref(s)))
+        """n fused iterations (gaus_iterate) on the state dict of new_state()/init_state()."""
+        self._check(lib().gaus_iterate(self._ctx, C.c_int32(n), C.byref(self._state(state))))
 
     def profile_iterate(self, n, state):
-        """Mean per-phase durations (ms) of n iterations:
-        [window table, node/edge pass, reductions + finalize, gradient + Adam]."""
-        torch = self.torch
-        VB, f32 = (self.V, self.B), torch.float32
-        s = State(*(self._dev(state[k], f32, VB).value for k in ("mu", "sigma", "m_mu", "v_mu", "m_sigma",
-                                                                   "v_sigma")),
-                  self._dev(state["lambda_"], f32, (self.B, K)).value,
-                  self._dev(state["step"], torch.int32, (self.B,)).value,
-                  self._dev(state["loss"], f32, (self.B,)).value,
-                  self._dev(state["terms"], f32, (self.B, NT)).value,
-                  self._dev(state["status"], torch.int32, (self.B,)).value)
+        """Mean per-iteration durations (ms) over n iterations launched kernel by kernel:
+        [node pass, edge pass, reductions + finalize, update] (gaus_profile_iterate)."""
         ms = (C.c_double * 4)(0.0, 0.0, 0.0, 0.0)
-        self._check(lib().gaus_profile_iterate(self._ctx, C.c_int32(n), C.byref(s), ms))
+        self._check(lib().gaus_profile_iterate(self._ctx, C.c_int32(n), C.byref(self._state(state)), ms))
         return list(ms)
 
     def _state(self, state):
