@@ -363,6 +363,28 @@ def gpu_arm(args):
                   "best_score_min": float(bsc[found].min()) if found.any() else None,
                   "best_score_mean": float(bsc[found].mean()) if found.any() else None,
                   "score": "L_res + alpha L_com of the best legal schedule (no resource overflow)"}
+        # the same solver from the timed workload's initialization (mu = ASAP + N(0, 2),
+        # sigma = 1.5), twice as long: how many restarts reach a feasible schedule, and when
+        bufs = ctxS.init_state(kappa=1.0 / 6.0, mu0=dmu0, out=bufs)
+        bufs[0]["sigma"].copy_(dsg0)
+        bufs[1].copy_(dsg0)
+        n_long = 2 * iters // period
+        torch.cuda.synchronize()
+        evS[0].record()
+        ctxS.solve(n_long, period, *bufs, work=work)
+        evS[1].record()
+        torch.cuda.synchronize()
+        lms = evS[0].elapsed_time(evS[1])
+        bsc = bufs[2]["score"].cpu().numpy()
+        bit = bufs[2]["iter"].cpu().numpy()
+        found = np.isfinite(bsc)
+        solver["from_workload_init"] = {
+            "iterations": n_long * period, "restart_iterations_per_s": n_long * period * B / (lms / 1e3),
+            "restarts_with_feasible_best": int(found.sum()),
+            "best_found_at_iteration_min": int(bit[found].min()) if found.any() else None,
+            "best_found_at_iteration_median": float(np.median(bit[found])) if found.any() else None,
+            "best_score_min": float(bsc[found].min()) if found.any() else None,
+            "best_score_mean": float(bsc[found].mean()) if found.any() else None}
         ctxS.close()
 
     # ---- Formulation C (modulo scheduling) sweep: II in {MII, 1.25 MII, 1.5 MII} on the
