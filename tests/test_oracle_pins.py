@@ -380,3 +380,18 @@ def test_upper_tail_bin_masses_keep_relative_accuracy():
     Q = oracle.bin_masses(14, 13.0, 1.0)
     for d in range(1, 7):
         assert Q[d] == pytest.approx(norm.cdf(d + 0.5 - 13.0) - norm.cdf(d - 0.5 - 13.0), rel=1e-12)
+
+
+@pytest.mark.parametrize("tau", [0.01, 0.3, 2.0])
+def test_lse_bounds(tau):
+    # Eq. max: max_d x_d <= LSE_tau(x) <= max_d x_d + tau ln(#bins), per class and for storage
+    p = W.random_small(41, V=9, D=12, C=3, max_lat=2, p_edge=0.3)
+    rng = np.random.default_rng(int(tau * 100))
+    mu, sigma = rng.uniform(0, 11, p.V), rng.uniform(0.3, 2.0, p.V)
+    op = oracle.OracleProblem(p)
+    _, T, _, _ = oracle.loss_grad(op, oracle.hparams(tau=tau, terms=W.RES_OBJ | W.REG_OBJ), mu[:, None],
+                                  sigma[:, None], np.zeros((1, 3)))
+    U, R = oracle.expected_hist(op, mu, sigma)
+    lo = U.max(axis=1).sum()
+    assert lo - 1e-12 <= T[0, oracle.T_RES] <= lo + p.C * tau * math.log(p.D) + 1e-12
+    assert R.max() - 1e-12 <= T[0, oracle.T_REG] <= R.max() + tau * math.log(p.D) + 1e-12
