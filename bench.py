@@ -53,17 +53,18 @@ def parse():
     ap.add_argument("--no-solver", action="store_true", help="skip the complete-solver runs (gaus_solve)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-families", action="store_true", help="skip the CDF-family timings")
+    ap.add_argument("--restarts", type=int, default=64,
+                    help="restarts per rank (64 is the benchmark configuration; others for scaling studies)")
     ap.add_argument("--profile-range", action="store_true",
                     help="bracket the timed steps with cudaProfilerStart/Stop (for ncu --profile-from-start off)")
     return ap.parse_args()
 
 
-def workload(rank=0):
+def workload(rank=0, B=64):
     """The benchmark workload of one rank: the same logic-network DAG on every rank,
-    and B = 64 restarts of its own (initial state seeded by the rank), so the ranks'
+    and B (64) restarts of its own (initial state seeded by the rank), so the ranks'
     restarts are independent and need no data-path collective (weak scaling)."""
     p = W.logic_network(1)
-    B = 64
     mu, sg = W.init_state(p, B, seed=1 + rank)
     return p, B, mu, sg
 
@@ -199,7 +200,7 @@ def gpu_arm(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     torch.cuda.set_device(local)
     g.build()
-    p, B, mu0, sg0 = workload(rank)
+    p, B, mu0, sg0 = workload(rank, args.restarts)
     hp = g.default_hparams(terms=p.terms)
     ctx = g.Gaus(p, B, hp)
     iters, period = args.iters, args.period
