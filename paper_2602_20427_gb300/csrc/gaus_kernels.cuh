@@ -1,21 +1,22 @@
 // gaus_kernels.cuh -- device code of one GauS iteration (Sec. 3.2-3.3, App. B).
 //
-// Work item: one (node v, restart b).  Threads of a warp are restarts of the same
-// node (lanes = b), so every mu/sigma gather of a neighbour is one coalesced
-// 128-byte load.  Each thread keeps its own window of CDF points
-//   C_v(t) = Phi((t + 1/2 - mu_v) / sigma_v),  t in [a_v, b_v] = points within
+// Work item: one (node v, restart b).  A warp row of RB (16) lanes holds RB
+// restarts of the same node (lanes = b; two nodes or edges per warp), so every
+// mu/sigma gather of a neighbour is one coalesced 64-byte load.  Each (node,
+// restart) has its window of CDF points
+//   C_v(t) = F((t + 1/2 - mu_v) / sigma_v),  t in [a_v, b_v] = points within
 //   window_k * sigma_v of mu_v, with C_v(t) = 0 below and 1 above (Eq. round and
-// its open end bins), and evaluates each neighbour's CDF at the points it needs.
+// its open end bins; F the normal CDF, or another family of App. D).
 //
 // k_nodes   : windows, the CDF table (C at each window point, computed once per
 //             (node, restart) and read by every incident edge) and bin masses ->
-//             usage histogram (shared-memory fixed point, one class per block, no
-//             global atomics).
+//             usage histogram (shared-memory fixed point, one class per block).
 // k_edges   : every edge term, once per (edge, restart), from both endpoints'
-//             table rows: forward sums and each endpoint's unscaled partial
-//             gradients, written to per-edge slots (no atomics).
-// k_finalize: one block per restart -- usage per class, LogSumExp (Eq. max),
-//             ReLU (Eq. relu), the augmented-Lagrangian coefficients (Sec. 3.3).
+//             table rows: forward sums (exact fixed point) and each endpoint's
+//             unscaled partial gradients, written to per-edge slots.
+// k_reduce  : usage per (restart, class, bin) from the node pass's block partials.
+// k_finalize: one block per restart -- LogSumExp (Eq. max), ReLU (Eq. relu), the
+//             augmented-Lagrangian coefficients and multiplier step (Sec. 3.3).
 // k_update  : usage adjoint of the node's own window, the node's edge slots
 //             gathered in a fixed order, the combined gradient and (optionally)
 //             the Adam step.
