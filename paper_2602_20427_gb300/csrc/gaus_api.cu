@@ -224,10 +224,12 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     ctx->err = "no CUDA device";
     return GAUS_ECUDA;
   }
+  // restarts per warp row: up to kMaxRB, fewer for long horizons so that the node
+  // pass's usage histogram (two u32 halves per bin and restart) fits shared memory
   ctx->RB = 1;
   while (ctx->RB < P.B && ctx->RB < kMaxRB) ctx->RB <<= 1;
+  while (ctx->RB > 1 && 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned) > kMaxSmem - 1024) ctx->RB >>= 1;
   ctx->G = (P.B + ctx->RB - 1) / ctx->RB;
-  // k_nodes shared memory: the two halves of the usage histogram
   ctx->smem_nodes = 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned);
   if (ctx->smem_nodes > kMaxSmem - 1024) {
     ctx->err = "usage histogram of this horizon/II does not fit in shared memory";
@@ -246,7 +248,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     }
     return std::max(1, occ) * nsm;
   };
-  plan_segments(P, resident((const void *)ks.nodes, kFwdThreads, ctx->smem_nodes));
+  plan_segments(P, resident((const void *)ks.nodes, kFwdThreads, ctx->smem_nodes), ctx->RB);
   ctx->nblk = P.nseg * ctx->G;
   // edge pass: one wave of blocks, the same number per restart group (rows of
   // edges grid-stride); k_dep_cf: one block per chunk of a warp pass per group

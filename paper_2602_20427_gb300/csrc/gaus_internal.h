@@ -73,7 +73,7 @@ struct Plan {
 
 // Returns GAUS_OK or an error with a message.
 gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err);
-void plan_segments(Plan &P, int target_blocks);
+void plan_segments(Plan &P, int target_blocks, int RB);
 gaus_status check_hparams(const gaus_hparams *hp, std::string *err);
 float family_window_k(float window_k, int family);
 

@@ -65,12 +65,10 @@ static bool valid_csr(int V, int E, const int32_t *ptr, const int32_t *idx) {
 }
 
 // Segments: contiguous internal nodes of one class, sized so that the per-node
-// kernels launch about target_blocks blocks over all restart groups.
-void plan_segments(Plan &P, int target_blocks) {
+// kernels launch about target_blocks blocks over all restart groups of RB restarts.
+void plan_segments(Plan &P, int target_blocks, int RB) {
   const int V = P.V, C = P.C;
   P.seg.clear();
-  int RB = 1;
-  while (RB < P.B && RB < kMaxRB) RB <<= 1;
   int G = (P.B + RB - 1) / RB;
   long want = std::max(1L, (long)target_blocks / G);
   int seglen = (int)std::max(1L, ((long)V + want - 1) / want);
@@ -355,7 +353,9 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
     P.lq_ptr[q + 1] = (int32_t)P.lq_src.size();
   }
 
-  plan_segments(P, target_blocks);
+  int RB = 1;
+  while (RB < P.B && RB < kMaxRB) RB <<= 1;
+  plan_segments(P, target_blocks, RB);
   return GAUS_OK;
 }
 

@@ -315,3 +315,16 @@ def test_set_hparams_turns_terms_on_and_off(g):
                 assert np.max(np.abs(got[:, b] - ref[:, b])) <= 1e-4 * np.max(np.abs(ref[:, b])) + 1e-7
     ctx.close()
 
+
+def test_long_horizon_fewer_restarts_per_row(g):
+    # D = 3,000: sixteen restarts per row would need 384 KB of shared memory for the
+    # node pass's usage histogram, so the rows shrink to four restarts
+    p = W.random_small(51, V=40, D=3000, C=2, max_lat=3, p_edge=0.12)
+    p.terms = W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL
+    rng = np.random.default_rng(51)
+    B = 16
+    mu = (rng.uniform(0, p.D - 1, size=(p.V, B))).astype(np.float32)
+    sg = rng.uniform(0.3, 40.0, size=(p.V, B)).astype(np.float32)
+    hp = g.default_hparams(terms=p.terms, tau=0.5, rho=0.01)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, rng), hp, restarts=[0, 7, 15])
+
