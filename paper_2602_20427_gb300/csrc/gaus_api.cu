@@ -157,6 +157,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   F.beta1 = ctx->hp.beta1; F.beta2 = ctx->hp.beta2;
   F.H = ctx->d_H; F.coef = ctx->d_coef; F.loss = loss; F.terms_out = terms;
   F.wstat = ctx->d_wstat; F.thr = ctx->d_thr; F.W = ctx->W;
+  F.usmem = ctx->smem_fin > 0;
   F.status = status; F.nonfinite = ctx->d_nonfinite;
   k_finalize<<<P.B, 256, ctx->smem_fin, st>>>(F);
   CK(cudaGetLastError(), "k_finalize launch");
@@ -290,13 +291,13 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   ctx->nblk_r = P.nseg * ctx->Gr;
   ctx->smem_rfwd = rfwd_bytes(ctx->RBr);
   ctx->smem_rbwd = (size_t)P.Dh * ctx->RBr * sizeof(float);
+  // finalize and verifier pass 2 stage a restart's rows in shared memory when they
+  // fit (else the kernels read them in place)
   ctx->smem_fin = (size_t)(P.C + 1) * P.Dh * sizeof(double);
   ctx->smem_ver = ((size_t)P.C * P.Dh + (P.D + 1) + P.Dh) * sizeof(long long);
+  if (ctx->smem_fin > kMaxSmem - 4096) ctx->smem_fin = 0;
+  if (ctx->smem_ver > kMaxSmem - 1024) ctx->smem_ver = 0;
   ctx->smem_leg = (size_t)P.V * sizeof(int) <= kMaxSmem - 1024 ? (size_t)P.V * sizeof(int) : 0;
-  if (ctx->smem_fin > kMaxSmem || ctx->smem_ver > kMaxSmem) {
-    ctx->err = "histogram of this horizon/II does not fit in shared memory";
-    return GAUS_EINVAL;
-  }
   CK(cudaStreamCreateWithFlags(&ctx->side, cudaStreamNonBlocking), "side stream");
   {
     int least = 0, greatest = 0;
@@ -362,7 +363,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_hspan, (size_t)ctx->nblk));
   TRY(scratch(ctx, &ctx->d_fwdtot, (size_t)P.B * 3));
   // verifier: per-restart counts, usage counts and storage difference arrays
-  ctx->vacc_words = (size_t)P.B * (4 + (size_t)P.C * P.Dh + (size_t)P.D + 1);
+  ctx->vacc_words = (size_t)P.B * (4 + (size_t)P.C * P.Dh + (size_t)P.D + 1 + (size_t)P.Dh);
   TRY(scratch(ctx, &ctx->d_vacc, ctx->vacc_words));
   ctx->RBv = 1;
   while (ctx->RBv < P.B && ctx->RBv < 32) ctx->RBv <<= 1;
@@ -649,6 +650,8 @@ gaus_status gaus_verify(gaus_ctx *ctx, const int32_t *sched, gaus_report *rep) {
   A.vacc = ctx->d_vacc;
   A.vcnt = A.vacc + (size_t)P.B * 4;
   A.vdiff = A.vcnt + (size_t)P.B * P.C * P.Dh;
+  A.vmm = reinterpret_cast<long long *>(A.vdiff + (size_t)P.B * (P.D + 1));
+  A.vsmem = ctx->smem_ver > 0;
   CK(cudaMemsetAsync(ctx->d_vacc, 0, ctx->vacc_words * sizeof(unsigned long long), ctx->stream), "verify memset");
   k_verify_scan<<<ctx->nblk_v, 256, 0, ctx->stream>>>(A);
   CK(cudaGetLastError(), "k_verify_scan launch");

@@ -176,6 +176,8 @@ struct VerArgs {
   // zeroed before pass 1: per restart the counts (dep, com, lat, rec), the usage
   // counts (B, C, Dh) and the storage difference array (B, D + 1), exact int64
   unsigned long long *vacc, *vcnt, *vdiff;
+  long long *vmm;  // (B, Dh) folded storage when pass 2 cannot stage it in shared memory
+  int vsmem;       // 1: pass 2 stages its rows in shared memory
 };
 
 // Verifier pass 1 (Sec. 2.1 definitions; L_com of App. B.1): items are the edges,
@@ -251,12 +253,21 @@ __global__ void __launch_bounds__(256) k_verify_scan(const VerArgs A) {
 // its fold modulo II).
 __global__ void __launch_bounds__(256) k_verify_fin(const VerArgs A) {
   extern __shared__ __align__(16) unsigned char smem_v[];
-  long long *cnt = reinterpret_cast<long long *>(smem_v);
-  long long *diff = cnt + (size_t)A.C * A.Dh;
-  long long *mm = diff + (A.D + 1);
   const int b = blockIdx.x, tid = threadIdx.x;
-  for (int i = tid; i < A.C * A.Dh; i += 256) cnt[i] = (long long)A.vcnt[(size_t)b * A.C * A.Dh + i];
-  for (int i = tid; i <= A.D; i += 256) diff[i] = (long long)A.vdiff[(size_t)b * (A.D + 1) + i];
+  // the restart's rows staged in shared memory when they fit, else used in place
+  // (the folded storage then in its global scratch row)
+  long long *cnt = reinterpret_cast<long long *>(A.vcnt + (size_t)b * A.C * A.Dh);
+  long long *diff = reinterpret_cast<long long *>(A.vdiff + (size_t)b * (A.D + 1));
+  long long *mm = A.vmm + (size_t)b * A.Dh;
+  if (A.vsmem) {
+    long long *s_cnt = reinterpret_cast<long long *>(smem_v);
+    long long *s_diff = s_cnt + (size_t)A.C * A.Dh;
+    for (int i = tid; i < A.C * A.Dh; i += 256) s_cnt[i] = cnt[i];
+    for (int i = tid; i <= A.D; i += 256) s_diff[i] = diff[i];
+    cnt = s_cnt;
+    diff = s_diff;
+    mm = s_diff + (A.D + 1);
+  }
   for (int i = tid; i < A.Dh; i += 256) mm[i] = 0;
   __syncthreads();
   if (tid == 0) {

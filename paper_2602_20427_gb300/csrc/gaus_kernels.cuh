@@ -87,6 +87,7 @@ struct FinArgs {
   unsigned long long *wstat;  // read into thr and cleared for the next iteration
   int32_t *thr;
   int W;
+  int usmem;          // 1: the restart's usage and storage rows are staged in shared memory
 };
 
 struct UpdArgs {
@@ -787,9 +788,17 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   if (tid >= 64 && tid < 66) s_ws[tid - 64] = A.wstat[2 * b + tid - 64];
   if (tid == 96) s_bad = A.nonfinite[b];
   if (tid == 128) s_step = A.step ? A.step[b] : 0;
-  for (int i = tid; i < A.C * Dh; i += 256) U[i] = A.Ug[(size_t)b * A.C * Dh + i];
-  if (A.Ureg)
-    for (int t = tid; t < Dh; t += 256) U[A.C * Dh + t] = A.Ureg[(size_t)b * Dh + t];
+  // the restart's usage rows (then the storage row) in shared memory when they fit,
+  // else read from global memory where they are used (long horizons, many classes)
+  const long long *Ug = A.Ug + (size_t)b * A.C * Dh, *Ur = A.Ureg ? A.Ureg + (size_t)b * Dh : nullptr;
+  auto uget = [&](int c, int t) -> long long {
+    return A.usmem ? U[c * Dh + t] : (c < A.C ? Ug[c * Dh + t] : Ur[t]);
+  };
+  if (A.usmem) {
+    for (int i = tid; i < A.C * Dh; i += 256) U[i] = Ug[i];
+    if (A.Ureg)
+      for (int t = tid; t < Dh; t += 256) U[A.C * Dh + t] = Ur[t];
+  }
   if (tid < A.C) {
     const float R = A.limit[tid];
     // limits in fixed point; an infinite or huge limit never binds
@@ -812,7 +821,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
     const long long R = c < A.C ? s_R[c] : LLONG_MAX;
     long long m = LLONG_MIN;
     for (int t = tid; t < Dh; t += 256) {
-      const long long u = U[c * Dh + t];
+      const long long u = uget(c, t);
       m = max(m, u);
       if (R != LLONG_MAX && u > R) ex += u - R;
     }
@@ -840,7 +849,7 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   for (int c = 0; c < nh; ++c) {
     const long long m = s_m[c];
     float sacc = 0.f;
-    for (int t = tid; t < Dh; t += 256) sacc += soft_exp(U[c * Dh + t] - m, A.tau);
+    for (int t = tid; t < Dh; t += 256) sacc += soft_exp(uget(c, t) - m, A.tau);
     sacc = warp_sum(sacc);
     if (lane == 0) s_wsum[c][wid] = sacc;
   }
@@ -905,14 +914,15 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   // usage adjoint dL/dU_c(t) = w_res softmax_c(t) + c_res [U_c(t) > R_c], [class][bin][restart]
   for (int i = tid; i < A.C * Dh; i += 256) {
     const int c = i / Dh;
+    const long long u = uget(c, i - c * Dh);
     float h = 0.f;
-    if (on_robj) h += A.w_res * soft_exp(U[i] - s_m[c], A.tau) / s_s[c];
-    if (on_rv && s_R[c] != LLONG_MAX && U[i] > s_R[c]) h += c_res;
+    if (on_robj) h += A.w_res * soft_exp(u - s_m[c], A.tau) / s_s[c];
+    if (on_rv && s_R[c] != LLONG_MAX && u > s_R[c]) h += c_res;
     A.H[(size_t)i * A.B + b] = h;
   }
   if (A.Ureg)
     for (int t = tid; t < Dh; t += 256)
-      A.Hreg[(size_t)b * Dh + t] = A.w_mem * soft_exp(U[A.C * Dh + t] - s_m[A.C], A.tau) / s_s[A.C];
+      A.Hreg[(size_t)b * Dh + t] = A.w_mem * soft_exp(uget(A.C, t) - s_m[A.C], A.tau) / s_s[A.C];
   (void)kInvFixF;
 }
 #endif  // GAUS_FAMILY_KERNELS_ONLY

@@ -328,3 +328,29 @@ def test_long_horizon_fewer_restarts_per_row(g):
     hp = g.default_hparams(terms=p.terms, tau=0.5, rho=0.01)
     check_loss_grad(p, g, B, mu, sg, _lam(B, rng), hp, restarts=[0, 7, 15])
 
+
+def test_many_classes_long_horizon_rows_in_global_memory(g):
+    # 16 classes and D = 2,000: a restart's usage rows (and the verifier's counts) no
+    # longer fit one block's shared memory, so the finalize and verifier pass 2 read
+    # them in place; loss and gradient against the oracle, reports bit-exact
+    p = W.random_small(61, V=60, D=2000, C=16, max_lat=3, p_edge=0.05)
+    p.terms = W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL | W.REG_OBJ
+    rng = np.random.default_rng(61)
+    B = 8
+    mu = (rng.uniform(0, p.D - 1, size=(p.V, B))).astype(np.float32)
+    sg = rng.uniform(0.3, 20.0, size=(p.V, B)).astype(np.float32)
+    hp = g.default_hparams(terms=p.terms, tau=0.5, rho=0.01)
+    check_loss_grad(p, g, B, mu, sg, _lam(B, rng), hp, restarts=[0, 5])
+    ctx = g.Gaus(p, B, hp)
+    sched = ctx.round(torch.from_numpy(mu).cuda())
+    reps = ctx.verify(sched)
+    torch.cuda.synchronize()
+    op = oracle.OracleProblem(p)
+    s_np = sched.cpu().numpy()
+    for b in range(B):
+        r = oracle.verify(op, s_np[:, b])
+        for k in oracle.REPORT_FIELDS:
+            assert reps[b][k] == r[k], (b, k)
+        assert reps[b]["peak"] == r["peak"]
+    ctx.close()
+
