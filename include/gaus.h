@@ -2,7 +2,8 @@
  * gaus.h -- C ABI of the GB300 (sm_103a) GauS hot path.
  *
  * GauS (arXiv 2602.20427) relaxes each operator's start step to a Gaussian
- * X_v ~ N(mu_v, sigma_v^2) (Sec. 3.1), turns objectives and constraint
+ * X_v ~ N(mu_v, sigma_v^2) (Sec. 3.1; App. D: or a scale-matched logistic,
+ * Laplace or Cauchy variable), turns objectives and constraint
  * violations into expectations over the rounded steps (Sec. 3.2, App. B) and
  * minimises them with an augmented Lagrangian and Adam (Sec. 3.3).  This
  * library evaluates that loss and its gradient, applies Adam and the
