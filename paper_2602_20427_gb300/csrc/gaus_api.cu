@@ -157,9 +157,9 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   F.beta1 = ctx->hp.beta1; F.beta2 = ctx->hp.beta2;
   F.H = ctx->d_H; F.coef = ctx->d_coef; F.loss = loss; F.terms_out = terms;
   F.wstat = ctx->d_wstat; F.thr = ctx->d_thr; F.W = ctx->W;
-  F.usmem = ctx->smem_fin > 0;
   F.status = status; F.nonfinite = ctx->d_nonfinite;
-  k_finalize<<<P.B, 256, ctx->smem_fin, st>>>(F);
+  if (ctx->smem_fin > 0) k_finalize<true><<<P.B, 256, ctx->smem_fin, st>>>(F);
+  else k_finalize<false><<<P.B, 256, 0, st>>>(F);
   CK(cudaGetLastError(), "k_finalize launch");
   if (reg) {
     ks.reg_bwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rbwd, st>>>(RA);
@@ -194,7 +194,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
 // different sizes can be used side by side (each launch still requests its own size).
 gaus_status set_smem_attrs(gaus_ctx *ctx) {
   const KernelSet &ks = kernels(ctx->hp.family);
-  const void *fns[] = {(const void *)ks.nodes, (const void *)k_finalize, (const void *)ks.reg_fwd,
+  const void *fns[] = {(const void *)ks.nodes, (const void *)k_finalize<true>, (const void *)ks.reg_fwd,
                        (const void *)ks.reg_bwd, (const void *)k_verify_fin, (const void *)k_legalize_regular_smem};
   int dev = 0, optin = 0;
   CK(cudaGetDevice(&dev), "cudaGetDevice");

@@ -87,7 +87,6 @@ struct FinArgs {
   unsigned long long *wstat;  // read into thr and cleared for the next iteration
   int32_t *thr;
   int W;
-  int usmem;          // 1: the restart's usage and storage rows are staged in shared memory
 };
 
 struct UpdArgs {
@@ -765,9 +764,12 @@ __device__ __forceinline__ long long block_max_ll(long long x, long long *sh) {
 }
 
 #ifndef GAUS_FAMILY_KERNELS_ONLY
-// One block (256 threads) per restart.  Usage and storage stay exact 2^32 fixed
-// point (max and ReLU excess in integers); the softmax runs in fp32 on exact
-// differences from the max, and only thread 0 assembles the loss in fp64.
+// One block (256 threads) per restart; kSmem: the restart's usage and storage rows
+// are staged in shared memory (else read in place: long horizons, many classes).
+// Usage and storage stay exact 2^32 fixed point (max and ReLU excess in integers);
+// the softmax runs in fp32 on exact differences from the max, and only thread 0
+// assembles the loss in fp64.
+template <bool kSmem>
 __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   extern __shared__ __align__(16) unsigned char smem_f[];
   long long *U = reinterpret_cast<long long *>(smem_f);  // (C + 1) * Dh
@@ -792,9 +794,9 @@ __global__ void __launch_bounds__(256) k_finalize(const FinArgs A) {
   // else read from global memory where they are used (long horizons, many classes)
   const long long *Ug = A.Ug + (size_t)b * A.C * Dh, *Ur = A.Ureg ? A.Ureg + (size_t)b * Dh : nullptr;
   auto uget = [&](int c, int t) -> long long {
-    return A.usmem ? U[c * Dh + t] : (c < A.C ? Ug[c * Dh + t] : Ur[t]);
+    return kSmem ? U[c * Dh + t] : (c < A.C ? Ug[c * Dh + t] : Ur[t]);
   };
-  if (A.usmem) {
+  if (kSmem) {
     for (int i = tid; i < A.C * Dh; i += 256) U[i] = Ug[i];
     if (A.Ureg)
       for (int t = tid; t < Dh; t += 256) U[A.C * Dh + t] = Ur[t];
