@@ -41,7 +41,10 @@ typedef enum {
   GAUS_ENOMEM = 4,      /* device or host allocation failed                        */
   GAUS_ECUDA = 5,       /* a CUDA runtime call failed (see gaus_last_error)        */
   GAUS_ENONFINITE = 6,  /* per restart: a mu or sigma was NaN/Inf or sigma < 1e-30 */
-  GAUS_ENOTCONV = 7     /* per restart: Alg. 2 did not settle within |V| sweeps    */
+  GAUS_ENOTCONV = 7,    /* per restart: Alg. 2 did not settle within |V| sweeps    */
+  GAUS_ETIMEOUT = 8     /* per restart: a barrier of the persistent iteration kernel
+                           waited longer than its limit (4 s); that call's outputs
+                           for the restart are unspecified                            */
 } gaus_status;
 
 /* Terms of the loss (bit mask).  Objectives are weighted, constraints enter the
@@ -214,6 +217,19 @@ gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st);
  * Synchronises the context's stream.  Library feature for measurement; not on the
  * hot path. */
 gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st, double *ms_out);
+
+/* Phase profile of the persistent iteration kernel (measurement helper, not on the
+ * hot path): runs n_iters iterations exactly as gaus_iterate does, with every block
+ * recording the device's global timer at the start and end of each of its three
+ * phases, and writes to out[0..11] (host, milliseconds, means over the
+ * iterations): [0..2] critical path of phase 1 (windows, CDF table, usage
+ * histogram), phase 2 (usage terms, edge terms) and phase 3 (gradient, Adam) --
+ * the last block's end minus the first block's start; [3..5] the mean block's time
+ * in each phase; [6..7] latency of the two group barriers (last arrival to first
+ * release); [8] the whole iteration; [9..11] the slowest block in each phase.
+ * Synchronises the context's stream.  EINVAL when the context's terms or sizes run
+ * the multi-kernel path (storage term, continuous dependency penalty, D > 32767). */
+gaus_status gaus_profile_phases(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st, double *out);
 
 /* Round every mean to s = floor(mu + 1/2) (Sec. 3.3 Sampling; exact for every
  * fp32 value) and legalize it: Alg. 1 (clamp to [ASAP, ALAP], then a forward push

@@ -28,7 +28,7 @@ K, NT = 3, 6
 # logistic, Laplace or Cauchy CDF (App. D)
 GAUSSIAN, LOGISTIC, LAPLACE, CAUCHY = 0, 1, 2, 3
 STATUS = {0: "OK", 1: "EINVAL", 2: "ECYCLE", 3: "EHORIZON", 4: "ENOMEM", 5: "ECUDA",
-          6: "ENONFINITE", 7: "ENOTCONV"}
+          6: "ENONFINITE", 7: "ENOTCONV", 8: "ETIMEOUT"}
 
 _HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "gaus.h")
 
@@ -250,6 +250,17 @@ class Gaus:
         ms = (C.c_double * 4)(0.0, 0.0, 0.0, 0.0)
         self._check(lib().gaus_profile_iterate(self._ctx, C.c_int32(n), C.byref(self._state(state)), ms))
         return list(ms)
+
+    PHASE_KEYS = ("p1_crit", "p2_crit", "p3_crit", "p1_mean", "p2_mean", "p3_mean", "bar1", "bar2",
+                  "iteration", "p1_max", "p2_max", "p3_max")
+
+    def profile_phases(self, n, state):
+        """Phase profile of n fused iterations of the persistent kernel (ms, means over
+        the iterations; gaus_profile_phases): critical path, mean and slowest block of
+        each phase, the two barrier latencies and the iteration time."""
+        out = (C.c_double * 12)()
+        self._check(lib().gaus_profile_phases(self._ctx, C.c_int32(n), C.byref(self._state(state)), out))
+        return dict(zip(self.PHASE_KEYS, list(out)))
 
     def _state(self, state):
         torch = self.torch

@@ -189,6 +189,116 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
   return GAUS_OK;
 }
 
+// The persistent kernel covers every term but the storage term and the continuous
+// dependency penalty (those run on the multi-kernel path).
+bool fused_ok(const gaus_ctx *ctx) {
+  return ctx->fK > 0 && !(ctx->hp.terms & (GAUS_REG_OBJ | GAUS_DEP_CF));
+}
+
+// Enqueue n_iters fused iterations (adam) or one loss + gradient evaluation
+// (!adam) as cooperative launches of the persistent kernel, one per batch of
+// restart groups the device holds at once (a single launch unless B is huge).
+gaus_status enqueue_fused(gaus_ctx *ctx, cudaStream_t st, int n_iters, bool adam, const float *mu, const float *sg,
+                          float *m_mu, float *v_mu, float *m_sg, float *v_sg, float *lambda, int32_t *step,
+                          float *grad_mu, float *grad_sg, float *loss, float *terms, int32_t *status,
+                          unsigned long long *prof) {
+  const Plan &P = ctx->plan;
+  FusedArgs A;
+  A.V = P.V; A.B = P.B; A.D = P.D; A.II = P.II; A.Dh = P.Dh; A.C = P.C; A.K = ctx->fK;
+  A.RG = ctx->fRG; A.RBp = ctx->fRBp; A.RB1 = ctx->fRB1;
+  A.W = ctx->fW; A.n_iters = n_iters; A.nseg = P.nfseg;
+  A.k_win = ctx->k_win; A.alpha = ctx->hp.alpha; A.tau = ctx->hp.tau; A.rho = ctx->hp.rho; A.w_res = ctx->hp.w_res;
+  A.lr = ctx->hp.lr; A.beta1 = ctx->hp.beta1; A.beta2 = ctx->hp.beta2; A.eps = ctx->hp.eps;
+  A.sigma_min = ctx->hp.sigma_min; A.terms = ctx->hp.terms; A.adam = adam ? 1 : 0;
+  A.perm = ctx->d_perm; A.w = ctx->d_w; A.lat = ctx->d_lat; A.cls = ctx->d_cls; A.seg = ctx->d_fseg;
+  A.finc = ctx->d_finc; A.chunk = ctx->d_chunk; A.cptr = ctx->d_cptr;
+  A.nchunk = P.nchunk;
+  A.in_ptr = ctx->d_in_ptr; A.fin = ctx->d_fin; A.out_ptr = ctx->d_out_ptr; A.fout = ctx->d_fout;
+  A.bin_ptr = ctx->d_bin_ptr; A.fbin = ctx->d_fbin; A.bout_ptr = ctx->d_bout_ptr; A.fbout = ctx->d_fbout;
+  A.limit = ctx->d_limit;
+  A.mu = const_cast<float *>(mu); A.sg = const_cast<float *>(sg);
+  A.m_mu = m_mu; A.v_mu = v_mu; A.m_sg = m_sg; A.v_sg = v_sg;
+  A.lambda = lambda; A.step = step; A.grad_mu = grad_mu; A.grad_sg = grad_sg;
+  A.loss = loss; A.terms_out = terms; A.status = status;
+  A.xs = ctx->d_xs; A.adm = ctx->d_adm; A.win = ctx->d_win; A.tab = ctx->d_tab; A.part = ctx->d_part;
+  A.partr = ctx->d_partr; A.H = ctx->d_H;
+  A.bar = reinterpret_cast<unsigned *>(ctx->d_facc);
+  A.abort_flag = reinterpret_cast<int32_t *>(ctx->d_facc + ctx->off_abort);
+  A.ctr = reinterpret_cast<unsigned *>(ctx->d_facc + ctx->off_ctr);
+  A.U = reinterpret_cast<long long *>(ctx->d_facc + ctx->off_U);
+  A.fwd = reinterpret_cast<unsigned long long *>(ctx->d_facc + ctx->off_fwd);
+  A.wst = reinterpret_cast<unsigned long long *>(ctx->d_facc + ctx->off_wst);
+  A.nonf = reinterpret_cast<int32_t *>(ctx->d_facc + ctx->off_nonf);
+  A.rstat = ctx->d_rstat; A.prof = prof;
+  const void *fn = (const void *)kernels(ctx->hp.family).fused[(ctx->hp.terms & GAUS_COM) ? 1 : 0];
+  for (int g0 = 0; g0 < ctx->fG; g0 += ctx->fGl) {
+    A.g0 = g0;
+    A.G = std::min(ctx->fGl, ctx->fG - g0);
+    A.ord = ctx->d_ord + (size_t)g0 * P.V * 64;
+    CK(cudaMemsetAsync(ctx->d_facc, 0, ctx->facc_bytes, st), "fused memset");
+    void *args[] = {(void *)&A};
+    CK(cudaLaunchCooperativeKernel(fn, dim3((unsigned)(A.G * A.K)), dim3(kFusedThreads), args, ctx->smem_fused, st),
+       "k_fused launch");
+    if (prof) break;  // phase stamps: the first batch of groups
+  }
+  return GAUS_OK;
+}
+
+// Blocks per restart group and segments of the fused kernel: one wave of blocks of
+// every family's and variant's kernel (so a family switch needs no re-plan), at
+// most one segment per block; 0 when the sizes need the multi-kernel path.
+gaus_status plan_fused(gaus_ctx *ctx, int nsm) {
+  Plan &P = ctx->plan;
+  ctx->fK = 0;
+  if (P.D > 32767) return GAUS_OK;
+  // groups of up to 64 restarts; phases 2-3 rows of RBp lanes; phase 1 rows of RB1
+  // restarts, as many as keep its histogram within the staging buffer's size
+  ctx->fRG = std::min(P.B, kMaxRG);
+  ctx->fG = (P.B + ctx->fRG - 1) / ctx->fRG;
+  ctx->fRBp = 32;  // one node per warp in phases 2 and 3
+  const size_t stage = (size_t)kFusedWarps * kStage * 32 * sizeof(float2);
+  // phase 1: the whole group's histogram when it fits the staging buffer, else rows
+  // of a power of two <= 32 restarts
+  if (2 * (size_t)ctx->fRG * P.Dh * sizeof(unsigned) <= stage) {
+    ctx->fRB1 = ctx->fRG;
+  } else {
+    ctx->fRB1 = 32;
+    while (ctx->fRB1 > 1 && 2 * (size_t)ctx->fRB1 * P.Dh * sizeof(unsigned) > stage) ctx->fRB1 >>= 1;
+  }
+  const size_t hist = 2 * (size_t)ctx->fRB1 * P.Dh * sizeof(unsigned);
+  ctx->smem_fused = std::max(hist, stage);
+  int dev = 0, optin = 0;
+  CK(cudaGetDevice(&dev), "cudaGetDevice");
+  CK(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev), "smem opt-in");
+  int occ = INT32_MAX;
+  for (int fam = GAUS_GAUSSIAN; fam <= GAUS_CAUCHY; ++fam)
+    for (int c = 0; c < 2; ++c) {
+      const void *fn = (const void *)kernels(fam).fused[c];
+      cudaFuncAttributes fa;
+      CK(cudaFuncGetAttributes(&fa, fn), "cudaFuncGetAttributes");
+      if (fa.sharedSizeBytes + ctx->smem_fused > (size_t)optin) return GAUS_OK;
+      CK(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes),
+         "smem attr");
+      int o = 0;
+      CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, kFusedThreads, ctx->smem_fused), "occupancy");
+      occ = std::min(occ, o);
+    }
+  if (occ < 1) return GAUS_OK;
+  const int resident = occ * nsm;
+  if (ctx->fG <= resident) {
+    const int per_group = resident / ctx->fG;
+    // the fewest rows per segment that keep the segment count within one block each
+    plan_fused_segments(P, per_group, ctx->fRB1);
+    ctx->fK = std::min(per_group, P.nfseg);
+    ctx->fGl = ctx->fG;
+  } else {
+    plan_fused_segments(P, 1, ctx->fRB1);
+    ctx->fK = 1;
+    ctx->fGl = resident;
+  }
+  return GAUS_OK;
+}
+
 // The dynamic shared-memory limit is a per-kernel attribute of the process, not of
 // a context: set it to the device maximum once per kernel, so that contexts of
 // different sizes can be used side by side (each launch still requests its own size).
@@ -199,7 +309,9 @@ gaus_status set_smem_attrs(gaus_ctx *ctx) {
   int dev = 0, optin = 0;
   CK(cudaGetDevice(&dev), "cudaGetDevice");
   CK(cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev), "smem opt-in");
-  for (const void *f : fns) {
+  std::vector<const void *> all(fns, fns + sizeof(fns) / sizeof(fns[0]));
+  for (int c = 0; c < 2; ++c) all.push_back((const void *)ks.fused[c]);
+  for (const void *f : all) {
     cudaFuncAttributes fa;
     CK(cudaFuncGetAttributes(&fa, f), "cudaFuncGetAttributes");
     CK(cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes),
@@ -275,6 +387,10 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     size_t w = std::min<size_t>(kTableMax, kTableBytes / per_pt);
     w = std::max<size_t>(4, w & ~(size_t)3);
     ctx->W = (int)w;
+    // fused path: rows of up to kTableMaxFused entries, never longer than a window
+    // can use (D - 1 points and the two sentinels)
+    const size_t wf = std::min<size_t>(std::min<size_t>(kTableMaxFused, (size_t)P.D + 2), kTableBytesFused / per_pt);
+    ctx->fW = (int)std::max<size_t>(4, wf);
   }
   // storage-term kernels: their own restarts-per-row so that the storage histogram
   // (two u32 halves), its difference array and constants fit in shared memory
@@ -371,7 +487,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   ctx->nblk_v = std::max(1, resident((const void *)k_verify_scan, 256, 0) / ctx->Gv) * ctx->Gv;
   TRY(scratch(ctx, &ctx->d_eslot4, 2 * ((size_t)P.E + P.NB) * P.B));
   TRY(scratch(ctx, &ctx->d_win, VB));
-  TRY(scratch(ctx, &ctx->d_tab, VB * ctx->W));
+  TRY(scratch(ctx, &ctx->d_tab, VB * std::max(ctx->W, ctx->fW)));
   TRY(scratch(ctx, &ctx->d_H, (size_t)P.B * P.C * P.Dh));
   TRY(scratch(ctx, &ctx->d_coef, (size_t)P.B * 4));
   TRY(scratch(ctx, &ctx->d_wstat, (size_t)P.B * 2));
@@ -381,6 +497,52 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_status_tmp, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_loss_tmp, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_terms_tmp, (size_t)P.B * GAUS_NT));
+  // fused persistent kernel
+  TRY(plan_fused(ctx, nsm));
+  if (ctx->fK > 0) {
+    TRY(upload(ctx, &ctx->d_fseg, P.fseg));
+    TRY(upload(ctx, &ctx->d_cptr, P.cptr));
+    {
+      int32_t *t4 = nullptr;
+      TRY(upload(ctx, &t4, P.finc));
+      ctx->d_finc = reinterpret_cast<int4 *>(t4);
+      TRY(upload(ctx, &t4, P.chunk));
+      ctx->d_chunk = reinterpret_cast<int4 *>(t4);
+    }
+    int32_t *tmp = nullptr;
+    TRY(upload(ctx, &tmp, P.fout));
+    ctx->d_fout = reinterpret_cast<int2 *>(tmp);
+    TRY(upload(ctx, &tmp, P.fin));
+    ctx->d_fin = reinterpret_cast<int2 *>(tmp);
+    TRY(upload(ctx, &tmp, P.fbin));
+    ctx->d_fbin = reinterpret_cast<int2 *>(tmp);
+    TRY(upload(ctx, &tmp, P.fbout));
+    ctx->d_fbout = reinterpret_cast<int2 *>(tmp);
+    TRY(scratch(ctx, &ctx->d_xs, VB));
+    TRY(scratch(ctx, &ctx->d_adm, VB));
+    TRY(scratch(ctx, &ctx->d_part, (size_t)std::max(1, P.nchunk) * P.B));
+    TRY(scratch(ctx, &ctx->d_partr, (size_t)std::max(1, P.nchunk) * P.B));
+    TRY(scratch(ctx, &ctx->d_rstat, (size_t)P.B * 2));
+    {
+      // every node's restart order starts as the identity (restart l + 32 q in pass q)
+      std::vector<signed char> ord((size_t)ctx->fG * P.V * 64);
+      for (size_t i = 0; i < ord.size(); ++i) {
+        const int r = (int)(i % 64);
+        ord[i] = (signed char)(r < ctx->fRG ? r : -1);
+      }
+      TRY(upload(ctx, &ctx->d_ord, ord));
+    }
+    auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    size_t off = al((size_t)ctx->fG * sizeof(unsigned));
+    ctx->off_ctr = off; off = al(off + 2 * (size_t)ctx->fG * sizeof(unsigned));
+    ctx->off_abort = off; off = al(off + sizeof(int32_t));
+    ctx->off_U = off; off = al(off + 2 * (size_t)P.B * P.C * P.Dh * sizeof(long long));
+    ctx->off_fwd = off; off = al(off + 2 * (size_t)P.B * 3 * sizeof(unsigned long long));
+    ctx->off_wst = off; off = al(off + 2 * (size_t)P.B * 2 * sizeof(unsigned long long));
+    ctx->off_nonf = off; off = al(off + 2 * (size_t)P.B * sizeof(int32_t));
+    ctx->facc_bytes = off;
+    TRY(scratch(ctx, &ctx->d_facc, ctx->facc_bytes));
+  }
   CK(cudaDeviceSynchronize(), "setup sync");
   return GAUS_OK;
 }
@@ -443,6 +605,59 @@ gaus_status capture_iterations(gaus_ctx *ctx, const gaus_state *S, int iters, cu
     *out = nullptr;
     return cuda_fail(ctx, e, "graph instantiate");
   }
+  return GAUS_OK;
+}
+
+// Per-block phase stamps of n_iters fused iterations, summarised (ms, means over
+// the iterations): [0..2] critical path of phases 1-3 (last block done - first
+// block started), [3..5] mean block time per phase, [6..7] barrier latency (last
+// arrival to first release), [8] iteration time, [9..11] slowest block per phase.
+gaus_status fused_phases(gaus_ctx *ctx, int n_iters, const gaus_state *S, double *out) {
+  for (int k = 0; k < 12; ++k) out[k] = 0.0;
+  if (n_iters <= 0) return GAUS_OK;
+  const int nb = std::min(ctx->fGl, ctx->fG) * ctx->fK;
+  const size_t need = (size_t)n_iters * nb * 6;
+  if ((size_t)ctx->prof_cap < need) {
+    if (ctx->d_prof) cudaFree(ctx->d_prof);
+    ctx->d_prof = nullptr;
+    ctx->prof_cap = 0;
+    CK(cudaMalloc((void **)&ctx->d_prof, need * sizeof(unsigned long long)), "cudaMalloc prof");
+    ctx->prof_cap = (int)need;
+  }
+  TRY(enqueue_fused(ctx, ctx->stream, n_iters, true, S->mu, S->sigma, S->m_mu, S->v_mu, S->m_sigma, S->v_sigma,
+                    S->lambda, S->step, nullptr, nullptr, S->loss, S->terms, S->status, ctx->d_prof));
+  std::vector<unsigned long long> ts(need);
+  CK(cudaMemcpyAsync(ts.data(), ctx->d_prof, need * sizeof(unsigned long long), cudaMemcpyDeviceToHost, ctx->stream),
+     "prof copy");
+  CK(cudaStreamSynchronize(ctx->stream), "profile sync");
+  auto at = [&](int it, int b, int q) { return (double)ts[((size_t)it * nb + b) * 6 + q]; };
+  for (int it = 0; it < n_iters; ++it) {
+    double mn[6], mx[6], sum[3] = {0, 0, 0}, wmx[3] = {0, 0, 0};
+    for (int q = 0; q < 6; ++q) { mn[q] = 1e300; mx[q] = -1e300; }
+    for (int b = 0; b < nb; ++b) {
+      for (int q = 0; q < 6; ++q) { mn[q] = std::min(mn[q], at(it, b, q)); mx[q] = std::max(mx[q], at(it, b, q)); }
+      for (int q = 0; q < 3; ++q) {
+        const double w = at(it, b, 2 * q + 1) - at(it, b, 2 * q);
+        sum[q] += w;
+        wmx[q] = std::max(wmx[q], w);
+      }
+    }
+    out[0] += mx[1] - mn[0];
+    out[1] += mx[3] - mn[2];
+    out[2] += mx[5] - mn[4];
+    for (int q = 0; q < 3; ++q) { out[3 + q] += sum[q] / nb; out[9 + q] += wmx[q]; }
+    out[6] += mn[2] - mx[1];
+    out[7] += mn[4] - mx[3];
+    double next = 0;
+    if (it + 1 < n_iters) {
+      next = 1e300;
+      for (int b = 0; b < nb; ++b) next = std::min(next, at(it + 1, b, 0));
+    } else {
+      next = mx[5];
+    }
+    out[8] += next - mn[0];
+  }
+  for (int k = 0; k < 12; ++k) out[k] *= 1e-6 / n_iters;
   return GAUS_OK;
 }
 
@@ -531,6 +746,10 @@ gaus_status gaus_loss_grad(gaus_ctx *ctx, const float *mu, const float *sigma, c
     ctx->err = "gaus_loss_grad: NULL pointer";
     return GAUS_EINVAL;
   }
+  if (fused_ok(ctx))
+    return enqueue_fused(ctx, ctx->stream, 1, false, mu, sigma, nullptr, nullptr, nullptr, nullptr,
+                         const_cast<float *>(lambda), nullptr, grad_mu, grad_sigma, loss, terms,
+                         status ? status : ctx->d_status_tmp, nullptr);
   return enqueue_iteration(ctx, ctx->stream, mu, sigma, const_cast<float *>(lambda), false, grad_mu, grad_sigma,
                            loss, terms, status ? status : ctx->d_status_tmp, nullptr);
 }
@@ -563,6 +782,9 @@ gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *S) {
     return GAUS_EINVAL;
   }
   if (n_iters == 0) return GAUS_OK;
+  if (fused_ok(ctx))
+    return enqueue_fused(ctx, ctx->stream, n_iters, true, S->mu, S->sigma, S->m_mu, S->v_mu, S->m_sigma, S->v_sigma,
+                         S->lambda, S->step, nullptr, nullptr, S->loss, S->terms, S->status, nullptr);
   // two captured graphs of the same iteration: kGraphUnroll iterations, and one
   const uint64_t h = state_hash(S);
   if (!ctx->gexec || ctx->ghash != h) {
@@ -584,6 +806,15 @@ gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_stat
     ctx->err = "gaus_profile_iterate: NULL pointer or n_iters < 0";
     return GAUS_EINVAL;
   }
+  if (fused_ok(ctx)) {
+    double ph[12];
+    TRY(fused_phases(ctx, n_iters, S, ph));
+    // iteration start to the first barrier's release, to the second's, to the next start
+    ms_out[0] += ph[0] + ph[6];
+    ms_out[1] += ph[1] + ph[7];
+    ms_out[3] += ph[8] - (ph[0] + ph[6]) - (ph[1] + ph[7]);
+    return GAUS_OK;
+  }
   constexpr int kEv = 5;  // before k_nodes, before / after k_edges, after finalize, after update
   std::vector<cudaEvent_t> ev(kEv * (size_t)n_iters);
   for (auto &e : ev) CK(cudaEventCreate(&e), "event create");
@@ -604,6 +835,20 @@ gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_stat
   if (e != cudaSuccess) return cuda_fail(ctx, e, "profile sync");
   for (int k = 0; k < kEv - 1; ++k) ms_out[k] += n_iters ? acc[k] / n_iters : 0.0;
   return GAUS_OK;
+}
+
+gaus_status gaus_profile_phases(gaus_ctx *ctx, int32_t n_iters, const gaus_state *S, double *out) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!S || !out || n_iters < 0 || !S->mu || !S->sigma || !S->m_mu || !S->v_mu || !S->m_sigma || !S->v_sigma ||
+      !S->lambda || !S->step || !S->loss || !S->terms || !S->status) {
+    ctx->err = "gaus_profile_phases: NULL pointer or n_iters < 0";
+    return GAUS_EINVAL;
+  }
+  if (!fused_ok(ctx)) {
+    ctx->err = "gaus_profile_phases: these terms or sizes run the multi-kernel path";
+    return GAUS_EINVAL;
+  }
+  return fused_phases(ctx, n_iters, S, out);
 }
 
 gaus_status gaus_round(gaus_ctx *ctx, const float *mu, int32_t *sched) {
@@ -737,6 +982,7 @@ void gaus_destroy(gaus_ctx *ctx) {
   drop_graph(ctx);
   if (ctx->side) cudaStreamSynchronize(ctx->side);
   for (void *p : ctx->allocs) cudaFree(p);
+  if (ctx->d_prof) cudaFree(ctx->d_prof);
   if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
   if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
   if (ctx->side) cudaStreamDestroy(ctx->side);

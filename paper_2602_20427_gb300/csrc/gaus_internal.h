@@ -22,10 +22,18 @@ constexpr int kReduceSpans = 1024;             // segment spans staged per k_red
 constexpr int kMaxRB = 16;
 constexpr int kTableMax = 32;                    // points per CDF table row, at most
 constexpr size_t kTableBytes = (size_t)64 << 20;  // CDF table size bound
+// The fused kernel's table ([node][point][restart]: a row's entries are B floats
+// apart, so a longer row costs address space, not cache lines): up to 64 points
+// per row and 256 MB.
+constexpr int kTableMaxFused = 64;
+constexpr size_t kTableBytesFused = (size_t)256 << 20;
 // Fixed-point scale of the usage histograms and forward sums: values * 2^32 in int64.
 constexpr double kInvFix = 1.0 / 4294967296.0;
 // Limits checked by gaus_create.
 constexpr int kMaxClasses = 16;
+// Incident edges per work item of the fused kernel's edge phase (longer lists are
+// cut into several items, so that no item is much longer than the others).
+constexpr int kChunkEdges = 4;
 
 // Host-side plan produced by plan_problem() (pure C++, no CUDA).
 struct Plan {
@@ -57,6 +65,20 @@ struct Plan {
   std::vector<int32_t> cls_seg_ptr;       // C + 1, segments of class c
   int nseg = 0;
   // caller-order data for the integer kernels
+  // fused kernel: incident edges by internal id -- in-edges (producer, Lat(producer)),
+  // out-edges (consumer, Lat(producer)), back edges into i (j, shift) and out of j
+  // (i, shift); int2 pairs
+  std::vector<int32_t> fin, fout, fbin, fbout;
+  // fused kernel segments (same layout as seg): start, end, class
+  std::vector<int32_t> fseg;
+  // fused kernel's edge phase: every node's incident edges in one list of int4
+  // (neighbour, latency or shift, kind 0 in / 1 out / 2 back in / 3 back out, 0),
+  // cut into chunks of at most kChunkEdges: int4 (node, first entry, entries, 0),
+  // in claim order (the most entries first; .w = the chunk's index in node-major
+  // order, cptr (V + 1) the node-major chunk indices of each node); p2ord: that order
+  std::vector<int32_t> finc, chunk, cptr, p2ord;
+  int nchunk = 0;
+  int nfseg = 0;
   std::vector<int32_t> lvl_ptr, lvl_nodes;           // nodes (caller ids) by level
   std::vector<int32_t> lq_ptr, lq_src, lq_lat;       // predecessors by level-order position
   std::vector<int32_t> cpred_ptr, cpred_src;         // CSC by caller consumer id
@@ -74,6 +96,9 @@ struct Plan {
 // Returns GAUS_OK or an error with a message.
 gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err);
 void plan_segments(Plan &P, int target_blocks, int RB);
+// Segments of the fused kernel: about target_per_group segments of whole rows of
+// RB-restart warp rows, each inside one class (written to P.fseg / P.nfseg).
+void plan_fused_segments(Plan &P, int target_per_group, int RB);
 gaus_status check_hparams(const gaus_hparams *hp, std::string *err);
 float family_window_k(float window_k, int family);
 
@@ -142,6 +167,24 @@ struct gaus_ctx {
   int32_t *d_nonfinite = nullptr;  // B flags
   int32_t *d_status_tmp = nullptr; // B
   float *d_loss_tmp = nullptr, *d_terms_tmp = nullptr;
+  // fused persistent iteration (gaus_fused.cuh): blocks per restart group, groups
+  // per cooperative launch, dynamic shared memory; 0 = the terms or sizes need the
+  // multi-kernel path (storage term, continuous dependency penalty, D > 32767)
+  int fK = 0, fGl = 0;
+  int fRG = 1, fRBp = 1, fRB1 = 1, fG = 1;
+  int fW = 0;  // table row length of the fused path ([node][point][restart] layout)  // restarts per group, lanes per row (phases 2-3, phase 1), groups
+  size_t smem_fused = 0;
+  int32_t *d_fseg = nullptr, *d_cptr = nullptr;
+  int4 *d_finc = nullptr, *d_chunk = nullptr;
+  signed char *d_ord = nullptr;  // fG * V * 64 restart orders (identity at creation)
+  int2 *d_fin = nullptr, *d_fout = nullptr, *d_fbin = nullptr, *d_fbout = nullptr;
+  float2 *d_xs = nullptr, *d_partr = nullptr;
+  float4 *d_adm = nullptr, *d_part = nullptr;
+  double *d_rstat = nullptr;
+  unsigned char *d_facc = nullptr;  // group barriers, abort flag and the parity-buffered accumulators
+  size_t facc_bytes = 0, off_ctr = 0, off_abort = 0, off_U = 0, off_fwd = 0, off_wst = 0, off_nonf = 0;
+  unsigned long long *d_prof = nullptr;
+  int prof_cap = 0;
   // captured iteration
   cudaGraphExec_t gexec = nullptr, gexec_n = nullptr;  // one iteration, kGraphUnroll iterations
   gaus_state gstate{};

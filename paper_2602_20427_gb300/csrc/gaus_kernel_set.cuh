@@ -4,6 +4,7 @@
 // (gaus_family.cu compiled once per family), so that the builds run side by side.
 #pragma once
 
+#include "gaus_fused.cuh"
 #include "gaus_kernels.cuh"
 
 namespace gaus {
@@ -12,6 +13,7 @@ using NodeKernel = void (*)(const IterArgs);
 using EdgeKernel = void (*)(const IterArgs);
 using UpdKernel = void (*)(const UpdArgs);
 using RegKernel = void (*)(const RegArgs);
+using FusedKernel = void (*)(const FusedArgs);
 
 constexpr int kEdgeVariants = 12;
 
@@ -20,6 +22,7 @@ struct KernelSet {
   EdgeKernel edges[kEdgeVariants] = {};  // by edge_variant()
   UpdKernel update[4] = {};              // [2 * adam + hist]
   RegKernel reg_fwd = nullptr, reg_bwd = nullptr;
+  FusedKernel fused[2] = {};             // [com]
 };
 
 // Edge-pass variant of a term mask: which of the dependency, communication and
@@ -52,6 +55,8 @@ KernelSet make_kernel_set() {
   s.update[3] = k_update<kFam, true, true>;
   s.reg_fwd = k_reg_fwd<kFam>;
   s.reg_bwd = k_reg_bwd<kFam>;
+  s.fused[0] = k_fused<kFam, false>;
+  s.fused[1] = k_fused<kFam, true>;
   return s;
 }
 

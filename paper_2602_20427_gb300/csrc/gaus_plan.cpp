@@ -101,6 +101,43 @@ void plan_segments(Plan &P, int target_blocks, int RB) {
   P.nseg = (int)P.seg.size() / 3;
 }
 
+void plan_fused_segments(Plan &P, int target_per_group, int RB) {
+  const int V = P.V, C = P.C;
+  const int target = std::max(1, target_per_group);
+  // the 16-bit halves of the shared-memory usage histogram cannot overflow:
+  // segment length * max demand * ceil(D / Dh) * 2^16 < 2^32
+  int maxw = 1;
+  for (int v = 0; v < V; ++v) maxw = std::max(maxw, P.c_dem[v]);
+  const long folds = (P.D + P.Dh - 1) / P.Dh;
+  const int cap = (int)std::max(1L, 32768L / ((long)maxw * folds));
+  std::vector<int> ncls(C, 0);
+  for (int i = 0; i < V; ++i) ncls[P.cls[i]]++;
+  auto count = [&](int len) {
+    long n = 0;
+    for (int c = 0; c < C; ++c) n += (ncls[c] + len - 1) / len;
+    return n;
+  };
+  // the shortest segments (whole warp rows of 32 / RB nodes) whose count is at most
+  // one per block of the group, unless the overflow cap forces more
+  const int npw = std::max(1, 32 / RB);
+  int seglen = std::max(1, (V + target - 1) / target);
+  seglen = (seglen + npw - 1) / npw * npw;
+  while (seglen < cap && count(seglen) > target) seglen += npw;
+  seglen = std::max(1, std::min(seglen, cap));
+  P.fseg.clear();
+  int i0 = 0;
+  for (int c = 0; c < C; ++c) {
+    const int i1 = i0 + ncls[c];
+    for (int s = i0; s < i1; s += seglen) {
+      P.fseg.push_back(s);
+      P.fseg.push_back(std::min(i1, s + seglen));
+      P.fseg.push_back(c);
+    }
+    i0 = i1;
+  }
+  P.nfseg = (int)P.fseg.size() / 3;
+}
+
 gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, std::string *err) {
   if (!p) return fail(err, GAUS_EINVAL, "problem is NULL");
   const int V = p->V, E = p->E, C = p->C, NB = p->n_back;
@@ -283,6 +320,62 @@ gaus_status plan_problem(const gaus_problem *p, int target_blocks, Plan *out, st
       P.bout_dst[b] = i; P.bout_shift[b] = shift;
       P.bin_eslot[a] = b;
     }
+  }
+  // incident edges by internal id (fused kernel)
+  P.fin.resize(2 * (size_t)E);
+  P.fout.resize(2 * (size_t)E);
+  for (int e = 0; e < E; ++e) {
+    P.fin[2 * (size_t)e] = P.inv[P.in_src[e]];
+    P.fin[2 * (size_t)e + 1] = P.in_lat[e];
+  }
+  for (int i = 0; i < V; ++i)
+    for (int o = P.out_ptr[i]; o < P.out_ptr[i + 1]; ++o) {
+      P.fout[2 * (size_t)o] = P.inv[P.out_dst[o]];
+      P.fout[2 * (size_t)o + 1] = P.lat[i];
+    }
+  P.fbin.resize(2 * (size_t)NB);
+  P.fbout.resize(2 * (size_t)NB);
+  for (int q = 0; q < NB; ++q) {
+    P.fbin[2 * (size_t)q] = P.inv[P.bin_src[q]];
+    P.fbin[2 * (size_t)q + 1] = P.bin_shift[q];
+    P.fbout[2 * (size_t)q] = P.inv[P.bout_dst[q]];
+    P.fbout[2 * (size_t)q + 1] = P.bout_shift[q];
+  }
+  // the fused kernel's edge phase: incident-edge lists, chunks, claim order (the
+  // chunks with the most edges first, so that the last items claimed are short)
+  {
+    P.finc.clear();
+    P.chunk.clear();
+    P.cptr.assign(V + 1, 0);
+    auto add = [&](int nb, int L, int kind) {
+      P.finc.push_back(nb); P.finc.push_back(L); P.finc.push_back(kind); P.finc.push_back(0);
+    };
+    for (int i = 0; i < V; ++i) {
+      const int first = (int)P.finc.size() / 4;
+      for (int e = P.in_ptr[i]; e < P.in_ptr[i + 1]; ++e) add(P.inv[P.in_src[e]], P.in_lat[e], 0);
+      for (int o = P.out_ptr[i]; o < P.out_ptr[i + 1]; ++o) add(P.inv[P.out_dst[o]], P.lat[i], 1);
+      for (int q = P.bin_ptr[i]; q < P.bin_ptr[i + 1]; ++q) add(P.inv[P.bin_src[q]], P.bin_shift[q], 2);
+      for (int q = P.bout_ptr[i]; q < P.bout_ptr[i + 1]; ++q) add(P.inv[P.bout_dst[q]], P.bout_shift[q], 3);
+      const int last = (int)P.finc.size() / 4;
+      for (int c = first; c < last; c += kChunkEdges) {
+        P.chunk.push_back(i); P.chunk.push_back(c); P.chunk.push_back(std::min(kChunkEdges, last - c));
+        P.chunk.push_back(0);
+      }
+      P.cptr[i + 1] = (int)P.chunk.size() / 4;
+    }
+    P.nchunk = (int)P.chunk.size() / 4;
+    P.p2ord.resize(P.nchunk);
+    std::iota(P.p2ord.begin(), P.p2ord.end(), 0);
+    std::stable_sort(P.p2ord.begin(), P.p2ord.end(),
+                     [&](int a, int b) { return P.chunk[4 * (size_t)a + 2] > P.chunk[4 * (size_t)b + 2]; });
+    // descriptors in claim order, with the chunk index (where its partials go)
+    std::vector<int32_t> claim(P.chunk.size());
+    for (int q = 0; q < P.nchunk; ++q) {
+      const int c = P.p2ord[q];
+      for (int k = 0; k < 3; ++k) claim[4 * (size_t)q + k] = P.chunk[4 * (size_t)c + k];
+      claim[4 * (size_t)q + 3] = c;
+    }
+    P.chunk.swap(claim);
   }
   P.unit_lat = 1;
   for (int i = 0; i < V; ++i)
