@@ -880,7 +880,10 @@ __device__ __forceinline__ int p1_lane(const FusedArgs &A, FusedShared &S, unsig
   }
   const int nact = __popc(__ballot_sync(FULL, valid));
   const int mean = nact ? __reduce_add_sync(FULL, max(n, 0)) / nact : 0;
-  const bool is_long = valid && n > max(8, 2 * mean + 8);
+  // long: well above the warp's typical window, or above the staging capacity (a pass
+  // of the sorted order can hold many long windows, which would make every lane's
+  // loop run to the longest)
+  const bool is_long = valid && n > min(kStage, max(8, 2 * mean + 8));
   const int nl = is_long ? -1 : n;
   const int nmax = __reduce_max_sync(FULL, nl);
   // table row: [node][point][restart], so that a warp's restarts write and read
@@ -1189,7 +1192,9 @@ __global__ void __launch_bounds__(kFusedThreads, 1) k_fused(const FusedArgs A) {
         const bool actk[3] = {on_dep, on_rv, on_rec};
         S.coef[tid][0] = on_dep ? (float)((double)S.lam[tid][GAUS_K_DEP] + (double)A.rho * Vk[0]) : 0.f;
         S.coef[tid][1] = on_rec ? (float)((double)S.lam[tid][GAUS_K_REC] + (double)A.rho * Vk[2]) : 0.f;
-        if (k == 0) {
+        if (tid % A.K == k) {
+          // the loss and terms of restart bb: by one block per restart, so that no
+          // block's items wait for all of them
           double L = 0.0;
           if (on & GAUS_RES_OBJ) L += (double)A.w_res * lse;
           if (on & GAUS_COM) L += (double)A.alpha * lcom;

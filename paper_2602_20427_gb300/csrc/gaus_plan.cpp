@@ -109,32 +109,47 @@ void plan_fused_segments(Plan &P, int target_per_group, int RB) {
   int maxw = 1;
   for (int v = 0; v < V; ++v) maxw = std::max(maxw, P.c_dem[v]);
   const long folds = (P.D + P.Dh - 1) / P.Dh;
-  const int cap = (int)std::max(1L, 32768L / ((long)maxw * folds));
+  const long cap = std::max(1L, 32768L / ((long)maxw * folds));
+  // estimated work of each node in phases 1 and 3: a node without predecessors starts
+  // at the horizon's lower edge, where the window's clipped mass leaves sigma little
+  // gradient, and keeps a wider window through a run (about five times the others'
+  // points late in a run of the logic-network workload)
+  std::vector<long> wt(V);
+  long total = 0;
+  for (int i = 0; i < V; ++i) {
+    wt[i] = P.in_ptr[i + 1] > P.in_ptr[i] ? 1 : 5;
+    total += wt[i];
+  }
   std::vector<int> ncls(C, 0);
   for (int i = 0; i < V; ++i) ncls[P.cls[i]]++;
-  auto count = [&](int len) {
-    long n = 0;
-    for (int c = 0; c < C; ++c) n += (ncls[c] + len - 1) / len;
-    return n;
-  };
-  // the shortest segments (whole warp rows of 32 / RB nodes) whose count is at most
-  // one per block of the group, unless the overflow cap forces more
+  // segments of about total / target weight each, cut at class boundaries and at the
+  // overflow cap; the budget grows until the segments fit one block each (unless the
+  // cap forces more)
   const int npw = std::max(1, 32 / RB);
-  int seglen = std::max(1, (V + target - 1) / target);
-  seglen = (seglen + npw - 1) / npw * npw;
-  while (seglen < cap && count(seglen) > target) seglen += npw;
-  seglen = std::max(1, std::min(seglen, cap));
-  P.fseg.clear();
-  int i0 = 0;
-  for (int c = 0; c < C; ++c) {
-    const int i1 = i0 + ncls[c];
-    for (int s = i0; s < i1; s += seglen) {
-      P.fseg.push_back(s);
-      P.fseg.push_back(std::min(i1, s + seglen));
-      P.fseg.push_back(c);
+  auto cut = [&](long budget, std::vector<int32_t> *out) {
+    long nseg = 0;
+    int i0 = 0;
+    for (int c = 0; c < C; ++c) {
+      const int i1 = i0 + ncls[c];
+      int s = i0;
+      while (s < i1) {
+        long w = 0;
+        int e = s;
+        while (e < i1 && (e == s || (w + wt[e] <= budget && e - s < cap))) w += wt[e++];
+        // whole warp rows where the budget allows
+        if (e < i1 && e - s > npw) e = s + std::max(npw, (e - s) / npw * npw);
+        if (out) { out->push_back(s); out->push_back(e); out->push_back(c); }
+        ++nseg;
+        s = e;
+      }
+      i0 = i1;
     }
-    i0 = i1;
-  }
+    return nseg;
+  };
+  long budget = std::max(1L, (total + target - 1) / target);
+  while (cut(budget, nullptr) > target && budget < total) budget += std::max(1L, budget / 64);
+  P.fseg.clear();
+  cut(budget, &P.fseg);
   P.nfseg = (int)P.fseg.size() / 3;
 }
 
