@@ -54,6 +54,14 @@ constexpr int kFusedThreads = 768;  // one block per SM: its warps balance the p
 constexpr int kFusedWarps = kFusedThreads / 32;
 constexpr int kStage = 32;  // own window points staged per lane in phase 2 (C and density)
 constexpr int kMaxRG = 64;  // restarts per group
+// CDF table layout: [node][point][restart] (a warp's restarts write neighbouring
+// words) or [node][restart][point] (a lane's consecutive points share a line)
+constexpr bool kTabPointMajor = true;
+// Table row of (node, restart) and the distance between its entries.
+__device__ __forceinline__ size_t tab_row(int W, int B, int node, int b) {
+  return kTabPointMajor ? (size_t)node * W * B + b : ((size_t)node * B + b) * W;
+}
+__device__ __forceinline__ size_t tab_stride(int B) { return kTabPointMajor ? (size_t)B : 1; }
 // Phase-2 items whose own window exceeds the staging capacity, queued per block and
 // done by all its warps after the block's chunks (a node's long windows would
 // otherwise run one after another in one warp).
@@ -205,76 +213,71 @@ struct Own {
 };
 
 // Consumer side of an edge u -> v (own = v), Lat = L, or of a back edge j -> i
-// (own = i, L = Lat(j) - k II):
+// (own = i, L = Lat(j) - k II; kBack):
 //   V_e = 1 - C_u(b_v + 1 - L) + sum_{t in own} C_v(t) P_u(t + 1 - L)
 //   dV_e/dC_v(t) = P_u(t + 1 - L);  L_com part sum_{t in own} C_u(t) (1 - C_v(t))
 //   dL_com/dC_v(t) = -C_u(t)
 // Visits only the own points where a term can be nonzero (warp-wide trip count).
-template <int kFam, bool kCom, bool kTab>
-__device__ __forceinline__ void cons_side(const Own &O, const FNb<kFam> &U, int L, bool fw, bool bk, bool dep,
-                                          float alpha, float &Ad, float &Bd, float &Ao, float &Bo, float &Ar,
-                                          float &Br, float &fd, float &fc, float &fr) {
+// kL1: L = 1, so C_u(t) is the bin mass's upper value (no second table read).
+template <int kFam, bool kCom, bool kTab, bool kBack, bool kL1>
+__device__ __forceinline__ void cons_side(const Own &O, const FNb<kFam> &U, int L, bool on, bool dep, float alpha,
+                                          float &Ad, float &Bd, float &Ao, float &Bo, float &fd, float &fc) {
   const int nv = O.b - O.a + 1;
   int jlo = 0, jhi = -1;
-  if (fw) {
-    jlo = max(0, U.a + min(dep ? L - 1 : 0, 0) - O.a);
-    jhi = kCom ? nv - 1 : min(nv - 1, U.b + L - O.a);
-  } else if (bk) {
-    jlo = max(0, U.a + L - 1 - O.a);
-    jhi = min(nv - 1, U.b + L - O.a);
+  if (on) {
+    if (kBack) {
+      jlo = max(0, U.a + L - 1 - O.a);
+      jhi = min(nv - 1, U.b + L - O.a);
+    } else {
+      jlo = max(0, U.a + min(dep ? L - 1 : 0, 0) - O.a);
+      jhi = kCom ? nv - 1 : min(nv - 1, U.b + L - O.a);
+    }
   }
   const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
   const int cmax = __reduce_max_sync(0xffffffffu, cnt);
   float c_lo = cnt ? U.template val<kTab>(O.a + jlo - L) : 0.f;
+  const float z0 = ((float)(O.a + jlo) + 0.5f - O.mu) * O.inv;  // z of the first point; then + inv per point
   for (int k2 = 0; k2 < cmax; ++k2) {
     if (k2 < cnt) {
       const int j = jlo + k2, t = O.a + j;
       const float c_hi = U.template val<kTab>(t + 1 - L);
       const float p = c_hi - c_lo;
       const float2 cf = O.st[j * 32];
-      const float z = ((float)t + 0.5f - O.mu) * O.inv;
+      const float z = fmaf((float)k2, O.inv, z0);
       const float f = cf.y, zf = z * f;
-      if (bk) {
-        fr += cf.x * p;
-        Ar += p * f;
-        Br += p * zf;
-      } else {
-        if (dep) {
-          fd += cf.x * p;
-          Ad += p * f;
-          Bd += p * zf;
-        }
-        if (kCom) {
-          const float cu = (L == 1) ? c_hi : U.template val<kTab>(t);
-          fc += cu * (1.0f - cf.x);
-          Ao -= alpha * cu * f;
-          Bo -= alpha * cu * zf;
-        }
+      if (kBack || dep) {
+        fd += cf.x * p;
+        Ad += p * f;
+        Bd += p * zf;
+      }
+      if (kCom && !kBack) {
+        const float cu = kL1 ? c_hi : U.template val<kTab>(t);
+        fc += cu * (1.0f - cf.x);
+        Ao -= alpha * cu * f;
+        Bo -= alpha * cu * zf;
       }
       c_lo = c_hi;
     }
   }
   __syncwarp();
-  if ((dep && fw) || bk) {
-    const float tail = 1.0f - U.template val<kTab>(O.b + 1 - L);
-    if (bk) fr += tail; else fd += tail;
-  }
+  if (on && (kBack || dep)) fd += 1.0f - U.template val<kTab>(O.b + 1 - L);
 }
 
-// Producer side of an edge u -> v (own = u, L = Lat(u)), or of a back edge (own = j):
+// Producer side of an edge u -> v (own = u, L = Lat(u)), or of a back edge (own = j;
+// kBack):
 //   dV_e/dC_u(x) = -P_v(x + L), nonzero for x in [a_v - L, b_v + 1 - L]
 //   dL_com/dC_u(x) = 1 - C_v(x), nonzero for x <= b_v
 //   L_com part sum_{x in own, x < a_v} C_u(x) + max(0, a_v - 1 - b_u)
-template <int kFam, bool kCom, bool kTab>
-__device__ __forceinline__ void prod_side(const Own &O, const FNb<kFam> &Vn, int L, bool fw, bool bk, bool dep,
-                                          float alpha, float &Ad, float &Bd, float &Ao, float &Bo, float &Ar,
-                                          float &Br, float &fc) {
+// kL1: L = 1, so C_v(x) is the bin mass's lower value.
+template <int kFam, bool kCom, bool kTab, bool kBack, bool kL1>
+__device__ __forceinline__ void prod_side(const Own &O, const FNb<kFam> &Vn, int L, bool on, bool dep, float alpha,
+                                          float &Ad, float &Bd, float &Ao, float &Bo, float &fc) {
   const int nu = O.b - O.a + 1;
   int jlo = 0, jhi = -1;
-  if (fw || bk) {
+  if (on) {
     jlo = max(0, Vn.a - L - O.a);
     jhi = min(nu - 1, Vn.b + 1 - L - O.a);
-    if (kCom && fw) {
+    if (kCom && !kBack) {
       jlo = 0;
       jhi = max(jhi, min(nu - 1, Vn.b - O.a));
     }
@@ -282,34 +285,30 @@ __device__ __forceinline__ void prod_side(const Own &O, const FNb<kFam> &Vn, int
   const int cnt = jhi >= jlo ? jhi - jlo + 1 : 0;
   const int cmax = __reduce_max_sync(0xffffffffu, cnt);
   float c_lo = cnt ? Vn.template val<kTab>(O.a + jlo + L - 1) : 0.f;
+  const float z0 = ((float)(O.a + jlo) + 0.5f - O.mu) * O.inv;
   for (int k2 = 0; k2 < cmax; ++k2) {
     if (k2 < cnt) {
       const int j = jlo + k2, x = O.a + j;
       const float c_hi = Vn.template val<kTab>(x + L);
       const float2 cf = O.st[j * 32];
-      const float z = ((float)x + 0.5f - O.mu) * O.inv;
+      const float z = fmaf((float)k2, O.inv, z0);
       const float f = cf.y, zf = z * f;
       const float p = c_hi - c_lo;
-      if (bk) {
-        Ar -= p * f;
-        Br -= p * zf;
-      } else {
-        if (dep) {
-          Ad -= p * f;
-          Bd -= p * zf;
-        }
-        if (kCom) {
-          const float cw = (L == 1) ? c_lo : Vn.template val<kTab>(x);
-          Ao += alpha * (1.0f - cw) * f;
-          Bo += alpha * (1.0f - cw) * zf;
-          if (x < Vn.a) fc += cf.x;
-        }
+      if (kBack || dep) {
+        Ad -= p * f;
+        Bd -= p * zf;
+      }
+      if (kCom && !kBack) {
+        const float cw = kL1 ? c_lo : Vn.template val<kTab>(x);
+        Ao += alpha * (1.0f - cw) * f;
+        Bo += alpha * (1.0f - cw) * zf;
+        if (x < Vn.a) fc += cf.x;
       }
       c_lo = c_hi;
     }
   }
   __syncwarp();
-  if (kCom && fw) fc += (float)max(0, Vn.a - 1 - O.b);
+  if (on && kCom && !kBack) fc += (float)max(0, Vn.a - 1 - O.b);
 }
 
 // A neighbour (node ni, restart b) of a phase-2 item from its packed window w:
@@ -320,8 +319,8 @@ __device__ __forceinline__ bool make_nb(const FusedArgs &A, int ni, int b, unsig
   const size_t ix = (size_t)ni * A.B + b;
   N.a = (int)(w & 0xFFFFu);
   N.b = (int)((w >> 16) & 0x7FFFu) - 1;
-  N.row = A.tab + (size_t)ni * A.W * A.B + b;
-  N.stride = A.B;
+  N.row = A.tab + tab_row(A.W, A.B, ni, b);
+  N.stride = (int)tab_stride(A.B);
   N.tab = N.b - N.a + 4 <= A.W;  // n + 3 <= W, as the node pass writes it
   N.mu = 0.f;
   N.inv = 1.f;
@@ -361,22 +360,37 @@ __device__ __forceinline__ void chunk_edges(const FusedArgs &A, int e0, int ne, 
     FNb<kFam> N;
     const bool on = make_nb<kFam>(A, en_a.x, b, w_a, act, N) && act;
     const bool tb = on && N.tab, dr = on && !N.tab;
+    // the entry (and so its kind and latency) is the same on every lane
     if (kind == 0 && (dep || com)) {
-      cons_side<kFam, kCom, true>(O, N, L, tb, false, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fd, fc, fr);
-      if (__any_sync(FULL, dr))
-        cons_side<kFam, kCom, false>(O, N, L, dr, false, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fd, fc, fr);
+      if (L == 1) {
+        cons_side<kFam, kCom, true, false, true>(O, N, L, tb, dep, A.alpha, Ad, Bd, Ao, Bo, fd, fc);
+        if (__any_sync(FULL, dr))
+          cons_side<kFam, kCom, false, false, true>(O, N, L, dr, dep, A.alpha, Ad, Bd, Ao, Bo, fd, fc);
+      } else {
+        cons_side<kFam, kCom, true, false, false>(O, N, L, tb, dep, A.alpha, Ad, Bd, Ao, Bo, fd, fc);
+        if (__any_sync(FULL, dr))
+          cons_side<kFam, kCom, false, false, false>(O, N, L, dr, dep, A.alpha, Ad, Bd, Ao, Bo, fd, fc);
+      }
     } else if (kind == 1 && (dep || com)) {
-      prod_side<kFam, kCom, true>(O, N, L, tb, false, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fc);
-      if (__any_sync(FULL, dr))
-        prod_side<kFam, kCom, false>(O, N, L, dr, false, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fc);
+      if (L == 1) {
+        prod_side<kFam, kCom, true, false, true>(O, N, L, tb, dep, A.alpha, Ad, Bd, Ao, Bo, fc);
+        if (__any_sync(FULL, dr))
+          prod_side<kFam, kCom, false, false, true>(O, N, L, dr, dep, A.alpha, Ad, Bd, Ao, Bo, fc);
+      } else {
+        prod_side<kFam, kCom, true, false, false>(O, N, L, tb, dep, A.alpha, Ad, Bd, Ao, Bo, fc);
+        if (__any_sync(FULL, dr))
+          prod_side<kFam, kCom, false, false, false>(O, N, L, dr, dep, A.alpha, Ad, Bd, Ao, Bo, fc);
+      }
     } else if (kind == 2 && rec) {
-      cons_side<kFam, false, true>(O, N, L, false, tb, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fd, fc, fr);
+      float dummy0 = 0.f, dummy1 = 0.f, dummy2 = 0.f;
+      cons_side<kFam, false, true, true, false>(O, N, L, tb, dep, A.alpha, Ar, Br, dummy0, dummy1, fr, dummy2);
       if (__any_sync(FULL, dr))
-        cons_side<kFam, false, false>(O, N, L, false, dr, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fd, fc, fr);
+        cons_side<kFam, false, false, true, false>(O, N, L, dr, dep, A.alpha, Ar, Br, dummy0, dummy1, fr, dummy2);
     } else if (kind == 3 && rec) {
-      prod_side<kFam, false, true>(O, N, L, false, tb, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fc);
+      float dummy0 = 0.f, dummy1 = 0.f, dummy2 = 0.f;
+      prod_side<kFam, false, true, true, false>(O, N, L, tb, dep, A.alpha, Ar, Br, dummy0, dummy1, dummy2);
       if (__any_sync(FULL, dr))
-        prod_side<kFam, false, false>(O, N, L, false, dr, dep, A.alpha, Ad, Bd, Ao, Bo, Ar, Br, fc);
+        prod_side<kFam, false, false, true, false>(O, N, L, dr, dep, A.alpha, Ar, Br, dummy0, dummy1, dummy2);
     }
     en_a = en_b;
     w_a = w_b;
@@ -888,7 +902,8 @@ __device__ __forceinline__ int p1_lane(const FusedArgs &A, FusedShared &S, unsig
   const int nmax = __reduce_max_sync(FULL, nl);
   // table row: [node][point][restart], so that a warp's restarts write and read
   // neighbouring words
-  float *row = A.tab + (size_t)vi * A.W * B + bs;
+  float *row = A.tab + tab_row(A.W, B, vi, bs);
+  const size_t ts = tab_stride(B);
   const bool tabled = n >= 0 && n + 3 <= A.W;
   if (tabled && !is_long) row[0] = 0.0f;
   float zp = 0.f, qp = 0.f;
@@ -896,7 +911,7 @@ __device__ __forceinline__ int p1_lane(const FusedArgs &A, FusedShared &S, unsig
     const bool pt = j < nl;
     const float zc = ((float)(a + j) + 0.5f - mu) * inv_s;
     const float qc = pt ? Fam<kFam>::tail(zc) : 0.f;
-    if (tabled && j <= nl) row[(size_t)(j + 1) * B] = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;
+    if (tabled && j <= nl) row[(size_t)(j + 1) * ts] = pt ? (zc <= 0.f ? qc : 1.0f - qc) : 1.0f;
     if (hist && j <= nl)
       hist_add(hlo, hhi, fold_bin(a + j, A.II) * cs + hc, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
     zp = zc;
@@ -911,7 +926,7 @@ __device__ __forceinline__ int p1_lane(const FusedArgs &A, FusedShared &S, unsig
     const int l_hc = __shfl_sync(FULL, hc, src), l_b = __shfl_sync(FULL, bs, src), l_vi = __shfl_sync(FULL, vi, src);
     const float l_mu = __shfl_sync(FULL, mu, src), l_inv = __shfl_sync(FULL, inv_s, src);
     const float l_w = __shfl_sync(FULL, wv, src);
-    float *l_row = A.tab + (size_t)l_vi * A.W * B + l_b;
+    float *l_row = A.tab + tab_row(A.W, B, l_vi, l_b);
     const bool l_tabled = l_n + 3 <= A.W;
     if (l_tabled && lane == 0) l_row[0] = 0.0f;
     float z_carry = 0.f, q_carry = 0.f;
@@ -920,7 +935,7 @@ __device__ __forceinline__ int p1_lane(const FusedArgs &A, FusedShared &S, unsig
       const bool pt = pp < l_n;
       const float z = ((float)(l_a + pp) + 0.5f - l_mu) * l_inv;
       const float q = pt ? Fam<kFam>::tail(z) : 0.f;
-      if (l_tabled && pp <= l_n) l_row[(size_t)(pp + 1) * B] = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
+      if (l_tabled && pp <= l_n) l_row[(size_t)(pp + 1) * ts] = pt ? (z <= 0.f ? q : 1.0f - q) : 1.0f;
       float zpv = __shfl_up_sync(FULL, z, 1), qpv = __shfl_up_sync(FULL, q, 1);
       if (lane == 0) { zpv = z_carry; qpv = q_carry; }
       if (hist && pp <= l_n)
