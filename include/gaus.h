@@ -307,10 +307,13 @@ gaus_status gaus_solve(gaus_ctx *ctx, int32_t n_periods, int32_t period, int32_t
  *
  *   usage[b, c, t] = sum over nodes v of class c of demand[v] * P_v^d, summed over the
  *   bins d with d mod II = t (t < II) when II > 0, else d = t (t < D),
- * with P the bin masses of Eq. round truncated to +-window_k * sigma, exactly as
- * gaus_loss_grad computes them (exact fixed-point sums, deterministic).
- *   mu, sigma (V, B) fp32, res_class (V) int32 in 0..C-1, demand (V) int32 in
- *   0..64 or NULL (= 1): DEVICE pointers, read only.
+ * with P_v^d the mass the normal N(mu_v, sigma_v^2) rounds to step d, over the bins
+ * within window_k * sigma of mu (the mass beyond them lumped into the end bins), in
+ * exact fixed-point sums (deterministic), with the same bin-mass arithmetic as
+ * gaus_loss_grad.
+ *   mu, sigma (V, B) fp32, res_class (V) int32 in 0..C-1, demand (V) int32 or NULL
+ *   (= 1): DEVICE pointers, read only.  A demand outside 0..64 is not added: the
+ *   usage row (b, c) of every restart b that met it in class c is written as NaN.
  *   usage (B, C, II or D) fp64 DEVICE pointer, written.
  *   cuda_stream: cudaStream_t of the work (NULL = legacy default stream).
  * Limits: (II or D) * min(B, 32) <= 25,600; at most 1,024 (restart group, class)
@@ -318,7 +321,9 @@ gaus_status gaus_solve(gaus_ctx *ctx, int32_t n_periods, int32_t period, int32_t
  * in the 16 MiB array (EINVAL with a message otherwise, nothing enqueued).  A
  * restart whose mean or sigma is non-finite (or sigma < 1e-30) contributes nothing.
  * The first call on a device looks up the array's device address and sets the
- * kernel's shared-memory limit; make that first call before any stream capture.
+ * kernel's shared-memory limit; make that first call before any stream capture.  A
+ * cudaDeviceReset of that device in the same process invalidates what it looked up:
+ * do not call this entry point on the device again after such a reset.
  * Every call shares the array: calls whose work overlaps on the GPU race and give
  * undefined results.  No cudaMalloc, cudaFree or allocating library routine is
  * called.  Errors: EINVAL, ECUDA (message in gaus_last_error(NULL)). */

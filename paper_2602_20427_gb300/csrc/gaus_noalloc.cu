@@ -35,7 +35,11 @@ namespace {
 using namespace gaus;
 
 constexpr size_t kNoAllocScratchBytes = 16u << 20;  // 16 MiB per device
-constexpr size_t kCounterBytes = 4096;              // one u32 counter per (restart group, class)
+// one u32 completion counter per (restart group, class), then one u32 per (restart
+// group, class) of flags: bit r set when restart r of the group met a demand
+// outside 0..kMaxDemand in that class
+constexpr size_t kCounterBytes = 8192;
+constexpr int kMaxPairs = 1024;
 constexpr int kMaxDevices = 64;
 constexpr int kMaxDemand = 64;
 
@@ -49,16 +53,20 @@ struct UsageArgs {
   const int32_t *cls, *dem;
   int V, B, C, D, II, Dh, RB, G, NC, CL;
   float k_win;
-  unsigned *counters;
+  unsigned *counters, *bad;
   long long *part;
   double *usage;
 };
 
 // Block = (restart group g, class c, node chunk ch).  Lanes are restarts; each
 // warp claims the chunk's nodes in groups of 32 / RB, skips other classes, and adds
-// its bin masses to a shared-memory histogram (exact fixed point).  The block's
-// histogram goes to the scratch array; the last block of (g, c) to finish sums the
-// chunks in a fixed order and writes the usage.
+// its bin masses to a shared-memory histogram (exact fixed point; the bin masses
+// from the same upper-tail evaluation as the context path's node pass).  The
+// block's histogram goes to the scratch array; the last block of (g, c) to finish
+// sums the chunks in a fixed order and writes the usage.  A demand outside
+// 0..kMaxDemand (the bound that keeps the histogram's 16-bit halves from
+// overflowing) is not added: it marks the restart's row of that class, which is
+// then written as NaN.
 __global__ void __launch_bounds__(256) k_usage_noalloc(const UsageArgs A) {
   extern __shared__ __align__(16) unsigned char smem[];
   constexpr unsigned FULL = 0xffffffffu;
@@ -66,10 +74,11 @@ __global__ void __launch_bounds__(256) k_usage_noalloc(const UsageArgs A) {
   unsigned *hlo = reinterpret_cast<unsigned *>(smem);
   unsigned *hhi = hlo + (size_t)Dh * RB;
   __shared__ int s_next, s_last;
+  __shared__ unsigned s_bad;
   const int blk = blockIdx.x, ch = blk % A.NC, gc = blk / A.NC, c = gc % A.C, g = gc / A.C;
   const int v0 = ch * A.CL, v1 = min(A.V, v0 + A.CL);
   for (int i = tid; i < 2 * Dh * RB; i += 256) hlo[i] = 0u;
-  if (tid == 0) s_next = 0;
+  if (tid == 0) { s_next = 0; s_bad = 0u; }
   __syncthreads();
 
   const int lane = tid & 31, r = tid % RB, b = g * RB + r, npw = 32 / RB;
@@ -82,8 +91,13 @@ __global__ void __launch_bounds__(256) k_usage_noalloc(const UsageArgs A) {
     bool valid = b < A.B && v < v1 && A.cls[v] == c;
     const float mu = valid ? A.mu[(size_t)v * A.B + b] : 0.f, sg = valid ? A.sg[(size_t)v * A.B + b] : 1.f;
     valid = valid && usable(mu, sg);
+    const int dm = valid ? (A.dem ? A.dem[v] : 1) : 0;
+    if (valid && (dm < 0 || dm > kMaxDemand)) {
+      atomicOr(&s_bad, 1u << r);
+      valid = false;
+    }
     const float inv_s = valid ? 1.0f / sg : 1.0f;
-    const float wv = valid ? (A.dem ? (float)A.dem[v] : 1.0f) : 0.f;
+    const float wv = valid ? (float)dm : 0.f;
     int a = 0, bw = -2;
     if (valid) window(mu, sg, A.k_win, A.D, a, bw);
     const int n = bw - a + 1;
@@ -92,7 +106,7 @@ __global__ void __launch_bounds__(256) k_usage_noalloc(const UsageArgs A) {
     for (int j = 0; j <= nmax; ++j) {
       const bool pt = j < n;
       const float zc = ((float)(a + j) + 0.5f - mu) * inv_s;
-      const float qc = pt ? 0.5f * erfcf(fabsf(zc) * kInvSqrt2) : 0.f;
+      const float qc = pt ? tail_fast(zc) : 0.f;
       if (j <= n) hist_add(hlo, hhi, fold_bin(a + j, A.II) * RB + r, wv * bin_mass(pt, j == 0, zc, qc, zp, qp));
       zp = zc;
       qp = qc;
@@ -103,6 +117,7 @@ __global__ void __launch_bounds__(256) k_usage_noalloc(const UsageArgs A) {
   long long *mine = A.part + (size_t)blk * Dh * RB;
   for (int i = tid; i < Dh * RB; i += 256)
     mine[i] = (long long)(((unsigned long long)hhi[i] << 16) + (unsigned long long)hlo[i]);
+  if (tid == 0 && s_bad) atomicOr(&A.bad[gc], s_bad);
   __threadfence();
   __syncthreads();
   if (tid == 0) s_last = atomicAdd(&A.counters[gc], 1u) == (unsigned)(A.NC - 1);
@@ -110,12 +125,14 @@ __global__ void __launch_bounds__(256) k_usage_noalloc(const UsageArgs A) {
   if (!s_last) return;
   __threadfence();
   const long long *first = A.part + (size_t)gc * A.NC * Dh * RB;
+  const unsigned bad = __ldcg(&A.bad[gc]);
   for (int i = tid; i < Dh * RB; i += 256) {
     const int d = i / RB, rr = i % RB, bb = g * RB + rr;
     if (bb >= A.B) continue;
     long long acc = 0;
     for (int k = 0; k < A.NC; ++k) acc += __ldcg(first + (size_t)k * Dh * RB + i);
-    A.usage[((size_t)bb * A.C + c) * Dh + d] = (double)acc * kInvFix;
+    A.usage[((size_t)bb * A.C + c) * Dh + d] = ((bad >> rr) & 1u) ? __longlong_as_double(0x7ff8000000000000ll)
+                                                                   : (double)acc * kInvFix;
   }
   if (tid == 0) A.counters[gc] = 0u;
 }
@@ -145,7 +162,7 @@ extern "C" gaus_status gaus_expected_usage_noalloc(const float *mu, const float 
   if (smem > 200 * 1024)
     return fail(GAUS_EINVAL, "gaus_expected_usage_noalloc: histogram length (II or D) times min(B, 32) "
                              "exceeds 25,600");
-  if ((size_t)G * C * sizeof(unsigned) > kCounterBytes)
+  if (G * C > kMaxPairs)
     return fail(GAUS_EINVAL, "gaus_expected_usage_noalloc: more than 1,024 (restart group, class) pairs");
   const size_t per_block = (size_t)Dh * RB * sizeof(long long);
   const size_t cap_blocks = (kNoAllocScratchBytes - kCounterBytes) / per_block;
@@ -165,6 +182,7 @@ extern "C" gaus_status gaus_expected_usage_noalloc(const float *mu, const float 
   void *base = nullptr;
   {
     // once per device, with that device current: the device address of the array
+    // (a cudaDeviceReset in this process invalidates it; see include/gaus.h)
     std::lock_guard<std::mutex> lock(g_setup_mu);
     if (!g_scratch_addr[dev]) {
       void *p = nullptr;
@@ -183,9 +201,10 @@ extern "C" gaus_status gaus_expected_usage_noalloc(const float *mu, const float 
   A.V = V; A.B = B; A.C = C; A.D = D; A.II = II; A.Dh = Dh; A.RB = RB; A.G = G; A.NC = NC; A.CL = CL;
   A.k_win = window_k;
   A.counters = reinterpret_cast<unsigned *>(base);
+  A.bad = A.counters + kMaxPairs;
   A.part = reinterpret_cast<long long *>(reinterpret_cast<unsigned char *>(base) + kCounterBytes);
   A.usage = usage;
-  e = cudaMemsetAsync(A.counters, 0, (size_t)G * C * sizeof(unsigned), st);
+  e = cudaMemsetAsync(A.counters, 0, kCounterBytes, st);
   if (e != cudaSuccess) return fail(GAUS_ECUDA, std::string("cudaMemsetAsync: ") + cudaGetErrorString(e));
   k_usage_noalloc<<<G * C * NC, 256, smem, st>>>(A);
   e = cudaGetLastError();

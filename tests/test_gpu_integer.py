@@ -126,15 +126,28 @@ def test_adam_step_matches_oracle(g):
     lam = torch.full((B, 3), 1e-6, device="cuda")
     th = [mu.astype(np.float64).ravel().copy(), sg.astype(np.float64).ravel().copy()]
     mo = [np.zeros(p.V * B) for _ in range(4)]
+    # the multiplier update of Sec. 3.3, lambda_k <- lambda_k + rho V_k for every active
+    # constraint k (dependency, resource excess, recurrence), others unchanged
+    lam_ref = np.full((B, 3), 1e-6)
+    active = [(oracle.K_DEP, oracle.T_VDEP, bool(p.terms & W.DEP)),
+              (oracle.K_RES, oracle.T_VRES, bool(p.terms & W.RES_VIOL)),
+              (oracle.K_REC, oracle.T_VREC, bool(p.terms & W.REC))]
+    assert any(a for _, _, a in active)
     for step in range(1, 4):
         gm = (rng.normal(size=(p.V, B)) * 10 ** rng.uniform(-3, 1)).astype(np.float32)
         gs = (rng.normal(size=(p.V, B)) * 10 ** rng.uniform(-3, 1)).astype(np.float32)
-        terms = torch.from_numpy(rng.uniform(0, 5, size=(B, 6)).astype(np.float32)).cuda()
+        T = rng.uniform(0, 5, size=(B, 6)).astype(np.float32)
+        terms = torch.from_numpy(T).cuda()
         ctx.adam_step(t["mu"], t["sg"], torch.from_numpy(gm).cuda(), torch.from_numpy(gs).cuda(), *z, lam,
                       terms, step)
         oracle.adam(th[0], gm.astype(np.float64).ravel().copy(), mo[0], mo[1], step, hp.lr)
         oracle.adam(th[1], gs.astype(np.float64).ravel().copy(), mo[2], mo[3], step, hp.lr)
         th[1] = np.maximum(th[1], hp.sigma_min)
+        for k, tk, on in active:
+            if on:
+                lam_ref[:, k] += hp.rho * T[:, tk].astype(np.float64)
+        torch.cuda.synchronize()
+        np.testing.assert_allclose(lam.cpu().numpy(), lam_ref, rtol=1e-6, atol=0)
     torch.cuda.synchronize()
     np.testing.assert_allclose(t["mu"].cpu().numpy().ravel(), th[0], rtol=0, atol=2e-5)
     np.testing.assert_allclose(t["sg"].cpu().numpy().ravel(), th[1], rtol=0, atol=2e-5)
@@ -162,6 +175,41 @@ def test_iterate_equals_separate_calls(g):
     np.testing.assert_allclose(st["sigma"].cpu().numpy(), m["sg"].cpu().numpy(), rtol=0, atol=1e-4)
     np.testing.assert_allclose(st["lambda_"].cpu().numpy(), lam.cpu().numpy(), rtol=1e-5)
     assert np.all(st["step"].cpu().numpy() == 5)
+    ctx.close()
+
+
+def test_iterate_multiplier_update(g):
+    # the fused iteration's multiplier update (Sec. 3.3): after every iteration,
+    # lambda_k = lambda_k(before) + rho V_k for the active constraints, with V_k the
+    # values the iteration reports (exactly, up to the final rounding to float) and
+    # against the oracle's V_k at the same state (within the parity tolerance)
+    p = W.random_layered(3)
+    p.terms = W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL
+    B = 8
+    mu, sg = W.init_state(p, B, 3)
+    hp = g.default_hparams(terms=p.terms, rho=1e-2)
+    ctx = g.Gaus(p, B, hp)
+    st = ctx.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), 1e-3)
+    op = oracle.OracleProblem(p)
+    ohp = oracle.hparams(tau=hp.tau, rho=hp.rho, alpha=hp.alpha, w_res=hp.w_res, w_mem=hp.w_mem, terms=p.terms)
+    for it in range(4):
+        lam0 = st["lambda_"].cpu().numpy().astype(np.float64)
+        m0 = st["mu"].cpu().numpy().astype(np.float64)
+        s0 = st["sigma"].cpu().numpy().astype(np.float64)
+        ctx.iterate(1, st)
+        torch.cuda.synchronize()
+        lam1 = st["lambda_"].cpu().numpy().astype(np.float64)
+        T = st["terms"].cpu().numpy().astype(np.float64)
+        own = lam0.copy()
+        own[:, oracle.K_DEP] += hp.rho * T[:, oracle.T_VDEP]
+        own[:, oracle.K_RES] += hp.rho * T[:, oracle.T_VRES]
+        np.testing.assert_allclose(lam1, own, rtol=2e-7, atol=0)
+        assert np.all(lam1[:, oracle.K_REC] == lam0[:, oracle.K_REC])
+        _, Tref, _, _ = oracle.loss_grad(op, ohp, m0, s0, lam0)
+        ref = lam0.copy()
+        ref[:, oracle.K_DEP] += hp.rho * Tref[:, oracle.T_VDEP]
+        ref[:, oracle.K_RES] += hp.rho * Tref[:, oracle.T_VRES]
+        np.testing.assert_allclose(lam1 - lam0, ref - lam0, rtol=1e-4, atol=2e-5 * hp.rho)
     ctx.close()
 
 

@@ -5,7 +5,9 @@ gaus_loss_grad reports, per restart, the sum over classes of LSE_tau(usage) and
 the summed ReLU excess over the limits; both are recomputed here (float64) from
 the usage that the allocation-free entry point writes, and must agree within the
 tolerance of the other parity tests, on two calls in a row (with different
-inputs, so that nothing left in the shared scratch array can leak through).
+inputs, so that nothing left in the shared scratch array can leak through).  The
+usage itself is checked against the fp64 oracle for several row widths, restart
+groups and demands, and a demand beyond the histogram's bound must show as NaN.
 The file is collected last on purpose: a failure here cannot hide another test.
 """
 import ctypes as C
@@ -31,7 +33,8 @@ def g():
     return g
 
 
-def _usage(g, p, mu, sg, window_k):
+def _usage(g, p, mu, sg, window_k, demand=True):
+    """Call the entry point; demand=False passes NULL (every demand 1)."""
     dev = torch.device("cuda")
     Dh = p.II if p.II > 0 else p.D
     out = torch.full((mu.shape[1], p.C, Dh), -1.0, dtype=torch.float64, device=dev)
@@ -39,8 +42,8 @@ def _usage(g, p, mu, sg, window_k):
          (mu, sg, np.asarray(p.cls, np.int32), np.asarray(p.demand, np.int32))]
     rc = g.lib().gaus_expected_usage_noalloc(
         C.c_void_p(t[0].data_ptr()), C.c_void_p(t[1].data_ptr()), C.c_void_p(t[2].data_ptr()),
-        C.c_void_p(t[3].data_ptr()), C.c_int32(p.V), C.c_int32(mu.shape[1]), C.c_int32(p.C), C.c_int32(p.D),
-        C.c_int32(p.II), C.c_float(window_k), C.c_void_p(out.data_ptr()),
+        C.c_void_p(t[3].data_ptr()) if demand else None, C.c_int32(p.V), C.c_int32(mu.shape[1]),
+        C.c_int32(p.C), C.c_int32(p.D), C.c_int32(p.II), C.c_float(window_k), C.c_void_p(out.data_ptr()),
         C.c_void_p(torch.cuda.current_stream().cuda_stream))
     assert rc == 0, g.lib().gaus_last_error(None)
     torch.cuda.synchronize()
@@ -75,6 +78,45 @@ def test_usage_noalloc_matches_loss_grad_on_two_calls(g, which):
             ref, _ = oracle.expected_hist(op, mu[:, b].astype(np.float64), sg[:, b].astype(np.float64))
             np.testing.assert_allclose(U[b], ref, rtol=1e-5, atol=1e-5)
     ctx.close()
+
+
+@pytest.mark.parametrize("B", [5, 40])
+@pytest.mark.parametrize("demand", ["null", "seeded"])
+def test_usage_noalloc_rows_groups_and_demands(g, B, demand):
+    # B = 5: rows of 8 restarts, four nodes per warp sharing shared-memory cells;
+    # B = 40: two restart groups with their own completion counters; demands NULL
+    # (every demand 1) or seeded integers in 1..64, against the fp64 oracle with the
+    # same demands, on two calls in a row
+    p = W.modulo_loop(5, V=300, levels=15, n_back=10)
+    rng = np.random.default_rng(70 + B)
+    if demand == "seeded":
+        p.demand = rng.integers(1, 65, size=p.V).astype(np.int32)
+    else:
+        p.demand = np.ones(p.V, np.int32)
+    op = oracle.OracleProblem(p)
+    for call in range(2):
+        mu, sg = W.init_state(p, B, seed=80 + call)
+        U = _usage(g, p, mu, sg, 6.0, demand=(demand == "seeded"))
+        for b in sorted({0, B // 2, B - 1}):
+            ref, _ = oracle.expected_hist(op, mu[:, b].astype(np.float64), sg[:, b].astype(np.float64))
+            np.testing.assert_allclose(U[b], ref, rtol=1e-5, atol=1e-5 * max(1.0, float(p.demand.max())))
+
+
+def test_usage_noalloc_flags_a_demand_above_64(g):
+    # a demand the fixed-point histogram cannot hold (65) is not added: the rows of
+    # its class become NaN for every restart, the other classes' rows are unaffected
+    p = W.logic_network(2, V=2000, depth=40)
+    B = 8
+    v = int(np.flatnonzero(np.asarray(p.cls) == 0)[5])
+    p.demand = np.ones(p.V, np.int32)
+    p.demand[v] = 65
+    mu, sg = W.init_state(p, B, seed=90)
+    U = _usage(g, p, mu, sg, 6.0)
+    assert np.all(np.isnan(U[:, 0, :]))
+    assert np.all(np.isfinite(U[:, 1, :]))
+    op = oracle.OracleProblem(p)
+    ref, _ = oracle.expected_hist(op, mu[:, 3].astype(np.float64), sg[:, 3].astype(np.float64))
+    np.testing.assert_allclose(U[3, 1], ref[1], rtol=1e-5, atol=1e-5)
 
 
 def test_usage_noalloc_rejects_oversized_problems(g):
