@@ -231,6 +231,21 @@ gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_stat
  * the multi-kernel path (storage term, continuous dependency penalty, D > 32767). */
 gaus_status gaus_profile_phases(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st, double *out);
 
+/* The execution plan the context chose for its sizes and current hyperparameters
+ * (host only: no CUDA call).  out (host, n entries, n <= 12 written):
+ *   [0] 1 when gaus_iterate and gaus_loss_grad run the persistent fused kernel,
+ *       0 for the multi-kernel path (storage term, continuous dependency penalty,
+ *       D > 32767, or a device that cannot hold one block per restart group);
+ *   [1] fused: cooperative kernel launches per gaus_iterate call (1 unless B
+ *       exceeds the restart groups the device holds at once), else 0;
+ *   [2] multi-kernel path: kernel launches per iteration, else 0;
+ *   [3] restart groups; [4] blocks per restart group; [5] restarts per group;
+ *   [6] points per CDF table row; [7] dynamic shared memory per fused block (bytes);
+ *   [8] streaming multiprocessors of the device; [9] node segments of the fused
+ *   kernel; [10] edge chunks of the fused kernel; [11] threads per fused block.
+ * EINVAL for a NULL context or out, or n < 1. */
+gaus_status gaus_plan_info(const gaus_ctx *ctx, int64_t *out, int32_t n);
+
 /* Round every mean to s = floor(mu + 1/2) (Sec. 3.3 Sampling; exact for every
  * fp32 value) and legalize it: Alg. 1 (clamp to [ASAP, ALAP], then a forward push
  * in topological order with +Lat(u)) when II = 0, Alg. 2 (fixed-point relaxation

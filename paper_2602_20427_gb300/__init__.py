@@ -201,6 +201,16 @@ class Gaus:
                                       C.byref(cp)))
         return asap, alap, cp.value
 
+    PLAN_KEYS = ("fused", "fused_launches_per_call", "launches_per_iteration", "restart_groups",
+                 "blocks_per_group", "restarts_per_group", "table_row_points", "fused_smem_bytes", "sms",
+                 "node_segments", "edge_chunks", "fused_threads")
+
+    def plan_info(self):
+        """The execution plan for the current sizes and hyperparameters (gaus_plan_info)."""
+        out = (C.c_int64 * len(self.PLAN_KEYS))()
+        self._check(lib().gaus_plan_info(self._ctx, out, C.c_int32(len(self.PLAN_KEYS))))
+        return dict(zip(self.PLAN_KEYS, [int(x) for x in out]))
+
     # -- entry points
     def loss_grad(self, mu, sigma, lam, out=None):
         torch = self.torch

@@ -136,6 +136,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
     RA.V = P.V; RA.B = P.B; RA.D = P.D; RA.II = P.II; RA.Dh = P.Dh; RA.RB = ctx->RBr; RA.G = ctx->Gr;
     RA.k_win = ctx->k_win; RA.perm = ctx->d_perm; RA.bits = ctx->d_bits;
     RA.out_ptr = ctx->d_out_ptr; RA.out_dst = ctx->d_out_dst; RA.seg = ctx->d_seg; RA.win = ctx->d_win;
+    RA.qtab = ctx->d_qtab + (size_t)2 * kTailRows * ctx->hp.family;
     RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gown = ctx->d_gown; RA.eslot = ctx->d_eslot;
     ks.reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_fwd launch");
@@ -328,6 +329,7 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   const bool have_dev = cudaGetDevice(&dev) == cudaSuccess &&
                         cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess;
   std::string err;
+  ctx->nsm = nsm;
   gaus_status st = plan_problem(prob, 8 * nsm, &ctx->plan, &err);
   if (st != GAUS_OK) { ctx->err = err; return st; }
   Plan &P = ctx->plan;
@@ -556,6 +558,10 @@ gaus_status alloc_storage_scratch(gaus_ctx *ctx) {
   TRY(scratch(ctx, &ctx->d_Hreg, (size_t)P.B * P.Dh));
   TRY(scratch(ctx, &ctx->d_gown, (size_t)P.V * P.B));
   TRY(scratch(ctx, &ctx->d_eslot, (size_t)std::max(1, P.E) * P.B));
+  TRY(scratch(ctx, &ctx->d_qtab, (size_t)2 * 4 * kTailRows));
+  k_tail_tables<<<(4 * kTailRows + 255) / 256, 256, 0, ctx->stream>>>(ctx->d_qtab);
+  CK(cudaGetLastError(), "k_tail_tables launch");
+  CK(cudaStreamSynchronize(ctx->stream), "k_tail_tables sync");
   return GAUS_OK;
 }
 
@@ -727,6 +733,21 @@ gaus_status gaus_set_hparams(gaus_ctx *ctx, const gaus_hparams *hp) {
   ctx->k_win = family_window_k(hp->window_k, hp->family);
   drop_graph(ctx);
   if (hp->family != old_family) return set_smem_attrs(ctx);
+  return GAUS_OK;
+}
+
+gaus_status gaus_plan_info(const gaus_ctx *ctx, int64_t *out, int32_t n) {
+  if (!ctx || !out || n < 1) return GAUS_EINVAL;
+  const Plan &P = ctx->plan;
+  const bool fused = fused_ok(ctx);
+  const unsigned on = ctx->hp.terms;
+  const int64_t per_iter = 5 + ((on & GAUS_DEP_CF) ? 1 : 0) + ((on & GAUS_REG_OBJ) ? 3 : 0);
+  const int64_t v[12] = {fused ? 1 : 0,
+                         fused ? (ctx->fG + ctx->fGl - 1) / std::max(1, ctx->fGl) : 0,
+                         fused ? 0 : per_iter,
+                         ctx->fG, ctx->fK, ctx->fRG, ctx->fW, (int64_t)ctx->smem_fused, ctx->nsm,
+                         P.nfseg, P.nchunk, kFusedThreads};
+  for (int i = 0; i < std::min(n, 12); ++i) out[i] = v[i];
   return GAUS_OK;
 }
 

@@ -148,6 +148,7 @@ struct gaus_ctx {
   long long *d_U = nullptr;      // B * C * Dh usage (k_reduce), 2^32 fixed point
   long long *d_rpart = nullptr;  // nblk_r * Dh * RBr storage partials
   long long *d_Ureg = nullptr;   // B * Dh expected (folded) storage, 2^32 fixed point
+  float4 *d_qtab = nullptr;      // tail tables of the storage forward (k_tail_tables), all families
   float *d_Hreg = nullptr;       // B * Dh storage adjoint
   float2 *d_eslot = nullptr;     // E * B successor shares of the storage gradient
   int32_t *d_in_eslot = nullptr; // E
@@ -171,6 +172,7 @@ struct gaus_ctx {
   // per cooperative launch, dynamic shared memory; 0 = the terms or sizes need the
   // multi-kernel path (storage term, continuous dependency penalty, D > 32767)
   int fK = 0, fGl = 0;
+  int nsm = 0;                   // streaming multiprocessors of the device
   int fRG = 1, fRBp = 1, fRB1 = 1, fG = 1;
   int fW = 0;  // table row length of the fused path ([node][point][restart] layout)  // restarts per group, lanes per row (phases 2-3, phase 1), groups
   size_t smem_fused = 0;

@@ -38,6 +38,7 @@ struct RegArgs {
   const int32_t *out_ptr, *out_dst;  // internal CSR, successors by caller id
   const int32_t *seg;
   const unsigned *win;               // packed windows
+  const float4 *qtab;                // the family's tail table (kTailRows x 2, k_tail_tables)
   long long *rpart;                  // blocks * Dh * RB
   // backward
   const float *Hreg;                 // (B, Dh): w_mem * softmax of (M)Reg
@@ -67,6 +68,110 @@ __device__ __forceinline__ void cdf_pair(int d, float mu, float inv_s, int a, in
   const float q = reg_tail<kFam>(z);
   C = z <= 0.f ? q : 1.0f - q;
   Q = z <= 0.f ? 1.0f - q : q;
+}
+
+// ---------------------------------------------------------------- storage forward in float pairs
+// The storage LSE's softmax at a small tau turns absolute errors of the expected
+// storage into relative errors of its weights divided by tau, and a bin sums
+// hundreds of contributions b_i C_i (1 - M_i) of up to 64 bits each: with fp32
+// contributions (~1e-7 relative each) the gradient would carry ~1e-4 relative
+// error.  The forward therefore carries the tails, the successors' product and
+// each contribution as unevaluated pairs hi + lo of floats (~1e-12 absolute, FP32
+// arithmetic throughout: GB300's FP64 rate is a small fraction of its FP32 rate)
+// and rounds each contribution once, into the fixed-point histogram.
+//
+// The upper tail Q(z) = 1 - F(z), z >= 0, comes from a table of Q and of the
+// density f and its first three derivatives at z0 = i / 64, 0 <= z0 <= 16, filled
+// once in double (k_tail_tables), and a Taylor step of four terms to z
+// (|z - z0| <= 1/128: truncation below 1e-12).  Beyond z = 16 the normal, logistic
+// and Laplace tails are below 1e-10 and are taken in fp32; the Cauchy tail
+// atan(1 / (c z)) / pi comes from the arctangent series in y = 1 / (c z) <= 0.074.
+constexpr int kTailPerUnit = 64, kTailZmax = 16, kTailRows = kTailZmax * kTailPerUnit + 1;
+
+struct FF {
+  float h, l;
+};
+// h + l = a + b exactly (two-sum)
+__device__ __forceinline__ FF ff_two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b), bb = __fsub_rn(s, a);
+  return {s, __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb))};
+}
+// h + l = a + b exactly when |a| >= |b| or a = 0 (fast two-sum)
+__device__ __forceinline__ FF ff_fast_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  return {s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+__device__ __forceinline__ FF ff_add(FF a, FF b) {
+  const FF s = ff_two_sum(a.h, b.h);
+  return ff_fast_sum(s.h, s.l + (a.l + b.l));
+}
+__device__ __forceinline__ FF ff_mul(FF a, FF b) {
+  const float p = __fmul_rn(a.h, b.h);
+  return ff_fast_sum(p, fmaf(a.h, b.h, -p) + (a.h * b.l + a.l * b.h));
+}
+__device__ __forceinline__ FF ff_mulf(FF a, float b) {
+  const float p = __fmul_rn(a.h, b);
+  return ff_fast_sum(p, fmaf(a.h, b, -p) + a.l * b);
+}
+// 1 - a for 0 <= a <= 1
+__device__ __forceinline__ FF ff_one_minus(FF a) {
+  const FF s = ff_fast_sum(1.0f, -a.h);
+  return ff_fast_sum(s.h, s.l - a.l);
+}
+
+// z = (d + 1/2 - mu) / sigma as a pair: the division's residual from an fma
+__device__ __forceinline__ FF z_pair(int d, float mu, float sg, float inv_s) {
+  const FF x = ff_two_sum((float)d + 0.5f, -mu);
+  const float zh = x.h * inv_s;
+  return {zh, (fmaf(-zh, sg, x.h) + x.l) * inv_s};
+}
+
+template <int kFam>
+__device__ __forceinline__ FF reg_tail_pair(const float4 *__restrict__ tab, float zh, float zl) {
+  if (zh >= (float)kTailZmax) {
+    if constexpr (kFam == GAUS_CAUCHY) {
+      constexpr double kC = 0.84932180028801904272, kInvPi = 0.31830988618379067154;
+      constexpr float kCh = (float)kC, kCl = (float)(kC - (double)kCh);
+      constexpr float kPh = (float)kInvPi, kPl = (float)(kInvPi - (double)kPh);
+      const FF cz = ff_mul({kCh, kCl}, {zh, zl});
+      const float yh = 1.0f / cz.h;
+      const FF y = ff_fast_sum(yh, yh * (fmaf(-yh, cz.h, 1.0f) - yh * cz.l));
+      const float y2 = yh * yh;
+      const float del = y2 * (-1.0f / 3.0f + y2 * (0.2f + y2 * (-1.0f / 7.0f + y2 * (1.0f / 9.0f))));
+      return ff_mul(ff_add(y, {yh * del, 0.0f}), {kPh, kPl});
+    } else {
+      return {Fam<kFam>::tail(zh), 0.0f};
+    }
+  }
+  const int i = __float2int_rn(zh * (float)kTailPerUnit);
+  const float hh = zh - (float)i * (1.0f / (float)kTailPerUnit);  // exact
+  const float4 q = __ldg(&tab[2 * i]), t = __ldg(&tab[2 * i + 1]);
+  // Q(z0 + h) = Q0 - f h - f' h^2 / 2 - f'' h^3 / 6 - f''' h^4 / 24, h = hh + zl
+  const float rest = hh * hh * (t.x + hh * (t.y + hh * t.z));
+  const float p = __fmul_rn(q.z, hh);
+  const float pe = fmaf(q.z, hh, -p) + (q.z * zl + q.w * hh);
+  const FF s = ff_two_sum(q.x, -p);
+  return ff_fast_sum(s.h, s.l + (q.y - (pe + rest)));
+}
+
+// C of a windowed CDF at integer point d as a pair (0 and 1 outside [a, b])
+template <int kFam>
+__device__ __forceinline__ FF cdf_pair_ff(const float4 *__restrict__ tab, int d, float mu, float sg, float inv_s,
+                                          int a, int b) {
+  if (d < a) return {0.0f, 0.0f};
+  if (d > b) return {1.0f, 0.0f};
+  const FF z = z_pair(d, mu, sg, inv_s);
+  const bool neg = z.h <= 0.0f;
+  const FF q = reg_tail_pair<kFam>(tab, neg ? -z.h : z.h, neg ? -z.l : z.l);
+  return neg ? q : ff_one_minus(q);
+}
+
+// hist_add of a pair in [0, 64]: rounded once to 2^-32
+__device__ __forceinline__ void hist_add_pair(unsigned *hlo, unsigned *hhi, int cell, FF v) {
+  long long F = __float2ll_rn(v.h * 4294967296.0f) + __float2ll_rn(v.l * 4294967296.0f);
+  F = F < 0 ? 0 : F;
+  atomicAdd(&hlo[cell], (unsigned)(F & 0xFFFF));
+  atomicAdd(&hhi[cell], (unsigned)(F >> 16));
 }
 
 // Adds the integer v to the (folded) bins d in [s, e] through a difference
@@ -125,6 +230,24 @@ __device__ __forceinline__ float one_minus_m(const RegArgs &A, int e0, int deg, 
   return t;
 }
 
+// 1 - M_i(d) = 1 - prod_j C_j(d) as a pair (the forward's product).
+template <int kFam>
+__device__ __forceinline__ FF one_minus_m_pair(const RegArgs &A, int e0, int deg, int dmax, int b, int d, int Amax) {
+  if (deg == 0 || d < Amax) return {1.0f, 0.0f};
+  FF P = {1.0f, 0.0f};
+  for (int q = 0; q < dmax; ++q) {
+    if (q < deg) {
+      const int jc = A.out_dst[e0 + q];
+      const unsigned wm = A.win[(size_t)jc * A.B + b];
+      const int aj = (int)(wm & 0xFFFFu), bj = (int)(wm >> 16) - 1;
+      const bool in = d >= aj && d <= bj;
+      const float mj = in ? A.mu[(size_t)jc * A.B + b] : 0.f, sj = in ? A.sg[(size_t)jc * A.B + b] : 1.f;
+      P = ff_mul(P, cdf_pair_ff<kFam>(A.qtab, d, mj, sj, 1.0f / sj, aj, bj));
+    }
+  }
+  return ff_one_minus(P);
+}
+
 template <int kFam>
 __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
   extern __shared__ __align__(16) unsigned char smem_r[];
@@ -178,10 +301,10 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
       const bool on = k < total;
       const bool own = k < n_own;
       const int d = own ? a + k : tail_lo + (k - n_own);
-      float Ci = 1.f, Qi;
-      if (on && own) cdf_pair<kFam>(d, mu, inv_s, a, bw, Ci, Qi);
-      const float L = one_minus_m<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
-      if (on && bits != 0.f) hist_add(hlo, hhi, fold_bin(d, A.II) * RB + r, bits * Ci * L);
+      FF Ci = {1.0f, 0.0f};
+      if (on && own) Ci = cdf_pair_ff<kFam>(A.qtab, d, mu, sg, inv_s, a, bw);
+      const FF L = one_minus_m_pair<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
+      if (on && bits != 0.f) hist_add_pair(hlo, hhi, fold_bin(d, A.II) * RB + r, ff_mulf(ff_mul(Ci, L), bits));
     }
     __syncwarp();
   }
@@ -200,6 +323,57 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
 }
 
 #ifndef GAUS_FAMILY_KERNELS_ONLY
+// The tail tables of the four families (GAUS_GAUSSIAN..GAUS_CAUCHY, kTailRows rows
+// each, row i at z0 = i / 64): float4 {Q hi, Q lo, f hi, f lo} and float4
+// {f' / 2, f'' / 6, f''' / 24, 0}, in double from the closed forms (scales c as in
+// Fam<k>: logistic pi / sqrt(3), Laplace sqrt(2), Cauchy 1 / sqrt(2 ln 2)).
+__global__ void k_tail_tables(float4 *tab) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= 4 * kTailRows) return;
+  const int fam = i / kTailRows;
+  const double z = (double)(i % kTailRows) / kTailPerUnit;
+  double Q, f, f1, f2, f3;
+  if (fam == GAUS_GAUSSIAN) {
+    Q = 0.5 * erfc(z * 0.70710678118654752440);
+    f = 0.39894228040143267794 * exp(-0.5 * z * z);
+    f1 = -z * f;
+    f2 = (z * z - 1.0) * f;
+    f3 = (3.0 * z - z * z * z) * f;
+  } else if (fam == GAUS_LOGISTIC) {
+    const double c = 1.81379936423421785059, e = exp(-c * z);
+    Q = e / (1.0 + e);
+    f = c * Q * (1.0 - Q);
+    f1 = -c * f * (1.0 - 2.0 * Q);
+    f2 = -c * (f1 * (1.0 - 2.0 * Q) + 2.0 * f * f);
+    f3 = -c * (f2 * (1.0 - 2.0 * Q) + 6.0 * f * f1);
+  } else if (fam == GAUS_LAPLACE) {
+    const double c = 1.41421356237309504880;
+    Q = 0.5 * exp(-c * z);
+    f = c * Q;
+    f1 = -c * f;
+    f2 = c * c * f;
+    f3 = -c * c * c * f;
+  } else {
+    const double c = 0.84932180028801904272, kp = c * 0.31830988618379067154, u = c * z, g = 1.0 / (1.0 + u * u);
+    Q = 0.31830988618379067154 * atan2(1.0, u);
+    f = kp * g;
+    f1 = kp * c * (-2.0 * u * g * g);
+    f2 = kp * c * c * (6.0 * u * u - 2.0) * g * g * g;
+    f3 = kp * c * c * c * 24.0 * u * (1.0 - u * u) * g * g * g * g;
+  }
+  float4 a, b;
+  a.x = (float)Q;
+  a.y = (float)(Q - (double)a.x);
+  a.z = (float)f;
+  a.w = (float)(f - (double)a.z);
+  b.x = (float)(f1 / 2.0);
+  b.y = (float)(f2 / 6.0);
+  b.z = (float)(f3 / 24.0);
+  b.w = 0.0f;
+  tab[2 * i] = a;
+  tab[2 * i + 1] = b;
+}
+
 // Reg per (restart, bin) from every block's partials: block = (group, bin),
 // threads = restarts x slices of the segment list, slices combined in order.
 __global__ void __launch_bounds__(256) k_reduce_reg(const long long *rpart, long long *Ureg, int B, int Dh, int RB,

@@ -78,6 +78,24 @@ def test_storage_modulo(g, fam):
     check_loss_grad(p, g, B, mu, sg, _lam(B, np.random.default_rng(12)), hp, restarts=[0, 3, 7])
 
 
+@pytest.mark.parametrize("fam", [oracle.GAUSSIAN] + FAMS)
+def test_storage_small_tau(g, fam):
+    # the loop body at full size (V = 5,000, D = 3 II = 1,659), where a folded step
+    # sums hundreds of storage contributions, with tau = 3e-3 dividing their absolute
+    # error by tau in the softmax weights: every family's tail table and Taylor step,
+    # and the Cauchy series beyond the table (its windows span the horizon, z > 16),
+    # against the oracle with the per-component bound from 1 % of the largest
+    # component (test_modulo_loop_full_size_sampled_usage_and_storage is the normal's
+    # case that contributions rounded to fp32 fail)
+    p = W.modulo_loop(1, ii_factor=1.25)
+    p.terms = W.RES_OBJ | W.RES_VIOL | W.REG_OBJ
+    B = 8
+    mu, sg = W.init_state(p, B, 13)
+    hp = g.default_hparams(terms=p.terms, tau=3e-3, rho=1e-3, family=fam)
+    lam = np.full((B, 3), 1e-6, np.float32)
+    check_loss_grad(p, g, B, mu, sg, lam, hp, restarts=[0, 5])
+
+
 @pytest.mark.parametrize("fam", FAMS)
 def test_mixed_window_lengths(g, fam):
     # sigma over two orders of magnitude inside every warp
