@@ -342,20 +342,26 @@ __device__ __forceinline__ bool load_nb(const FusedArgs &A, int ni, int b, bool 
 // The own side of every edge of a chunk (consumer side of in-edges and back edges
 // in, producer side of out-edges and back edges out) for the phase-2 lanes of a
 // warp, which all work on the same node: the entries and their kinds are
-// warp-uniform, and the next entry and the neighbour's window are loaded while the
-// current one is evaluated.
+// warp-uniform.  The chunk's entries (at most kChunkEdges) and then all their
+// neighbours' windows are loaded before the first edge is evaluated (two round
+// trips per chunk instead of two per edge), and rotate through registers.
 template <int kFam, bool kCom>
 __device__ __forceinline__ void chunk_edges(const FusedArgs &A, int e0, int ne, int b, bool act, const Own &O,
                                             bool dep, bool com, bool rec, float &Ad, float &Bd, float &Ao, float &Bo,
                                             float &Ar, float &Br, float &fd, float &fc, float &fr) {
   constexpr unsigned FULL = 0xffffffffu;
+  static_assert(kChunkEdges == 4, "the register pipeline holds four entries");
   if (ne <= 0) return;
+  const int4 none = make_int4(0, 1, -1, 0);
   int4 en_a = __ldg(A.finc + e0);
-  int4 en_b = ne > 1 ? __ldg(A.finc + e0 + 1) : make_int4(0, 1, 0, 0);
+  int4 en_b = ne > 1 ? __ldg(A.finc + e0 + 1) : none;
+  int4 en_c = ne > 2 ? __ldg(A.finc + e0 + 2) : none;
+  int4 en_d = ne > 3 ? __ldg(A.finc + e0 + 3) : none;
   unsigned w_a = act ? A.win[(size_t)en_a.x * A.B + b] : 0x80000000u;
+  unsigned w_b = (ne > 1 && act) ? A.win[(size_t)en_b.x * A.B + b] : 0x80000000u;
+  unsigned w_c = (ne > 2 && act) ? A.win[(size_t)en_c.x * A.B + b] : 0x80000000u;
+  unsigned w_d = (ne > 3 && act) ? A.win[(size_t)en_d.x * A.B + b] : 0x80000000u;
   for (int q = 0; q < ne; ++q) {
-    const unsigned w_b = (q + 1 < ne && act) ? A.win[(size_t)en_b.x * A.B + b] : 0x80000000u;
-    const int4 en_c = q + 2 < ne ? __ldg(A.finc + e0 + q + 2) : make_int4(0, 1, 0, 0);
     const int kind = en_a.z, L = en_a.y;
     FNb<kFam> N;
     const bool on = make_nb<kFam>(A, en_a.x, b, w_a, act, N) && act;
@@ -392,9 +398,8 @@ __device__ __forceinline__ void chunk_edges(const FusedArgs &A, int e0, int ne, 
       if (__any_sync(FULL, dr))
         prod_side<kFam, false, false, true, false>(O, N, L, dr, dep, A.alpha, Ar, Br, dummy0, dummy1, dummy2);
     }
-    en_a = en_b;
-    w_a = w_b;
-    en_b = en_c;
+    en_a = en_b; en_b = en_c; en_c = en_d;
+    w_a = w_b; w_b = w_c; w_c = w_d;
   }
 }
 
@@ -409,6 +414,9 @@ __device__ void coop_node(const FusedArgs &A, int e0, int ne, int b, int a, int 
   float Ad = 0.f, Bd = 0.f, Ao = 0.f, Bo = 0.f, Ar = 0.f, Br = 0.f, fd = 0.f, fc = 0.f, fr = 0.f;
   const int n = bw - a + 1;
   const float alpha = A.alpha;
+  // the neighbours' windows, once for all the point batches: lane q holds entry q's
+  // (the warp works on one restart); the entries themselves are L1 hits
+  const unsigned my_w = lane < ne ? A.win[(size_t)__ldg(A.finc + e0 + lane).x * A.B + b] : 0x80000000u;
   for (int p0 = 0; p0 == 0 || p0 < n; p0 += 32) {
     const int j = p0 + lane;
     const bool pt = j < n;
@@ -419,13 +427,14 @@ __device__ void coop_node(const FusedArgs &A, int e0, int ne, int b, int a, int 
     const float f = pt ? Fam<kFam>::pdf(z) : 0.f;
     const float zf = z * f;
     const bool first = p0 == 0 && lane == 0;
-    for (int e = e0; e < e0 + ne; ++e) {
-      const int4 en = __ldg(A.finc + e);
+    for (int e = 0; e < ne; ++e) {
+      const unsigned wn = __shfl_sync(0xffffffffu, my_w, e);
+      const int4 en = __ldg(A.finc + e0 + e);
       const int kind = en.z, L = en.y;
       if (kind <= 1 && !(dep || com)) continue;
       if (kind >= 2 && !rec) continue;
       FNb<kFam> N;
-      if (!load_nb<kFam>(A, en.x, b, true, N)) continue;
+      if (!make_nb<kFam>(A, en.x, b, wn, true, N)) continue;
       if (kind == 0) {
         const float hi = N.at(t + 1 - L), lo = N.at(t - L), p = hi - lo;
         if (pt) {
@@ -621,15 +630,32 @@ __device__ __forceinline__ void p2_lane(const FusedArgs &A, FusedShared &S, int 
     // terms that do not depend on them -- the dependency and recurrence tails
     // 1 - C_u(b_v + 1 - L) of the in-edges and the communication gaps
     // max(0, a_w - 1 - b_v) of the out-edges -- with the general path's arithmetic
-    for (int q = 0; q < ne; ++q) {
-      const int4 en = __ldg(A.finc + e0 + q);
-      const int kind = en.z, L = en.y;
-      if (!act || (kind == 0 && !dep) || (kind == 1 && !kCom) || kind == 3 || (kind == 2 && !rec)) continue;
+    // (entries, then windows, then table values: three round trips per chunk)
+    int4 en[kChunkEdges];
+    unsigned w[kChunkEdges];
+    float cv[kChunkEdges];
+#pragma unroll
+    for (int q = 0; q < kChunkEdges; ++q) {
+      en[q] = q < ne ? __ldg(A.finc + e0 + q) : make_int4(0, 1, -1, 0);
+      const int kind = en[q].z;
+      const bool need = act && ((kind == 0 && dep) || (kind == 1 && kCom) || (kind == 2 && rec));
+      if (!need) en[q].z = -1;
+    }
+#pragma unroll
+    for (int q = 0; q < kChunkEdges; ++q) w[q] = en[q].z >= 0 ? A.win[(size_t)en[q].x * A.B + bs] : 0x80000000u;
+#pragma unroll
+    for (int q = 0; q < kChunkEdges; ++q) {
       FNb<kFam> N;
-      if (!load_nb<kFam>(A, en.x, bs, true, N)) continue;
-      if (kind == 0) fd += 1.0f - N.at(a - L);
-      else if (kind == 1) fc += (float)max(0, N.a - a);
-      else fr += 1.0f - N.at(a - L);
+      const bool ok_q = make_nb<kFam>(A, en[q].x, bs, w[q], en[q].z >= 0, N);
+      if (!ok_q) en[q].z = -1;
+      // kind 1 keeps the neighbour's first point in cv
+      cv[q] = (en[q].z == 0 || en[q].z == 2) ? N.at(a - en[q].y) : (float)N.a;
+    }
+#pragma unroll
+    for (int q = 0; q < kChunkEdges; ++q) {
+      if (en[q].z == 0) fd += 1.0f - cv[q];
+      else if (en[q].z == 1) fc += (float)max(0, (int)cv[q] - a);
+      else if (en[q].z == 2) fr += 1.0f - cv[q];
     }
   } else {
     const int nst = __reduce_max_sync(FULL, nl);
@@ -1133,14 +1159,14 @@ __global__ void __launch_bounds__(kFusedThreads, 1) k_fused(const FusedArgs A) {
       // warp items claimed from the group's counter over all its nodes (balances the
       // blocks); the next claim is issued before the current item is worked on
       unsigned *ctr = A.ctr + (size_t)p * A.G + (g - A.g0);
-      int nxt = 0;
-      if (lane == 0) nxt = (int)atomicAdd(ctr, 1u);
-      nxt = __shfl_sync(FULL, nxt, 0);
+      // (every lane takes part in the claim's atomic, lane 0 adding 1: the result is
+      // waited for only where the next item starts, not at a branch's reconvergence)
+      const unsigned one = lane == 0 ? 1u : 0u;
+      int nxt = __shfl_sync(FULL, (int)atomicAdd(ctr, one), 0);
       for (;;) {
         const int base = nxt;
         if (base >= A.nchunk) break;
-        int nn = 0;
-        if (lane == 0) nn = (int)atomicAdd(ctr, 1u);
+        const int nn = (int)atomicAdd(ctr, one);
         const int4 cd = __ldg(A.chunk + base);
         const int vi = cd.x, ch = cd.w;
         if (passes == 1) {

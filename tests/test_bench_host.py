@@ -41,3 +41,49 @@ def test_measured_hbm_peak_is_read_or_falls_back():
 def test_profiled_traffic_is_a_byte_count_or_none():
     t = bench.profiled_traffic()
     assert t is None or (math.isfinite(t) and 1e6 < t < 1e10)
+
+
+def test_storage_point_edges_pair_consumer_points_with_producers():
+    rng = np.random.default_rng(5)
+    V, B, D, k = 6, 3, 25, 6.0
+    mu = rng.uniform(0, D, size=(V, B)).astype(np.float32)
+    sg = rng.uniform(0.1, 2.0, size=(V, B)).astype(np.float32)
+    src = np.array([0, 0, 1, 3, 4], np.int64)
+    dst = np.array([1, 2, 3, 5, 5], np.int64)
+    T = torch.from_numpy
+    f, n_pt, n_eb, n_st = bench.algorithmic_work(torch, T(mu), T(sg), T(src), T(dst), k, D, storage=True)
+    pts = np.zeros((V, B))
+    for v in range(V):
+        for b in range(B):
+            pts[v, b] = sum(1 for t in range(0, D - 1) if abs(t + 0.5 - float(mu[v, b])) <= k * float(sg[v, b]))
+    assert n_st == pytest.approx(sum(pts[w].sum() for w in dst))
+    assert f == pytest.approx(20 * n_pt + 8 * (n_eb + n_st))
+    _, _, _, none = bench.algorithmic_work(torch, T(mu), T(sg), T(src), T(dst), k, D, storage=False)
+    assert none == 0.0
+
+
+@pytest.mark.parametrize("factor", [1.0, 1.5])
+def test_modulo_list_schedule_is_a_verified_witness(factor):
+    import oracle
+    import workloads as W
+    p = W.modulo_loop(3, ii_factor=factor, V=600, levels=20, n_back=30)
+    s = bench.modulo_list_schedule(p)
+    assert s is not None and s.dtype == np.int32 and s.shape == (p.V,)
+    r = oracle.verify(oracle.OracleProblem(p), s)
+    assert r["feasible"] == 1 and r["res_ok"] == 1
+
+
+def test_modulo_list_schedule_gives_up_without_room():
+    import workloads as W
+    p = W.modulo_loop(3, ii_factor=1.0, V=600, levels=20, n_back=30)
+    p.limit = np.where(np.isfinite(p.limit), 0.0, p.limit)   # no slot for any node
+    assert bench.modulo_list_schedule(p) is None
+
+
+def test_launch_count_per_step():
+    fused = {"fused": 1, "fused_launches_per_call": 1, "launches_per_iteration": 0}
+    multi = {"fused": 0, "fused_launches_per_call": 0, "launches_per_iteration": 8}
+    # 20 calls of 100 iterations: one k_fused launch per call, or 8 kernels per
+    # iteration, plus legalize and the verifier's two passes per call
+    assert bench.launches_per_step(fused, 2000, 100) == 20 * (1 + 3)
+    assert bench.launches_per_step(multi, 2000, 100) == 20 * (800 + 3)
