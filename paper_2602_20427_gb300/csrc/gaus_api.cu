@@ -137,6 +137,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
     RA.k_win = ctx->k_win; RA.perm = ctx->d_perm; RA.bits = ctx->d_bits;
     RA.out_ptr = ctx->d_out_ptr; RA.out_dst = ctx->d_out_dst; RA.seg = ctx->d_seg; RA.win = ctx->d_win;
     RA.qtab = ctx->d_qtab + (size_t)2 * kTailRows * ctx->hp.family;
+    RA.tab = ctx->d_tab; RA.W = ctx->W;
     RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gown = ctx->d_gown; RA.eslot = ctx->d_eslot;
     ks.reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_fwd launch");

@@ -38,6 +38,8 @@ struct RegArgs {
   const int32_t *out_ptr, *out_dst;  // internal CSR, successors by caller id
   const int32_t *seg;
   const unsigned *win;               // packed windows
+  const float *tab;                  // the node pass's CDF table rows (V, B, W) by caller id
+  int W;
   const float4 *qtab;                // the family's tail table (kTailRows x 2, k_tail_tables)
   long long *rpart;                  // blocks * Dh * RB
   // backward
@@ -394,6 +396,35 @@ __global__ void __launch_bounds__(256) k_reduce_reg(const long long *rpart, long
 }
 #endif  // GAUS_FAMILY_KERNELS_ONLY
 
+// C_j(d) of node jc (caller id), restart b, packed window wm, for the backward: the
+// node pass's table row [0, C(a), ..., C(b), 1] when the window fits it (n + 3 <= W),
+// else evaluated from (mu, sigma).
+template <int kFam>
+__device__ __forceinline__ float reg_cdf_tab(const RegArgs &A, int jc, int b, unsigned wm, int d) {
+  const int aj = (int)(wm & 0xFFFFu), bj = (int)(wm >> 16) - 1;
+  if (d < aj) return 0.0f;
+  if (d > bj) return 1.0f;
+  const size_t ix = (size_t)jc * A.B + b;
+  if (bj - aj + 4 <= A.W) return __ldg(A.tab + ix * A.W + (d - aj + 1));
+  const float m = __ldg(A.mu + ix), iv = 1.0f / __ldg(A.sg + ix);
+  const float z = ((float)d + 0.5f - m) * iv;
+  const float q = reg_tail<kFam>(z);
+  return z <= 0.f ? q : 1.0f - q;
+}
+
+// 1 - M_i(d) for the backward, from the table.
+template <int kFam>
+__device__ __forceinline__ float one_minus_m_tab(const RegArgs &A, int e0, int deg, int dmax, int b, int d, int Amax) {
+  if (deg == 0 || d < Amax) return 1.0f;
+  float P = 1.0f;
+  for (int q = 0; q < dmax; ++q)
+    if (q < deg) {
+      const int jc = A.out_dst[e0 + q];
+      P *= reg_cdf_tab<kFam>(A, jc, b, A.win[(size_t)jc * A.B + b], d);
+    }
+  return 1.0f - P;
+}
+
 template <int kFam>
 __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
   extern __shared__ __align__(16) unsigned char smem_rb[];
@@ -426,6 +457,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
     const float inv_s = valid ? 1.0f / sg : 1.0f, bits = A.bits[vcl];
     int a = 0, bw = -2;
     if (valid) window(mu, sg, A.k_win, A.D, a, bw);
+    const unsigned own_w = (unsigned)a | ((unsigned)(bw + 1) << 16);
     const int e0 = A.out_ptr[vcl], deg = valid ? A.out_ptr[vcl + 1] - e0 : 0;
     const int dmax = __reduce_max_sync(FULL, deg);
     int Amax, Bm;
@@ -437,7 +469,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
     for (int k = 0; k < nmax; ++k) {
       const bool on = k < n_own;
       const int d = a + k;
-      const float L = one_minus_m<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
+      const float L = one_minus_m_tab<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
       if (on) {
         const float z = ((float)d + 0.5f - mu) * inv_s;
         const float f = reg_pdf<kFam>(z);
@@ -463,21 +495,13 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
       for (int k = 0; k < cmax; ++k) {
         const bool on = k < cnt;
         const int d = lo + k;
-        float Ci = 1.f, Qi;
-        if (on) cdf_pair<kFam>(d, mu, inv_s, a, bw, Ci, Qi);
+        const float Ci = on ? reg_cdf_tab<kFam>(A, vc, b, own_w, d) : 1.0f;
         // product of the other successors' CDFs at d
         float prod = 1.f;
         for (int q2 = 0; q2 < dmax; ++q2) {
           if (on && q2 < deg && q2 != q) {
             const int kc2 = A.out_dst[e0 + q2];
-            const unsigned wm2 = A.win[(size_t)kc2 * A.B + b];
-            const int a2 = (int)(wm2 & 0xFFFFu), b2 = (int)(wm2 >> 16) - 1;
-            const bool in2 = d >= a2 && d <= b2;
-            const float m2 = in2 ? A.mu[(size_t)kc2 * A.B + b] : 0.f;
-            const float i2 = in2 ? 1.0f / A.sg[(size_t)kc2 * A.B + b] : 1.f;
-            float C2, Q2;
-            cdf_pair<kFam>(d, m2, i2, a2, b2, C2, Q2);
-            prod *= C2;
+            prod *= reg_cdf_tab<kFam>(A, kc2, b, A.win[(size_t)kc2 * A.B + b], d);
           }
         }
         if (on) {
