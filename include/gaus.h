@@ -246,6 +246,16 @@ gaus_status gaus_profile_phases(gaus_ctx *ctx, int32_t n_iters, const gaus_state
  * EINVAL for a NULL context or out, or n < 1. */
 gaus_status gaus_plan_info(const gaus_ctx *ctx, int64_t *out, int32_t n);
 
+/* Exercises the fused kernel's bounded barrier waits (a check of the failure path,
+ * not part of the method): one iteration of gaus_iterate whose group barriers can
+ * never complete, each wait ending after limit_ns.  Every restart's status becomes
+ * GAUS_ETIMEOUT; mu, sigma, the Adam moments, lambda and step are left as they were
+ * (the kernel writes the caller's state only at the end of a completed call), and
+ * the context stays usable.  limit_ns in 1,000 .. 1,000,000,000.  EINVAL for NULL
+ * pointers, a limit outside that range, or a context on the multi-kernel path.
+ * Asynchronous on the context's stream. */
+gaus_status gaus_check_barrier_timeout(gaus_ctx *ctx, const gaus_state *st, uint64_t limit_ns);
+
 /* Round every mean to s = floor(mu + 1/2) (Sec. 3.3 Sampling; exact for every
  * fp32 value) and legalize it: Alg. 1 (clamp to [ASAP, ALAP], then a forward push
  * in topological order with +Lat(u)) when II = 0, Alg. 2 (fixed-point relaxation

@@ -211,6 +211,10 @@ class Gaus:
         self._check(lib().gaus_plan_info(self._ctx, out, C.c_int32(len(self.PLAN_KEYS))))
         return dict(zip(self.PLAN_KEYS, [int(x) for x in out]))
 
+    def check_barrier_timeout(self, state, limit_ns):
+        """gaus_check_barrier_timeout: one fused iteration whose barriers never complete."""
+        self._check(lib().gaus_check_barrier_timeout(self._ctx, C.byref(self._state(state)), C.c_uint64(limit_ns)))
+
     # -- entry points
     def loss_grad(self, mu, sigma, lam, out=None):
         torch = self.torch

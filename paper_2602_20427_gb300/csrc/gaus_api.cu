@@ -203,9 +203,12 @@ bool fused_ok(const gaus_ctx *ctx) {
 gaus_status enqueue_fused(gaus_ctx *ctx, cudaStream_t st, int n_iters, bool adam, const float *mu, const float *sg,
                           float *m_mu, float *v_mu, float *m_sg, float *v_sg, float *lambda, int32_t *step,
                           float *grad_mu, float *grad_sg, float *loss, float *terms, int32_t *status,
-                          unsigned long long *prof) {
+                          unsigned long long *prof, unsigned bar_extra = 0,
+                          unsigned long long bar_limit_ns = kBarrierTimeoutNs) {
   const Plan &P = ctx->plan;
   FusedArgs A;
+  A.bar_extra = bar_extra;
+  A.bar_limit_ns = bar_limit_ns;
   A.V = P.V; A.B = P.B; A.D = P.D; A.II = P.II; A.Dh = P.Dh; A.C = P.C; A.K = ctx->fK;
   A.RG = ctx->fRG; A.RBp = ctx->fRBp; A.RB1 = ctx->fRB1;
   A.W = ctx->fW; A.n_iters = n_iters; A.nseg = P.nfseg;
@@ -735,6 +738,22 @@ gaus_status gaus_set_hparams(gaus_ctx *ctx, const gaus_hparams *hp) {
   drop_graph(ctx);
   if (hp->family != old_family) return set_smem_attrs(ctx);
   return GAUS_OK;
+}
+
+gaus_status gaus_check_barrier_timeout(gaus_ctx *ctx, const gaus_state *S, uint64_t limit_ns) {
+  if (!ctx) return GAUS_EINVAL;
+  if (!S || !S->mu || !S->sigma || !S->m_mu || !S->v_mu || !S->m_sigma || !S->v_sigma || !S->lambda ||
+      !S->step || !S->loss || !S->terms || !S->status || limit_ns < 1000 || limit_ns > 1000000000ull) {
+    ctx->err = "gaus_check_barrier_timeout: NULL state pointer or limit outside 1 us .. 1 s";
+    return GAUS_EINVAL;
+  }
+  if (!fused_ok(ctx)) {
+    ctx->err = "gaus_check_barrier_timeout: the context runs the multi-kernel path";
+    return GAUS_EINVAL;
+  }
+  return enqueue_fused(ctx, ctx->stream, 1, true, S->mu, S->sigma, S->m_mu, S->v_mu, S->m_sigma, S->v_sigma,
+                       S->lambda, S->step, nullptr, nullptr, S->loss, S->terms, S->status, nullptr, 1u,
+                       (unsigned long long)limit_ns);
 }
 
 gaus_status gaus_plan_info(const gaus_ctx *ctx, int64_t *out, int32_t n) {

@@ -67,6 +67,7 @@ __device__ __forceinline__ size_t tab_stride(int B) { return kTabPointMajor ? (s
 // otherwise run one after another in one warp).
 constexpr int kLongQueue = 512;
 constexpr unsigned long long kBarrierTimeoutNs = 4000000000ull;  // 4 s per barrier wait
+constexpr unsigned kBarrierMaxPolls = 1u << 26;                   // and at most 2^26 polls
 
 struct FusedArgs {
   // RG restarts per group (<= 64); phases 2 and 3 process a node's RG restarts in rows
@@ -122,6 +123,8 @@ struct FusedArgs {
   int32_t *nonf;            // [2][B]
   double *rstat;            // [B][2]: sum_c LSE_tau(U_c), V_res
   unsigned *bar;            // [G] group arrival counters (zeroed before the launch)
+  unsigned bar_extra;       // added to every barrier target: 0 (a test sets 1: no barrier completes)
+  unsigned long long bar_limit_ns;  // a barrier wait's time limit
   unsigned *ctr;            // [2][G] phase-2 work counters of the groups, by iteration parity
   int32_t *abort_flag;
   unsigned long long *prof; // optional: globaltimer stamps [n_iters][blocks][6]: iteration start,
@@ -142,9 +145,10 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
 }
 
 // Group barrier: every block of the group has arrived `target` times.  Bounded:
-// after kBarrierTimeoutNs (or once another group has aborted) the abort flag is
-// set and false is returned to every thread of the block.
-__device__ __forceinline__ bool group_barrier(unsigned *bar, unsigned target, int32_t *abort_flag, int *s_ok) {
+// after limit_ns of waiting, or kBarrierMaxPolls polls, or once another group has
+// aborted, the abort flag is set and false is returned to every thread of the block.
+__device__ __forceinline__ bool group_barrier(unsigned *bar, unsigned target, int32_t *abort_flag, int *s_ok,
+                                              unsigned long long limit_ns) {
   __syncthreads();
   if (threadIdx.x == 0) {
     int ok = 1;
@@ -157,7 +161,7 @@ __device__ __forceinline__ bool group_barrier(unsigned *bar, unsigned target, in
         if (*(volatile int32_t *)abort_flag) { ok = 0; break; }
         const unsigned long long t = global_ns();
         if (t0 == 0) t0 = t;
-        else if (t - t0 > kBarrierTimeoutNs) {
+        if (t - t0 > limit_ns || polls >= kBarrierMaxPolls) {
           atomicExch(abort_flag, 1);
           ok = 0;
           break;
@@ -1127,7 +1131,7 @@ __global__ void __launch_bounds__(kFusedThreads, 1) k_fused(const FusedArgs A) {
     }
     stamp(it, 1);
     nbar += A.K;
-    alive = group_barrier(A.bar + g, nbar, A.abort_flag, &S.ok);
+    alive = group_barrier(A.bar + g, nbar + A.bar_extra, A.abort_flag, &S.ok, A.bar_limit_ns);
     if (!alive) break;
     stamp(it, 2);
 
@@ -1212,7 +1216,7 @@ __global__ void __launch_bounds__(kFusedThreads, 1) k_fused(const FusedArgs A) {
         if (S.fw[q][tid]) atomicAdd(&A.fwd[3 * ((size_t)p * B + g * RG + tid) + q], S.fw[q][tid]);
     stamp(it, 3);
     nbar += A.K;
-    alive = group_barrier(A.bar + g, nbar, A.abort_flag, &S.ok);
+    alive = group_barrier(A.bar + g, nbar + A.bar_extra, A.abort_flag, &S.ok, A.bar_limit_ns);
     if (!alive) break;
     stamp(it, 4);
 

@@ -107,8 +107,8 @@ def test_ragged_restart_counts(g, B):
 
 
 def test_many_restart_groups(g):
-    # B = 200: thirteen groups of 16 restarts, the last one partly filled; the
-    # node, edge and update passes' one-wave grids then hold several groups each
+    # B = 200: four fused restart groups of up to 64 (the last one of 8), each with its
+    # own blocks and barriers; on the multi-kernel path thirteen groups of 16
     p = W.random_layered(6)
     p.terms = W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL
     B = 200
