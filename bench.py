@@ -291,13 +291,23 @@ class Solve:
         self.solve()
 
 
-def launches_per_step(plan, iters, period):
+def launches_per_step(plan, iters, period, fused_calls=None, multi_iters=None, choices=0):
     """Kernel launches of one step: per gaus_iterate call the cooperative k_fused
-    launches (fused path) or the per-iteration kernels (multi-kernel path), and per
-    period the legalization kernel and the verifier's two passes."""
+    launches (fused path) or the per-iteration kernels (multi-kernel path) and, when
+    the path is chosen per call, the window reduction of the choice; per period the
+    legalization kernel and the verifier's two passes.  Without the counts of a
+    measured step, every call is taken to run the plan's preferred path."""
     calls = iters // period
-    it = plan["fused_launches_per_call"] if plan["fused"] else period * plan["launches_per_iteration"]
-    return calls * (it + 3)
+    if fused_calls is None:
+        fused_calls = calls if plan["fused"] else 0
+        multi_iters = 0 if plan["fused"] else iters
+    return (fused_calls * plan["fused_launches_per_call"] + multi_iters * plan["launches_per_iteration"]
+            + choices + calls * 3)
+
+
+def path_counts(ctx):
+    i = ctx.plan_info()
+    return i["fused_calls"], i["multi_iterations"], i["path_choices"]
 
 
 def device_peaks(g, torch):
@@ -329,7 +339,9 @@ def iteration_roofline(torch, ctx, solve, p, B, hp, mu0, sg0, peaks, plan):
     ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
     calls_ms = []
     w0 = algorithmic_work(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D, storage)
+    fused_t, fused_bytes, fused_flop, fused_pts, fused_calls = 0.0, 0.0, 0.0, 0.0, 0
     for _ in range(nchunk):
+        f0 = path_counts(ctx)[0]
         torch.cuda.synchronize()
         ev[0].record()
         ctx.iterate(period, st)
@@ -337,6 +349,7 @@ def iteration_roofline(torch, ctx, solve, p, B, hp, mu0, sg0, peaks, plan):
         torch.cuda.synchronize()
         ms = ev[0].elapsed_time(ev[1])
         calls_ms.append(ms)
+        was_fused = path_counts(ctx)[0] > f0
         w1 = algorithmic_work(torch, st["mu"], st["sigma"], src, dst, hp.window_k, p.D, storage)
         fl, pt, eb, sp = (0.5 * (x + y) for x, y in zip(w0, w1))
         w0 = w1
@@ -351,24 +364,34 @@ def iteration_roofline(torch, ctx, solve, p, B, hp, mu0, sg0, peaks, plan):
         tot["storage_pe"] += period * sp
         tot["bytes"] += period * sb
         tot["t"] += ms * 1e-3
+        if was_fused:
+            fused_calls += 1
+            fused_t += ms * 1e-3
+            fused_bytes += period * sb
+            fused_flop += period * fl
+            fused_pts += period * pt
     res = max(tot["alg_t"], key=tot["alg_t"].get)
+    # the dominant kernel: k_fused over the calls it ran, when it ran any
+    kt, kb, kf, kp = (fused_t, fused_bytes, fused_flop, fused_pts) if fused_calls else \
+        (tot["t"], tot["bytes"], tot["flop"], tot["points"])
     if res == "hbm":
-        achieved, peak, unit, bound = tot["bytes"] / tot["t"] / 1e9, peaks["hbm"] / 1e9, "GB/s", "hbm"
+        achieved, peak, unit, bound = kb / kt / 1e9, peaks["hbm"] / 1e9, "GB/s", "hbm"
         pk_note = f"HBM copy bandwidth ({peaks['hbm_source']}, MEASURED_PEAKS.json)"
     elif res == "sfu":
-        achieved, peak, unit, bound = tot["points"] / tot["t"] / 1e9, peaks["ex2"] / 1e9, "Gexp2/s", "alu"
+        achieved, peak, unit, bound = kp / kt / 1e9, peaks["ex2"] / 1e9, "Gexp2/s", "alu"
         pk_note = "SFU exp2 results/s, measured on this device (gaus_measure_peak)"
     else:
-        achieved, peak, unit, bound = tot["flop"] / tot["t"] / 1e12, peaks["fp32"] / 1e12, "TFLOP/s", "alu"
+        achieved, peak, unit, bound = kf / kt / 1e12, peaks["fp32"] / 1e12, "TFLOP/s", "alu"
         pk_note = "FP32 FMA throughput, measured on this device (gaus_measure_peak)"
     iters = nchunk * period
-    kernel = "k_fused" if plan["fused"] else "iteration kernel sequence (k_nodes .. k_update" + \
+    kernel = "k_fused" if fused_calls else "iteration kernel sequence (k_nodes .. k_update" + \
         (", k_reg_fwd, k_reg_bwd)" if storage else ")")
     roof = {"bound": bound, "kernel": kernel, "achieved": achieved, "peak": peak, "unit": unit,
             "frac": achieved / peak, "peak_note": pk_note + " (of measured)",
-            "launches": nchunk * (plan["fused_launches_per_call"] if plan["fused"] else
-                                  period * plan["launches_per_iteration"]),
-            "mean_launch_ms": tot["t"] * 1e3 / nchunk if plan["fused"] else None,
+            "calls": {"fused": fused_calls, "multi_kernel": nchunk - fused_calls},
+            "launches": fused_calls * plan["fused_launches_per_call"] if fused_calls else
+            nchunk * period * plan["launches_per_iteration"],
+            "mean_launch_ms": fused_t * 1e3 / fused_calls if fused_calls else None,
             "cost_model": "20 flop and 1 exp2 per window point, 8 flop per edge-bin and per storage "
                           "point-edge; 48 V B + (2E + 6V) 4 state bytes per iteration",
             "per_iteration": {"points": tot["points"] / iters, "edge_bins": tot["edge_bins"] / iters,
@@ -485,14 +508,18 @@ def other_workload(torch, g, name, peaks, flush):
     dmu0, dsg0 = torch.from_numpy(mu0).cuda(), torch.from_numpy(sg0).cuda()
     S.step(dmu0, dsg0)
     torch.cuda.synchronize()
+    c0 = path_counts(ctx)
     ms = timed_steps(torch, S, dmu0, dsg0, 1, flush)[0]
+    c1 = path_counts(ctx)
     rep = ctx.verify(S.sched)
     ok = int(sum(1 for r in rep if r["feasible"] and r["res_ok"]))
     roof, it_roof = iteration_roofline(torch, ctx, S, p, B, hp, dmu0, dsg0, peaks, plan)
     ctx.close()
     return {"config": describe(name, p, B, p.iters, period), "value": p.iters * B / (ms / 1e3), "unit": UNIT,
-            "ms_per_step": ms, "path": "fused" if plan["fused"] else "multi-kernel",
-            "gpu_launches_per_step": launches_per_step(plan, p.iters, period),
+            "ms_per_step": ms,
+            "calls": {"fused": c1[0] - c0[0], "multi_kernel": p.iters // period - (c1[0] - c0[0])},
+            "gpu_launches_per_step": launches_per_step(plan, p.iters, period, c1[0] - c0[0], c1[1] - c0[1],
+                                                       c1[2] - c0[2]),
             "roofline": {k: roof[k] for k in ("bound", "kernel", "achieved", "peak", "unit", "frac")},
             "iteration_roofline": {k: it_roof[k] for k in ("t_star_ms", "t_ms", "frac", "us_per_iteration",
                                                            "us_per_iteration_last_call", "binding_iterations")},
@@ -674,8 +701,14 @@ def gpu_arm(args):
         sampler.start()
         time.sleep(0.5)
     wall0 = time.perf_counter()
+    c0 = path_counts(ctx)
     step_ms = timed_steps(torch, S, dmu0, dsg0, args.steps, flush, args.profile_range)
+    c1 = path_counts(ctx)
     wall = time.perf_counter() - wall0
+    # our kernels in the timed region: each call's path as the library counted it
+    df, dm, dc = (b - a for a, b in zip(c0, c1))
+    launches = (df * plan["fused_launches_per_call"] + dm * plan["launches_per_iteration"] + dc
+                + args.steps * (iters // period) * 3)
     clocks = sampler.stop() if sampler else None
     ms = sum(step_ms)
     if world > 1:
@@ -771,7 +804,8 @@ def gpu_arm(args):
                 "data": f"synthetic (seeded {p.name} DAG and initial means)",
                 "config": dict(describe(name, p, B, iters, period), l2="flushed between steps (256 MB write)",
                                parallelism=f"restarts sharded, {world} replica(s)"),
-                "e2e": e2e, "gpu_launches": args.steps * launches_per_step(plan, iters, period),
+                "e2e": e2e, "gpu_launches": launches,
+                "calls": {"fused": df, "multi_kernel": args.steps * (iters // period) - df},
                 "clocks": clocks, "roofline": roof, "iteration_roofline": it_roof,
                 "plan": plan, "fused_phases_us": phases,
                 "legalize_verify_ms": legalize_verify_ms, "step_ms": step_ms,

@@ -232,19 +232,36 @@ gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_stat
 gaus_status gaus_profile_phases(gaus_ctx *ctx, int32_t n_iters, const gaus_state *st, double *out);
 
 /* The execution plan the context chose for its sizes and current hyperparameters
- * (host only: no CUDA call).  out (host, n entries, n <= 12 written):
- *   [0] 1 when gaus_iterate and gaus_loss_grad run the persistent fused kernel,
- *       0 for the multi-kernel path (storage term, continuous dependency penalty,
- *       D > 32767, or a device that cannot hold one block per restart group);
- *   [1] fused: cooperative kernel launches per gaus_iterate call (1 unless B
+ * (host only: no CUDA call).  out (host, n entries, at most 16 written):
+ *   [0] 1 when the persistent fused kernel applies to the current terms and sizes,
+ *       0 when only the multi-kernel path does (storage term, continuous dependency
+ *       penalty, D > 32767, or a device that cannot hold one block per restart group);
+ *   [1] fused: cooperative kernel launches per fused gaus_iterate call (1 unless B
  *       exceeds the restart groups the device holds at once), else 0;
- *   [2] multi-kernel path: kernel launches per iteration, else 0;
+ *   [2] multi-kernel path: kernel launches per iteration;
  *   [3] restart groups; [4] blocks per restart group; [5] restarts per group;
  *   [6] points per CDF table row; [7] dynamic shared memory per fused block (bytes);
  *   [8] streaming multiprocessors of the device; [9] node segments of the fused
- *   kernel; [10] edge chunks of the fused kernel; [11] threads per fused block.
+ *   kernel; [10] edge chunks of the fused kernel; [11] threads per fused block;
+ *   [12] the path mode (gaus_set_path); since the context was created: [13]
+ *   gaus_iterate calls run by the fused kernel, [14] iterations run by the
+ *   multi-kernel path, [15] path-choice reductions launched (one kernel each).
  * EINVAL for a NULL context or out, or n < 1. */
 gaus_status gaus_plan_info(const gaus_ctx *ctx, int64_t *out, int32_t n);
+
+/* Which path gaus_iterate runs (gaus_set_path).  AUTO, the default, chooses per call
+ * from the state's windows (window points of every (node, restart) under the
+ * family's window, summed and maximised by one small reduction whose 16 bytes are
+ * read back, so an AUTO call synchronises the context's stream once; a call made
+ * while the stream is being captured takes the fused path): the persistent fused
+ * kernel when the mean window is under one point, or when the longest window is at
+ * most 32 points and at most twice the mean; the multi-kernel path otherwise.  FUSED
+ * and MULTI force a path (FUSED falls back to the multi-kernel path where the fused
+ * kernel does not apply).  gaus_loss_grad uses the fused kernel unless MULTI is set. */
+#define GAUS_PATH_AUTO 0
+#define GAUS_PATH_FUSED 1
+#define GAUS_PATH_MULTI 2
+gaus_status gaus_set_path(gaus_ctx *ctx, int32_t mode);
 
 /* Exercises the fused kernel's bounded barrier waits (a check of the failure path,
  * not part of the method): one iteration of gaus_iterate whose group barriers can

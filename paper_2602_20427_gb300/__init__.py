@@ -19,7 +19,8 @@ from .build import build
 
 __all__ = ["build", "lib", "Gaus", "default_hparams", "symbols_declared",
            "DEP", "COM", "RES_OBJ", "RES_VIOL", "REG_OBJ", "REC", "DEP_CF", "K", "NT", "STATUS",
-           "GAUSSIAN", "LOGISTIC", "LAPLACE", "CAUCHY", "PEAK_FP32", "PEAK_EX2", "measure_peak"]
+           "GAUSSIAN", "LOGISTIC", "LAPLACE", "CAUCHY", "PEAK_FP32", "PEAK_EX2", "measure_peak",
+           "PATH_AUTO", "PATH_FUSED", "PATH_MULTI"]
 
 DEP, COM, RES_OBJ, RES_VIOL, REG_OBJ, REC = 1, 2, 4, 8, 16, 32
 DEP_CF = 64  # continuous dependency penalty: a variant, not the paper's Eq. dep
@@ -104,6 +105,7 @@ def lib():
 
 
 PEAK_FP32, PEAK_EX2 = 0, 1
+PATH_AUTO, PATH_FUSED, PATH_MULTI = 0, 1, 2
 
 
 def measure_peak(what: int, stream=None) -> float:
@@ -203,7 +205,12 @@ class Gaus:
 
     PLAN_KEYS = ("fused", "fused_launches_per_call", "launches_per_iteration", "restart_groups",
                  "blocks_per_group", "restarts_per_group", "table_row_points", "fused_smem_bytes", "sms",
-                 "node_segments", "edge_chunks", "fused_threads")
+                 "node_segments", "edge_chunks", "fused_threads", "path_mode", "fused_calls", "multi_iterations",
+                 "path_choices")
+
+    def set_path(self, mode):
+        """gaus_set_path: PATH_AUTO (choose per call), PATH_FUSED or PATH_MULTI."""
+        self._check(lib().gaus_set_path(self._ctx, C.c_int32(mode)))
 
     def plan_info(self):
         """The execution plan for the current sizes and hyperparameters (gaus_plan_info)."""

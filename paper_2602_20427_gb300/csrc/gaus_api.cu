@@ -197,6 +197,30 @@ bool fused_ok(const gaus_ctx *ctx) {
   return ctx->fK > 0 && !(ctx->hp.terms & (GAUS_REG_OBJ | GAUS_DEP_CF));
 }
 
+// Window points of every (node, restart) of the state: their sum and maximum, for
+// the per-call choice between the fused kernel and the multi-kernel path.
+__global__ void __launch_bounds__(256) k_window_stats(const float *mu, const float *sg, size_t n, float k, int D,
+                                                      unsigned long long *out) {
+  unsigned long long sum = 0;
+  unsigned mx = 0;
+  for (size_t i = (size_t)blockIdx.x * 256 + threadIdx.x; i < n; i += (size_t)gridDim.x * 256) {
+    const float m = mu[i], s = sg[i];
+    int a = 0, b = -1;
+    if (usable(m, s)) window(m, s, k, D, a, b);
+    const unsigned w = (unsigned)max(b - a + 1, 0);
+    sum += w;
+    mx = max(mx, w);
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    sum += __shfl_down_sync(0xffffffffu, sum, o);
+    mx = max(mx, __shfl_down_sync(0xffffffffu, mx, o));
+  }
+  if ((threadIdx.x & 31) == 0) {
+    atomicAdd(out, sum);
+    atomicMax(out + 1, (unsigned long long)mx);
+  }
+}
+
 // Enqueue n_iters fused iterations (adam) or one loss + gradient evaluation
 // (!adam) as cooperative launches of the persistent kernel, one per batch of
 // restart groups the device holds at once (a single launch unless B is huge).
@@ -503,6 +527,8 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
   TRY(scratch(ctx, &ctx->d_status_tmp, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_loss_tmp, (size_t)P.B));
   TRY(scratch(ctx, &ctx->d_terms_tmp, (size_t)P.B * GAUS_NT));
+  TRY(scratch(ctx, &ctx->d_wsel, 2));
+  CK(cudaMallocHost((void **)&ctx->h_wsel, 2 * sizeof(unsigned long long)), "cudaMallocHost");
   // fused persistent kernel
   TRY(plan_fused(ctx, nsm));
   if (ctx->fK > 0) {
@@ -762,12 +788,23 @@ gaus_status gaus_plan_info(const gaus_ctx *ctx, int64_t *out, int32_t n) {
   const bool fused = fused_ok(ctx);
   const unsigned on = ctx->hp.terms;
   const int64_t per_iter = 5 + ((on & GAUS_DEP_CF) ? 1 : 0) + ((on & GAUS_REG_OBJ) ? 3 : 0);
-  const int64_t v[12] = {fused ? 1 : 0,
+  const int64_t v[16] = {fused ? 1 : 0,
                          fused ? (ctx->fG + ctx->fGl - 1) / std::max(1, ctx->fGl) : 0,
-                         fused ? 0 : per_iter,
+                         per_iter,
                          ctx->fG, ctx->fK, ctx->fRG, ctx->fW, (int64_t)ctx->smem_fused, ctx->nsm,
-                         P.nfseg, P.nchunk, kFusedThreads};
-  for (int i = 0; i < std::min(n, 12); ++i) out[i] = v[i];
+                         P.nfseg, P.nchunk, kFusedThreads, ctx->path_mode, ctx->n_fused_calls,
+                         ctx->n_multi_iters, ctx->n_path_stats};
+  for (int i = 0; i < std::min(n, 16); ++i) out[i] = v[i];
+  return GAUS_OK;
+}
+
+gaus_status gaus_set_path(gaus_ctx *ctx, int32_t mode) {
+  if (!ctx) return GAUS_EINVAL;
+  if (mode < GAUS_PATH_AUTO || mode > GAUS_PATH_MULTI) {
+    ctx->err = "gaus_set_path: mode must be GAUS_PATH_AUTO, GAUS_PATH_FUSED or GAUS_PATH_MULTI";
+    return GAUS_EINVAL;
+  }
+  ctx->path_mode = mode;
   return GAUS_OK;
 }
 
@@ -787,7 +824,7 @@ gaus_status gaus_loss_grad(gaus_ctx *ctx, const float *mu, const float *sigma, c
     ctx->err = "gaus_loss_grad: NULL pointer";
     return GAUS_EINVAL;
   }
-  if (fused_ok(ctx))
+  if (fused_ok(ctx) && ctx->path_mode != GAUS_PATH_MULTI)
     return enqueue_fused(ctx, ctx->stream, 1, false, mu, sigma, nullptr, nullptr, nullptr, nullptr,
                          const_cast<float *>(lambda), nullptr, grad_mu, grad_sigma, loss, terms,
                          status ? status : ctx->d_status_tmp, nullptr);
@@ -815,6 +852,37 @@ gaus_status gaus_adam_step(gaus_ctx *ctx, float *mu, float *sigma, const float *
   return GAUS_OK;
 }
 
+// The path of one gaus_iterate call (gaus_set_path).  The fused kernel wins where the
+// windows are short (under a point on average: its one launch per call and node-side
+// edges beat the five kernels per iteration) or uniform and within its 32-point
+// staging (as at a uniform initial sigma); the multi-kernel path wins where windows
+// vary across restarts or exceed the staging (the fused kernel's long items go one
+// warp at a time): measured on the logic-network workload along a 2,000-iteration
+// normal-family run and the logistic and kappa-initialized regimes.
+static gaus_status choose_path(gaus_ctx *ctx, const float *mu, const float *sg, bool *fused) {
+  *fused = false;
+  if (!fused_ok(ctx) || ctx->path_mode == GAUS_PATH_MULTI) return GAUS_OK;
+  *fused = true;
+  if (ctx->path_mode == GAUS_PATH_FUSED) return GAUS_OK;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  CK(cudaStreamIsCapturing(ctx->stream, &cs), "cudaStreamIsCapturing");
+  if (cs != cudaStreamCaptureStatusNone) return GAUS_OK;
+  const Plan &P = ctx->plan;
+  const size_t n = (size_t)P.V * P.B;
+  CK(cudaMemsetAsync(ctx->d_wsel, 0, 2 * sizeof(unsigned long long), ctx->stream), "path memset");
+  const int blocks = (int)std::min<size_t>((n + 255) / 256, (size_t)2 * std::max(1, ctx->nsm));
+  k_window_stats<<<blocks, 256, 0, ctx->stream>>>(mu, sg, n, ctx->k_win, P.D, ctx->d_wsel);
+  CK(cudaGetLastError(), "k_window_stats launch");
+  CK(cudaMemcpyAsync(ctx->h_wsel, ctx->d_wsel, 2 * sizeof(unsigned long long), cudaMemcpyDeviceToHost, ctx->stream),
+     "path copy");
+  CK(cudaStreamSynchronize(ctx->stream), "path sync");
+  ++ctx->n_path_stats;
+  const double mean = (double)ctx->h_wsel[0] / (double)n;
+  const double mx = (double)ctx->h_wsel[1];
+  *fused = mean < 1.0 || (mx <= (double)kStage && mx <= 2.0 * mean);
+  return GAUS_OK;
+}
+
 gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *S) {
   if (!ctx) return GAUS_EINVAL;
   if (!S || n_iters < 0 || !S->mu || !S->sigma || !S->m_mu || !S->v_mu || !S->m_sigma || !S->v_sigma ||
@@ -823,9 +891,14 @@ gaus_status gaus_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_state *S) {
     return GAUS_EINVAL;
   }
   if (n_iters == 0) return GAUS_OK;
-  if (fused_ok(ctx))
+  bool fused = false;
+  TRY(choose_path(ctx, S->mu, S->sigma, &fused));
+  if (fused) {
+    ++ctx->n_fused_calls;
     return enqueue_fused(ctx, ctx->stream, n_iters, true, S->mu, S->sigma, S->m_mu, S->v_mu, S->m_sigma, S->v_sigma,
                          S->lambda, S->step, nullptr, nullptr, S->loss, S->terms, S->status, nullptr);
+  }
+  ctx->n_multi_iters += n_iters;
   // two captured graphs of the same iteration: kGraphUnroll iterations, and one
   const uint64_t h = state_hash(S);
   if (!ctx->gexec || ctx->ghash != h) {
@@ -847,7 +920,9 @@ gaus_status gaus_profile_iterate(gaus_ctx *ctx, int32_t n_iters, const gaus_stat
     ctx->err = "gaus_profile_iterate: NULL pointer or n_iters < 0";
     return GAUS_EINVAL;
   }
-  if (fused_ok(ctx)) {
+  bool fused = false;
+  TRY(choose_path(ctx, S->mu, S->sigma, &fused));
+  if (fused) {
     double ph[12];
     TRY(fused_phases(ctx, n_iters, S, ph));
     // iteration start to the first barrier's release, to the second's, to the next start
@@ -1024,6 +1099,7 @@ void gaus_destroy(gaus_ctx *ctx) {
   if (ctx->side) cudaStreamSynchronize(ctx->side);
   for (void *p : ctx->allocs) cudaFree(p);
   if (ctx->d_prof) cudaFree(ctx->d_prof);
+  if (ctx->h_wsel) cudaFreeHost(ctx->h_wsel);
   if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
   if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
   if (ctx->side) cudaStreamDestroy(ctx->side);

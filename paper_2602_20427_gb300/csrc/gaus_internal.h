@@ -172,6 +172,10 @@ struct gaus_ctx {
   // per cooperative launch, dynamic shared memory; 0 = the terms or sizes need the
   // multi-kernel path (storage term, continuous dependency penalty, D > 32767)
   int fK = 0, fGl = 0;
+  int path_mode = 0;             // GAUS_PATH_AUTO, GAUS_PATH_FUSED or GAUS_PATH_MULTI (gaus_set_path)
+  long long n_fused_calls = 0, n_multi_iters = 0, n_path_stats = 0;  // what gaus_iterate ran so far
+  unsigned long long *d_wsel = nullptr;  // window points sum and maximum of the path choice
+  unsigned long long *h_wsel = nullptr;  // its pinned host copy
   int nsm = 0;                   // streaming multiprocessors of the device
   int fRG = 1, fRBp = 1, fRB1 = 1, fG = 1;
   int fW = 0;  // table row length of the fused path ([node][point][restart] layout)  // restarts per group, lanes per row (phases 2-3, phase 1), groups

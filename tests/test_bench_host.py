@@ -87,3 +87,7 @@ def test_launch_count_per_step():
     # iteration, plus legalize and the verifier's two passes per call
     assert bench.launches_per_step(fused, 2000, 100) == 20 * (1 + 3)
     assert bench.launches_per_step(multi, 2000, 100) == 20 * (800 + 3)
+    # the path chosen per call: 6 calls on the multi-kernel path (5 kernels per
+    # iteration), 14 fused calls, 20 window reductions of the choice
+    both = {"fused": 1, "fused_launches_per_call": 1, "launches_per_iteration": 5}
+    assert bench.launches_per_step(both, 2000, 100, 14, 600, 20) == 14 + 600 * 5 + 20 + 20 * 3

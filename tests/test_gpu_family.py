@@ -156,15 +156,17 @@ def test_set_hparams_switches_the_family(g):
     ctx.close()
 
 
+@pytest.mark.parametrize("path", ["fused", "multi"])
 @pytest.mark.parametrize("fam", FAMS)
-def test_iterate_tracks_oracle_trajectory(g, fam):
-    # the fused iteration (loss, gradient, multipliers, Adam) against the oracle's
-    # loss per step on the tiny workload, gated as for the normal
+def test_iterate_tracks_oracle_trajectory(g, fam, path):
+    # the iteration (loss, gradient, multipliers, Adam) on either path against the
+    # oracle's loss per step on the tiny workload, gated as for the normal
     p = W.tiny_layered(1)
     B = 2
     mu, sg = W.init_state(p, B, 1, mu_jitter="uniform01", sigma0=1.0)
     hp = g.default_hparams(terms=p.terms, lr=0.05, family=fam)
     ctx = g.Gaus(p, B, hp)
+    ctx.set_path(g.PATH_FUSED if path == "fused" else g.PATH_MULTI)
     st = ctx.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), 1e-6)
     op = oracle.OracleProblem(p)
     ohp = oracle.hparams(tau=hp.tau, rho=hp.rho, alpha=hp.alpha, w_res=hp.w_res, w_mem=hp.w_mem,

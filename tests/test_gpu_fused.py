@@ -27,7 +27,9 @@ def g():
 def test_plan_info_by_term_set(g):
     p = W.logic_network(3, V=1500, depth=30)
     B = 64
-    for terms, fused, per_iter in ((W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL, 1, 0),
+    # launches per iteration of the multi-kernel path: node, edge, reduce, finalize,
+    # update, and the storage pass's three or the continuous penalty's one
+    for terms, fused, per_iter in ((W.DEP | W.COM | W.RES_OBJ | W.RES_VIOL, 1, 5),
                                    (W.DEP | W.RES_VIOL | W.REG_OBJ, 0, 8),
                                    (W.DEP_CF | W.COM | W.RES_OBJ, 0, 6)):
         ctx = g.Gaus(p, B, g.default_hparams(terms=terms))
@@ -114,3 +116,46 @@ def test_barrier_wait_runs_out_and_reports(g):
         reg.check_barrier_timeout(reg.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda()), 2_000_000)
     reg.close()
     ctx.close()
+
+
+def test_auto_path_choice(g):
+    # GAUS_PATH_AUTO per call: the fused kernel for uniform windows within its staging
+    # (sigma = 1.5: about 18 points everywhere) and for windows under a point on
+    # average (sigma = 0.1); the multi-kernel path for windows that vary across
+    # restarts (sigma from 0.2 to 3) and for windows beyond the staging (logistic,
+    # about 34 points at sigma = 1.5); the forced modes whatever the windows
+    p = W.logic_network(4, V=2000, depth=40)
+    B = 64
+    rng = np.random.default_rng(5)
+    mu, _ = W.init_state(p, B, 5)
+    cases = (("uniform", g.GAUSSIAN, np.full((p.V, B), 1.5, np.float32), "fused"),
+             ("short", g.GAUSSIAN, np.full((p.V, B), 0.1, np.float32), "fused"),
+             ("varied", g.GAUSSIAN, rng.uniform(0.2, 3.0, size=(p.V, B)).astype(np.float32), "multi"),
+             ("wide tails", g.LOGISTIC, np.full((p.V, B), 1.5, np.float32), "multi"))
+    for name, fam, sg, want in cases:
+        ctx = g.Gaus(p, B, g.default_hparams(terms=p.terms, family=fam))
+        st = ctx.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), 1e-6)
+        i0 = ctx.plan_info()
+        ctx.iterate(3, st)
+        torch.cuda.synchronize()
+        i1 = ctx.plan_info()
+        got = "fused" if i1["fused_calls"] - i0["fused_calls"] == 1 else "multi"
+        assert got == want, (name, i0, i1)
+        assert i1["path_choices"] - i0["path_choices"] == 1
+        assert i1["multi_iterations"] - i0["multi_iterations"] == (3 if want == "multi" else 0)
+        for mode, forced in ((g.PATH_FUSED, "fused"), (g.PATH_MULTI, "multi")):
+            ctx.set_path(mode)
+            j0 = ctx.plan_info()
+            ctx.iterate(2, st)
+            j1 = ctx.plan_info()
+            assert j1["path_mode"] == mode and j1["path_choices"] == j0["path_choices"]
+            assert (j1["fused_calls"] - j0["fused_calls"]) == (1 if forced == "fused" else 0), (name, mode)
+        torch.cuda.synchronize()
+        assert np.all(st["status"].cpu().numpy() == 0)
+        ctx.close()
+    with pytest.raises(g.GausError):
+        c = g.Gaus(p, B, g.default_hparams(terms=p.terms))
+        try:
+            c.set_path(3)
+        finally:
+            c.close()

@@ -178,8 +178,9 @@ def test_iterate_equals_separate_calls(g):
     ctx.close()
 
 
-def test_iterate_multiplier_update(g):
-    # the fused iteration's multiplier update (Sec. 3.3): after every iteration,
+@pytest.mark.parametrize("path", ["fused", "multi"])
+def test_iterate_multiplier_update(g, path):
+    # the iteration's multiplier update (Sec. 3.3), on either path: after every iteration,
     # lambda_k = lambda_k(before) + rho V_k for the active constraints, with V_k the
     # values the iteration reports (exactly, up to the final rounding to float) and
     # against the oracle's V_k at the same state (within the parity tolerance)
@@ -189,6 +190,7 @@ def test_iterate_multiplier_update(g):
     mu, sg = W.init_state(p, B, 3)
     hp = g.default_hparams(terms=p.terms, rho=1e-2)
     ctx = g.Gaus(p, B, hp)
+    ctx.set_path(g.PATH_FUSED if path == "fused" else g.PATH_MULTI)
     st = ctx.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), 1e-3)
     op = oracle.OracleProblem(p)
     ohp = oracle.hparams(tau=hp.tau, rho=hp.rho, alpha=hp.alpha, w_res=hp.w_res, w_mem=hp.w_mem, terms=p.terms)
@@ -213,15 +215,17 @@ def test_iterate_multiplier_update(g):
     ctx.close()
 
 
-def test_iterate_tracks_oracle_trajectory(g):
-    # a short trajectory of the tiny workload against the oracle (reported
-    # quantity: the loss per step; gated loosely because first-step Adam is
+@pytest.mark.parametrize("path", ["fused", "multi"])
+def test_iterate_tracks_oracle_trajectory(g, path):
+    # a short trajectory of the tiny workload against the oracle, on either path
+    # (reported quantity: the loss per step; gated loosely because first-step Adam is
     # sign-like and can flip noise-level components)
     p = W.tiny_layered(1)
     B = 2
     mu, sg = W.init_state(p, B, 1, mu_jitter="uniform01", sigma0=1.0)
     hp = g.default_hparams(terms=p.terms, lr=0.05)
     ctx = g.Gaus(p, B, hp)
+    ctx.set_path(g.PATH_FUSED if path == "fused" else g.PATH_MULTI)
     st = ctx.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), 1e-6)
     op = oracle.OracleProblem(p)
     ohp = oracle.hparams(tau=hp.tau, rho=hp.rho, alpha=hp.alpha, w_res=hp.w_res, w_mem=hp.w_mem, terms=p.terms)
