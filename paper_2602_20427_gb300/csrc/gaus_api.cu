@@ -367,10 +367,12 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     ctx->err = "no CUDA device";
     return GAUS_ECUDA;
   }
-  // restarts per warp row: up to kMaxRB, fewer for long horizons so that the node
+  // restarts per warp row: up to kMaxRB (8 with the storage term, whose workloads
+  // measured faster with shorter rows), fewer for long horizons so that the node
   // pass's usage histogram (two u32 halves per bin and restart) fits shared memory
+  const int max_rb = (ctx->hp.terms & GAUS_REG_OBJ) ? kMaxRB / 2 : kMaxRB;
   ctx->RB = 1;
-  while (ctx->RB < P.B && ctx->RB < kMaxRB) ctx->RB <<= 1;
+  while (ctx->RB < P.B && ctx->RB < max_rb) ctx->RB <<= 1;
   while (ctx->RB > 1 && 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned) > kMaxSmem - 1024) ctx->RB >>= 1;
   ctx->G = (P.B + ctx->RB - 1) / ctx->RB;
   ctx->smem_nodes = 2 * (size_t)ctx->RB * P.Dh * sizeof(unsigned);
@@ -422,9 +424,11 @@ gaus_status build_ctx(gaus_ctx *ctx, const gaus_problem *prob) {
     const size_t wf = std::min<size_t>(std::min<size_t>(kTableMaxFused, (size_t)P.D + 2), kTableBytesFused / per_pt);
     ctx->fW = (int)std::max<size_t>(4, wf);
   }
-  // storage-term kernels: their own restarts-per-row so that the storage histogram
-  // (two u32 halves), its difference array and constants fit in shared memory
-  ctx->RBr = ctx->RB;
+  // storage-term kernels: their own restarts-per-row, at most 4 (a row's loops over
+  // successors and points run to the longest among its restarts; measured on the
+  // loop-body and wide workloads), fewer where the storage histogram (two u32
+  // halves), its difference array and constants would not fit in shared memory
+  ctx->RBr = std::min(ctx->RB, 4);
   auto rfwd_bytes = [&](int rb) {
     return (2 * (size_t)P.Dh * rb + (size_t)(P.Dh + 1) * rb + rb) * sizeof(unsigned);
   };
