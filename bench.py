@@ -645,6 +645,7 @@ def cdf_families(torch, g, p, B, dmu0, dsg0, n_f=100):
         sf = cf.new_state(dmu0, dsg0, hpf.lambda0)
         cf.iterate(10, sf)
         sf = cf.new_state(dmu0, dsg0, hpf.lambda0)
+        f0 = path_counts(cf)[0]
         ev = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
         torch.cuda.synchronize()
         ev[0].record()
@@ -652,8 +653,9 @@ def cdf_families(torch, g, p, B, dmu0, dsg0, n_f=100):
         ev[1].record()
         torch.cuda.synchronize()
         fms = ev[0].elapsed_time(ev[1])
-        families.append({"family": name, "iterations": n_f, "path": "fused" if cf.plan_info()["fused"]
-                         else "multi-kernel", "restart_iterations_per_s": n_f * B / (fms / 1e3),
+        families.append({"family": name, "iterations": n_f,
+                         "path": "fused" if path_counts(cf)[0] > f0 else "multi-kernel",
+                         "restart_iterations_per_s": n_f * B / (fms / 1e3),
                          "ms_per_iteration": fms / n_f, "mean_loss_after": float(sf["loss"].mean().item())})
         cf.close()
     return families
@@ -844,6 +846,7 @@ def fused_probe(args):
     g.build()
     p, B, mu0, sg0 = workload(0, None, args.workload)
     ctx = g.Gaus(p, B, g.default_hparams(terms=p.terms, lr=p.lr))
+    ctx.set_path(g.PATH_FUSED)   # the probe is of the fused kernel, whatever the windows
     st = ctx.new_state(torch.from_numpy(mu0).cuda(), torch.from_numpy(sg0).cuda())
     if args.fused_probe > 0:
         ctx.iterate(args.fused_probe, st)
