@@ -137,7 +137,7 @@ gaus_status enqueue_iteration(gaus_ctx *ctx, cudaStream_t st, const float *mu, c
     RA.k_win = ctx->k_win; RA.perm = ctx->d_perm; RA.bits = ctx->d_bits;
     RA.out_ptr = ctx->d_out_ptr; RA.out_dst = ctx->d_out_dst; RA.seg = ctx->d_seg; RA.win = ctx->d_win;
     RA.qtab = ctx->d_qtab + (size_t)2 * kTailRows * ctx->hp.family;
-    RA.tab = ctx->d_tab; RA.W = ctx->W;
+    RA.tab = ctx->d_tab; RA.W = ctx->W; RA.ptab = ctx->d_ptab; RA.WP = ctx->WP;
     RA.rpart = ctx->d_rpart; RA.Hreg = ctx->d_Hreg; RA.gown = ctx->d_gown; RA.eslot = ctx->d_eslot;
     ks.reg_fwd<<<ctx->nblk_r, kFwdThreads, ctx->smem_rfwd, st>>>(RA);
     CK(cudaGetLastError(), "k_reg_fwd launch");
@@ -593,6 +593,9 @@ gaus_status alloc_storage_scratch(gaus_ctx *ctx) {
   TRY(scratch(ctx, &ctx->d_gown, (size_t)P.V * P.B));
   TRY(scratch(ctx, &ctx->d_eslot, (size_t)std::max(1, P.E) * P.B));
   TRY(scratch(ctx, &ctx->d_qtab, (size_t)2 * 4 * kTailRows));
+  // rows of the successors' product for the backward: up to 32 points, 128 MB at most
+  ctx->WP = (int)std::max<size_t>(4, std::min<size_t>(32, ((size_t)128 << 20) / ((size_t)P.V * P.B * sizeof(float))));
+  TRY(scratch(ctx, &ctx->d_ptab, (size_t)P.V * P.B * ctx->WP));
   k_tail_tables<<<(4 * kTailRows + 255) / 256, 256, 0, ctx->stream>>>(ctx->d_qtab);
   CK(cudaGetLastError(), "k_tail_tables launch");
   CK(cudaStreamSynchronize(ctx->stream), "k_tail_tables sync");

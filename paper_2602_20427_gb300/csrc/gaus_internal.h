@@ -149,6 +149,8 @@ struct gaus_ctx {
   long long *d_rpart = nullptr;  // nblk_r * Dh * RBr storage partials
   long long *d_Ureg = nullptr;   // B * Dh expected (folded) storage, 2^32 fixed point
   float4 *d_qtab = nullptr;      // tail tables of the storage forward (k_tail_tables), all families
+  float *d_ptab = nullptr;       // (V, B, WP) successors' products, forward -> backward
+  int WP = 0;
   float *d_Hreg = nullptr;       // B * Dh storage adjoint
   float2 *d_eslot = nullptr;     // E * B successor shares of the storage gradient
   int32_t *d_in_eslot = nullptr; // E

@@ -40,6 +40,8 @@ struct RegArgs {
   const unsigned *win;               // packed windows
   const float *tab;                  // the node pass's CDF table rows (V, B, W) by caller id
   int W;
+  float *ptab;                       // (V, B, WP) by caller id: the successors' product P(d) for
+  int WP;                            // d = max(a, Amax) .. Bm, written by the forward
   const float4 *qtab;                // the family's tail table (kTailRows x 2, k_tail_tables)
   long long *rpart;                  // blocks * Dh * RB
   // backward
@@ -299,6 +301,10 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
     const int n_tail = valid ? max(0, Bm - tail_lo + 1) : 0;
     const int total = n_own + n_tail;
     const int tmax = __reduce_max_sync(FULL, total);
+    // the successors' product over d0 .. Bm for the backward, when the row holds it
+    const int d0 = max(a, Amax);
+    const bool prow = valid && deg > 0 && Bm >= d0 && Bm - d0 + 1 <= A.WP;
+    float *pr = A.ptab + ((size_t)vc * A.B + (b < A.B ? b : 0)) * A.WP;
     for (int k = 0; k < tmax; ++k) {
       const bool on = k < total;
       const bool own = k < n_own;
@@ -306,6 +312,10 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_fwd(const RegArgs A) {
       FF Ci = {1.0f, 0.0f};
       if (on && own) Ci = cdf_pair_ff<kFam>(A.qtab, d, mu, sg, inv_s, a, bw);
       const FF L = one_minus_m_pair<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
+      if (on && prow && d >= d0) {
+        const FF P = ff_one_minus(L);
+        pr[d - d0] = P.h + P.l;
+      }
       if (on && bits != 0.f) hist_add_pair(hlo, hhi, fold_bin(d, A.II) * RB + r, ff_mulf(ff_mul(Ci, L), bits));
     }
     __syncwarp();
@@ -462,6 +472,12 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
     const int dmax = __reduce_max_sync(FULL, deg);
     int Amax, Bm;
     succ_bounds(A, e0, deg, dmax, b, Amax, Bm);
+    // the successors' product P(d), d0 <= d <= Bm, as the forward stored it (else formed
+    // here from the table); below d0 = max(a, Amax) every share and 1 - M's complement
+    // vanish (C_i = 0 below a; some successor certainly not started below Amax)
+    const int d0 = max(a, Amax);
+    const bool prow = valid && deg > 0 && Bm >= d0 && Bm - d0 + 1 <= A.WP;
+    const float *pr = A.ptab + ((size_t)vc * A.B + (b < A.B ? b : 0)) * A.WP;
     // own adjoint on the own window: dL/dC_i(d) = G(d) b_i (1 - M_i(d))
     float Ao = 0.f, Bo = 0.f;
     const int n_own = valid ? bw - a + 1 : 0;
@@ -469,7 +485,8 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
     for (int k = 0; k < nmax; ++k) {
       const bool on = k < n_own;
       const int d = a + k;
-      const float L = one_minus_m_tab<kFam>(A, e0, on ? deg : 0, dmax, b, d, Amax);
+      const float L = (prow && d >= d0) ? 1.0f - pr[d - d0]
+                                        : one_minus_m_tab<kFam>(A, e0, on && !prow ? deg : 0, dmax, b, d, Amax);
       if (on) {
         const float z = ((float)d + 0.5f - mu) * inv_s;
         const float f = reg_pdf<kFam>(z);
@@ -486,7 +503,7 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
       const int jc = eon ? A.out_dst[e0 + q] : 0;
       const unsigned wm = eon ? A.win[(size_t)jc * A.B + b] : 0u;
       const int aj = (int)(wm & 0xFFFFu), bj = (int)(wm >> 16) - 1;
-      const int lo = max(aj, a);  // C_i(d) = 0 below the own window
+      const int lo = max(aj, d0);  // C_i(d) = 0 below the own window, the product 0 below Amax
       const int cnt = eon && bits != 0.f ? max(0, bj - lo + 1) : 0;
       const float mj = cnt ? A.mu[(size_t)jc * A.B + b] : 0.f;
       const float ij = cnt ? 1.0f / A.sg[(size_t)jc * A.B + b] : 1.f;
@@ -496,10 +513,18 @@ __global__ void __launch_bounds__(kFwdThreads) k_reg_bwd(const RegArgs A) {
         const bool on = k < cnt;
         const int d = lo + k;
         const float Ci = on ? reg_cdf_tab<kFam>(A, vc, b, own_w, d) : 1.0f;
-        // product of the other successors' CDFs at d
+        // product of the other successors' CDFs at d: P(d) / C_j(d) (C_j > 0 on j's
+        // window), or formed directly where P is not stored or C_j is below 1e-30
         float prod = 1.f;
-        for (int q2 = 0; q2 < dmax; ++q2) {
-          if (on && q2 < deg && q2 != q) {
+        bool direct = !prow;
+        if (on && prow) {
+          const float cj = reg_cdf_tab<kFam>(A, jc, b, wm, d);
+          if (cj > 1e-30f) prod = pr[d - d0] / cj;
+          else direct = true;
+        }
+        const bool dir_any = __any_sync(FULL, on && direct);
+        for (int q2 = 0; q2 < dmax && dir_any; ++q2) {
+          if (on && direct && q2 < deg && q2 != q) {
             const int kc2 = A.out_dst[e0 + q2];
             prod *= reg_cdf_tab<kFam>(A, kc2, b, A.win[(size_t)kc2 * A.B + b], d);
           }
