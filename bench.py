@@ -89,6 +89,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-families", action="store_true", help="skip the CDF-family timings")
     ap.add_argument("--no-workloads", action="store_true", help="skip the other workloads' timed solves")
+    ap.add_argument("--path", default="auto", choices=["auto", "fused", "multi"],
+                    help="gaus_iterate's path: chosen per call (default), or forced")
     ap.add_argument("--restarts", type=int, default=None,
                     help="restarts per rank (default: the workload's B; others for scaling studies)")
     ap.add_argument("--profile-range", action="store_true",
@@ -682,6 +684,7 @@ def gpu_arm(args):
     assert iters % period == 0, "--iters must be a multiple of --period"
     hp = g.default_hparams(terms=p.terms, lr=p.lr)
     ctx = g.Gaus(p, B, hp)
+    ctx.set_path({"auto": g.PATH_AUTO, "fused": g.PATH_FUSED, "multi": g.PATH_MULTI}[args.path])
     plan = ctx.plan_info()
     dmu0, dsg0 = torch.from_numpy(mu0).cuda(), torch.from_numpy(sg0).cuda()
     S = Solve(torch, ctx, p, B, hp, iters, period)
@@ -805,6 +808,7 @@ def gpu_arm(args):
                 "scaling": "weak", "vs_baseline": None, "dtype": "f32",
                 "data": f"synthetic (seeded {p.name} DAG and initial means)",
                 "config": dict(describe(name, p, B, iters, period), l2="flushed between steps (256 MB write)",
+                               path=args.path,
                                parallelism=f"restarts sharded, {world} replica(s)"),
                 "e2e": e2e, "gpu_launches": launches,
                 "calls": {"fused": df, "multi_kernel": args.steps * (iters // period) - df},

@@ -255,9 +255,13 @@ gaus_status gaus_plan_info(const gaus_ctx *ctx, int64_t *out, int32_t n);
  * read back, so an AUTO call synchronises the context's stream once; a call made
  * while the stream is being captured takes the fused path): the persistent fused
  * kernel when the mean window is under one point, or when the longest window is at
- * most 32 points and at most twice the mean; the multi-kernel path otherwise.  FUSED
+ * most 32 points and at most twice the mean; the multi-kernel path otherwise.  Without
+ * the reduction: problems of fewer than 16,384 (node, restart) items always take the
+ * fused kernel, and restart groups of fewer than 64 restarts (B < 64) the multi-kernel
+ * path.  FUSED
  * and MULTI force a path (FUSED falls back to the multi-kernel path where the fused
- * kernel does not apply).  gaus_loss_grad uses the fused kernel unless MULTI is set. */
+ * kernel does not apply).  gaus_loss_grad uses the fused kernel unless MULTI is set
+ * or AUTO's size rule picks the multi-kernel path. */
 #define GAUS_PATH_AUTO 0
 #define GAUS_PATH_FUSED 1
 #define GAUS_PATH_MULTI 2

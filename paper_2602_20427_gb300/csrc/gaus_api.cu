@@ -831,7 +831,11 @@ gaus_status gaus_loss_grad(gaus_ctx *ctx, const float *mu, const float *sigma, c
     ctx->err = "gaus_loss_grad: NULL pointer";
     return GAUS_EINVAL;
   }
-  if (fused_ok(ctx) && ctx->path_mode != GAUS_PATH_MULTI)
+  // the fused kernel unless MULTI is set, or AUTO's size rule picks the multi-kernel
+  // path (restart groups of fewer than 64 on a problem of 16,384 items or more)
+  const bool small_groups = ctx->path_mode == GAUS_PATH_AUTO && ctx->fRG < 64 &&
+                            (size_t)ctx->plan.V * ctx->plan.B >= 16384;
+  if (fused_ok(ctx) && ctx->path_mode != GAUS_PATH_MULTI && !small_groups)
     return enqueue_fused(ctx, ctx->stream, 1, false, mu, sigma, nullptr, nullptr, nullptr, nullptr,
                          const_cast<float *>(lambda), nullptr, grad_mu, grad_sigma, loss, terms,
                          status ? status : ctx->d_status_tmp, nullptr);
@@ -865,17 +869,28 @@ gaus_status gaus_adam_step(gaus_ctx *ctx, float *mu, float *sigma, const float *
 // staging (as at a uniform initial sigma); the multi-kernel path wins where windows
 // vary across restarts or exceed the staging (the fused kernel's long items go one
 // warp at a time): measured on the logic-network workload along a 2,000-iteration
-// normal-family run and the logistic and kappa-initialized regimes.
+// normal-family run and the logistic and kappa-initialized regimes.  Two cases are
+// decided by the sizes alone, with no reduction: problems of fewer than 16,384
+// (node, restart) items run the fused kernel (they are bound by launch latency, and
+// it is one launch per call), and restart groups of fewer than 64 restarts the
+// multi-kernel path (the fused kernel's phases 2 and 3 take one node per warp, so a
+// smaller group leaves lanes idle, where the multi-kernel path packs two nodes per
+// warp): measured with the logic-network DAG at B = 16 and 32 and the tiny DAG at B = 1.
 static gaus_status choose_path(gaus_ctx *ctx, const float *mu, const float *sg, bool *fused) {
   *fused = false;
   if (!fused_ok(ctx) || ctx->path_mode == GAUS_PATH_MULTI) return GAUS_OK;
   *fused = true;
   if (ctx->path_mode == GAUS_PATH_FUSED) return GAUS_OK;
+  const Plan &P = ctx->plan;
+  const size_t n = (size_t)P.V * P.B;
+  if (n < 16384) return GAUS_OK;
+  if (ctx->fRG < 64) {
+    *fused = false;
+    return GAUS_OK;
+  }
   cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
   CK(cudaStreamIsCapturing(ctx->stream, &cs), "cudaStreamIsCapturing");
   if (cs != cudaStreamCaptureStatusNone) return GAUS_OK;
-  const Plan &P = ctx->plan;
-  const size_t n = (size_t)P.V * P.B;
   CK(cudaMemsetAsync(ctx->d_wsel, 0, 2 * sizeof(unsigned long long), ctx->stream), "path memset");
   const int blocks = (int)std::min<size_t>((n + 255) / 256, (size_t)2 * std::max(1, ctx->nsm));
   k_window_stats<<<blocks, 256, 0, ctx->stream>>>(mu, sg, n, ctx->k_win, P.D, ctx->d_wsel);

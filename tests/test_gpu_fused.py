@@ -153,6 +153,18 @@ def test_auto_path_choice(g):
         torch.cuda.synchronize()
         assert np.all(st["status"].cpu().numpy() == 0)
         ctx.close()
+    # decided by the sizes, with no reduction: a tiny problem (64 nodes, one restart)
+    # runs the fused kernel, restart groups of 16 the multi-kernel path
+    for pp, BB, want in ((W.tiny_layered(1), 1, "fused"), (p, 16, "multi")):
+        mu_s, sg_s = W.init_state(pp, BB, 7)
+        c = g.Gaus(pp, BB, g.default_hparams(terms=pp.terms))
+        st = c.new_state(torch.from_numpy(mu_s).cuda(), torch.from_numpy(sg_s).cuda(), 1e-6)
+        c.iterate(2, st)
+        torch.cuda.synchronize()
+        i1 = c.plan_info()
+        assert i1["path_choices"] == 0
+        assert (i1["fused_calls"], i1["multi_iterations"]) == ((1, 0) if want == "fused" else (0, 2)), (BB, i1)
+        c.close()
     with pytest.raises(g.GausError):
         c = g.Gaus(p, B, g.default_hparams(terms=p.terms))
         try:

@@ -154,13 +154,15 @@ def test_adam_step_matches_oracle(g):
     ctx.close()
 
 
-def test_iterate_equals_separate_calls(g):
-    # the captured fused iteration computes the same as loss_grad + adam_step
+@pytest.mark.parametrize("path", ["fused", "multi"])
+def test_iterate_equals_separate_calls(g, path):
+    # the iteration computes the same as loss_grad + adam_step, on either path
     p = W.random_layered(2)
     B = 32
     mu, sg = W.init_state(p, B, 2)
     hp = g.default_hparams(terms=p.terms)
     ctx = g.Gaus(p, B, hp)
+    ctx.set_path(g.PATH_FUSED if path == "fused" else g.PATH_MULTI)
     st = ctx.new_state(torch.from_numpy(mu).cuda(), torch.from_numpy(sg).cuda(), 1e-6)
     m = {k: torch.from_numpy(v).cuda() for k, v in (("mu", mu), ("sg", sg))}
     z = [torch.zeros((p.V, B), device="cuda") for _ in range(4)]
